@@ -1,0 +1,520 @@
+"""CPU oracle for the Hadamard-domain INT8 convolution (HaTQ). TEST
+INFRASTRUCTURE ONLY: tests, the smoke check and the benchmark's CPU-baseline
+leg may import it; the CUDA path never does, and nothing here is shared with
+it (the two are written independently and meet only on the seeded inputs).
+
+Plain, slow and literal: dense Sylvester matrices, matrix-form transforms,
+scalar quantizers, a nested-loop direct convolution (conv_ref.c), fp64 for
+real arithmetic and int64 (or Python integers) for integer arithmetic.
+
+Section/equation names refer to the HaTQ paper ("Hadamard-Domain Model
+Quantization for Learned Image Coding") and its supplementary material.
+
+Readings the paper leaves open (the same list is kept with the design notes):
+  R1 transform order: a block-diagonal Sylvester transform I_{C/hb} (x) H_hb
+     along the channel axis (orthogonal, so the DH/WH identities hold), not the
+     single Paley/Kronecker order m(C) of Eq. (hadamard_order).
+  R2 round(.) is round-half-to-even everywhere (rint for reals; for a shift
+     by 2^n the exact rational v / 2^n rounded half to even).
+  R3 the multiplier/shift pair (M, n) of Eq. (integer_fixed_point_scale):
+     the largest shared n in [0, 62] such that every M_c = rint(rho_c 2^n) is
+     below 2^31 and max_c(M_c A_c) * g_out * g_next < 2^62, with A_c the
+     worst-case |accumulator| of channel c and g the gains (block sizes) of the
+     unnormalized transforms; fewer than 16 bits in max_c M_c is an error.
+  R4 symmetric INT8 range [-127, 127]; a zero range gives scale 1.
+  R5 bias enters the int32 accumulator before M (.) and before H_out.
+  R6 fixed summation order for real-valued transforms: for output j,
+     acc = 0; acc += H[i][j] * x_i for i = 0..hb-1; then acc / sqrt(hb).
+
+parity unpinned: the rounding convention R2 and the (M, n) rule R3 are
+conventions of this implementation (the paper fixes neither); the oracle pins
+them against exact rational arithmetic, not against the paper.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+import subprocess
+from fractions import Fraction
+
+import numpy as np
+
+QMAX = 127                      # q_max^s = 2^(b-1) - 1 for b = 8, Eq. (symmetric_q)
+
+# --------------------------------------------------------------------------
+# Hadamard matrices: Eq. (supp_sylvester), Eq. (hadamard_properties)
+# --------------------------------------------------------------------------
+
+
+def sylvester(m: int) -> np.ndarray:
+    """Unnormalized Sylvester Hadamard matrix H~_m by the recursion
+    H~_1 = [1], H~_2m = [[H~_m, H~_m], [H~_m, -H~_m]] (Eq. supp_sylvester)."""
+    if m < 1 or (m & (m - 1)) != 0:
+        raise ValueError("Sylvester order must be a power of two")
+    H = np.ones((1, 1), dtype=np.int64)
+    while H.shape[0] < m:
+        H = np.block([[H, H], [H, -H]])
+    return H
+
+
+def blockdiag_transform(c: int, hb: int) -> np.ndarray:
+    """Normalized block-diagonal transform T = I_{c/hb} (x) H_hb (reading R1),
+    H_hb = H~_hb / sqrt(hb) (Eq. hadamard_properties). Dense fp64 [c, c]."""
+    if c % hb:
+        raise ValueError("channel count must be a multiple of the block")
+    H = sylvester(hb).astype(np.float64) / math.sqrt(hb)
+    return np.kron(np.eye(c // hb), H)
+
+
+def _blocks(x: np.ndarray, hb: int) -> np.ndarray:
+    c = x.shape[-1]
+    if c % hb:
+        raise ValueError("channel count must be a multiple of the block")
+    return x.reshape(x.shape[:-1] + (c // hb, hb))
+
+
+def transform_int(x: np.ndarray, hb: int) -> np.ndarray:
+    """Unnormalized integer transform along the last axis, block by block:
+    y_blk = H~_hb x_blk, exact in int64 (the integer transforms of the
+    integer basis conversions, Table integer_transitions)."""
+    x = np.asarray(x, dtype=np.int64)
+    if hb <= 1:
+        return x.copy()
+    H = sylvester(hb)
+    y = _blocks(x, hb) @ H.T            # y_j = sum_i H~[j, i] x_i
+    return y.reshape(x.shape)
+
+
+def transform_real(x: np.ndarray, hb: int, normalize: bool = True) -> np.ndarray:
+    """Real-valued transform along the last axis in the fixed order of
+    reading R6: y_j = (sum_{i=0}^{hb-1} H~[i][j] x_i) / sqrt(hb)."""
+    x = np.asarray(x, dtype=np.float64)
+    if hb <= 1:
+        return x.copy()
+    H = sylvester(hb).astype(np.float64)
+    xb = _blocks(x, hb)
+    acc = np.zeros_like(xb)
+    for i in range(hb):
+        acc += H[i][None, :] * xb[..., i:i + 1]
+    if normalize:
+        acc = acc / math.sqrt(hb)
+    return acc.reshape(x.shape)
+
+
+# --------------------------------------------------------------------------
+# Quantizers: Eq. (symmetric_q), reading R2/R4
+# --------------------------------------------------------------------------
+
+
+def symmetric_scale(x) -> float:
+    """s = ||x||_inf / q_max (Eq. symmetric_q); 1.0 for an all-zero tensor (R4)."""
+    m = float(np.max(np.abs(np.asarray(x, dtype=np.float64)))) if np.size(x) else 0.0
+    return m / QMAX if m > 0 else 1.0
+
+
+def quantize_sym(x, s: float) -> np.ndarray:
+    """x_int = clamp(round(x / s), -q_max, q_max) (Eq. symmetric_q)."""
+    q = np.rint(np.asarray(x, dtype=np.float64) / s)
+    return np.clip(q, -QMAX, QMAX).astype(np.int64)
+
+
+def rshift_rne(v, n: int) -> np.ndarray:
+    """round(v / 2^n) for integer v, ties to even (R2), exact in int64."""
+    v = np.asarray(v, dtype=np.int64)
+    if n == 0:
+        return v.copy()
+    q = v >> n                                    # floor(v / 2^n)
+    r = v - (q << n)                              # in [0, 2^n)
+    half = np.int64(1) << (n - 1)
+    up = (r > half) | ((r == half) & ((q & 1) == 1))
+    return q + up.astype(np.int64)
+
+
+def fixed_point(rho, a_bound, gain: int = 1):
+    """Multiplier/shift pair of Eqs. (fixed_point_scale, integer_fixed_point_scale)
+    under reading R3. rho: per-channel real ratios (> 0); a_bound: per-channel
+    bound on |input| of the multiplication; gain: product of the unnormalized
+    transform gains applied after M (.). Returns (M int64 array, n)."""
+    rho = np.asarray(rho, dtype=np.float64)
+    a_bound = [int(a) for a in np.asarray(a_bound).ravel()]
+    if np.any(rho < 0) or not np.all(np.isfinite(rho)):
+        raise ValueError("scale ratios must be finite and nonnegative")
+    for n in range(62, -1, -1):
+        M = [int(np.rint(math.ldexp(float(r), n))) for r in rho]
+        if max(M) >= 2 ** 31:
+            continue
+        worst = max(m * a for m, a in zip(M, a_bound)) * int(gain)
+        if worst >= 2 ** 62:
+            continue
+        if max(M) < 2 ** 15:
+            raise OverflowError("fewer than 16 bits of multiplier precision")
+        return np.array(M, dtype=np.int64), n
+    raise OverflowError("no shift satisfies the multiplier and overflow bounds")
+
+
+def round_half_even_fraction(f: Fraction) -> int:
+    fl = f.numerator // f.denominator
+    r = f - fl
+    if r > Fraction(1, 2) or (r == Fraction(1, 2) and fl % 2 == 1):
+        return fl + 1
+    return fl
+
+
+def dynamic_multiplier(maxy: int, hb: int):
+    """(M, n) for the dynamic INT8-entry quantizer: rho = 127 / max|y| as an
+    exact rational, M = round(rho 2^n) half to even, n by reading R3."""
+    if maxy <= 0:
+        return 0, 0
+    for n in range(62, -1, -1):
+        M = round_half_even_fraction(Fraction(QMAX << n, maxy))
+        if M >= 2 ** 31 or M * QMAX * hb >= 2 ** 62:
+            continue
+        if M < 2 ** 15:
+            raise OverflowError("fewer than 16 bits of multiplier precision")
+        return M, n
+    raise OverflowError("no shift satisfies the bounds")
+
+
+# --------------------------------------------------------------------------
+# Weight preparation (offline): DH Eq. (double_hadamard_quantization),
+# WH Eq. (supp_padded_wh_parameters), bias Eq. (supp_bias_quantization),
+# requant Eq. (integer_fixed_point_scale) with Table integer_transitions.
+# --------------------------------------------------------------------------
+
+
+def transform_weights(w_ohwi, b, form: str, hb_in: int, hb_out: int):
+    """Hadamard-domain weights and bias (fp64).
+    DH: W' = W (I_{KhKw} (x) T_in): every tap's C_in vector is transformed
+        (Eq. input_hadamard_transform); bias unchanged.
+    WH: W_bar = T_out^T W along C_out, b_bar = b T_out
+        (Eq. supp_padded_wh_parameters)."""
+    w = np.asarray(w_ohwi, dtype=np.float64)
+    bb = np.zeros(w.shape[0]) if b is None else np.asarray(b, dtype=np.float64)
+    if form == "DH":
+        return transform_real(w, hb_in), bb.copy()
+    if form == "WH":
+        wt = np.moveaxis(w, 0, -1)                    # [kh, kw, ci, co]
+        wbar = np.moveaxis(transform_real(wt, hb_out), -1, 0)
+        return wbar, transform_real(bb, hb_out)
+    raise ValueError(form)
+
+
+class Prepared:
+    """One prepared layer: INT8 weights, per-channel scales, bias codes and
+    fixed-point requant parameters, in the Hadamard domain of its form."""
+
+    def __init__(self, **kw):
+        self.__dict__.update(kw)
+
+
+def prepare_layer(w_ohwi, b, form: str, hb_in: int, hb_out: int, s_x: float,
+                  s_y: float, act: str, hb_next: int, out_f32: bool,
+                  stride: int, pad: int) -> Prepared:
+    """Offline preparation of one layer (Sec. deployment realization).
+    s_x: scale of the INT8 operand this layer consumes; s_y: scale of the
+    INT8 operand the next layer consumes (or of this layer's output)."""
+    s_x = float(np.float32(s_x))
+    s_y = float(np.float32(s_y))
+    wprime, bbar = transform_weights(w_ohwi, b, form, hb_in, hb_out)
+    co = wprime.shape[0]
+    flat = wprime.reshape(co, -1)
+    maxabs = np.max(np.abs(flat), axis=1)
+    s_w = np.where(maxabs > 0, maxabs / QMAX, 1.0)               # channel-wise Eq. symmetric_q
+    w_int = np.clip(np.rint(flat / s_w[:, None]), -QMAX, QMAX).astype(np.int64)
+    s_a = s_x * s_w                                              # Eq. accumulator_scale
+    b_int = np.rint(bbar / s_a).astype(np.int64)                 # Eq. supp_bias_quantization
+    g_out = math.sqrt(hb_out) if form == "WH" else 1.0           # Table integer_transitions
+    g_in = math.sqrt(hb_next) if hb_next else 1.0
+    a_bound = QMAX * np.sum(np.abs(w_int), axis=1) + np.abs(b_int)
+    if int(np.max(a_bound)) >= 2 ** 31:
+        raise OverflowError("int32 accumulator bound exceeded")
+    prep = Prepared(form=form, hb_in=hb_in, hb_out=hb_out if form == "WH" else 0,
+                    hb_next=hb_next, act=act, out_f32=out_f32, stride=stride, pad=pad,
+                    s_x=s_x, s_y=s_y, s_w=s_w, b_int=b_int,
+                    w_int=w_int.reshape(wprime.shape).astype(np.int8),
+                    a_bound=a_bound, wprime=wprime, bbar=bbar)
+    if out_f32:
+        prep.deq = s_a / g_out
+        prep.M, prep.n = None, 0
+    else:
+        alpha = g_out * g_in
+        rho = s_a / (alpha * s_y)                                # Eq. integer_fixed_point_scale
+        gain = (hb_out if form == "WH" else 1) * (hb_next if hb_next else 1)
+        prep.M, prep.n = fixed_point(rho, a_bound, gain)
+        prep.rho = rho
+    return prep
+
+
+# --------------------------------------------------------------------------
+# Activation transform + quantize (online): Eqs. (double_hadamard_quantization,
+# symmetric_q); INT8 entry uses the integer input transform and fixed-point
+# rescaling of Eq. (supp_general_input_transition) with M^in, n^in.
+# --------------------------------------------------------------------------
+
+
+def quantize_act_f16(x, hb: int, s_x: float) -> np.ndarray:
+    """FP16 entry: codes of Q_a(X H_in): clamp(rint((H~ x)_j / (sqrt(hb) s_x)))."""
+    y = transform_real(np.asarray(x, dtype=np.float64), hb, normalize=False)
+    return np.clip(np.rint(y / (math.sqrt(hb) * float(np.float32(s_x)))), -QMAX, QMAX).astype(np.int8)
+
+
+def act_multiplier(hb: int, s_in: float, s_x: float):
+    """(M_q, n_q) with M_q / 2^n_q ~ s_in / (sqrt(hb) s_x), bound |y| <= 127 hb."""
+    rho = float(np.float32(s_in)) / (math.sqrt(hb) * float(np.float32(s_x)))
+    M, n = fixed_point([rho], [QMAX * hb], 1)
+    return int(M[0]), n
+
+
+def quantize_act_i8(x_i8, hb: int, s_in: float, s_x: float) -> np.ndarray:
+    """INT8 entry: y = H~ x (exact), codes = clamp(round(M_q y / 2^n_q))."""
+    M, n = act_multiplier(hb, s_in, s_x)
+    y = transform_int(x_i8, hb)
+    return np.clip(rshift_rne(M * y, n), -QMAX, QMAX).astype(np.int8)
+
+
+def quantize_act_dynamic_i8(x_i8, hb: int, s_in: float):
+    """Dynamic per-tensor scale (PTQ, Sec. network-wise PTQ): s from the
+    transformed tensor's max-abs, then the INT8 entry quantizer. Returns
+    (codes, s_used) with s_used = s_in max|H~x| / (sqrt(hb) 127) (fp64 -> fp32)."""
+    y = transform_int(x_i8, hb)
+    maxy = int(np.max(np.abs(y))) if y.size else 0
+    if maxy == 0:
+        return np.zeros(y.shape, dtype=np.int8), 1.0
+    M, n = dynamic_multiplier(maxy, hb)
+    codes = np.clip(rshift_rne(M * y, n), -QMAX, QMAX).astype(np.int8)
+    s_used = float(np.float32(float(np.float32(s_in)) * maxy / (math.sqrt(hb) * QMAX)))
+    return codes, s_used
+
+
+def quantize_act_dynamic_f16(x, hb: int):
+    """Dynamic FP16 entry: s = max|H x| / 127; returns (codes, s_used)."""
+    y = transform_real(np.asarray(x, dtype=np.float64), hb, normalize=False)
+    m = float(np.max(np.abs(y))) if y.size else 0.0
+    if m == 0.0:
+        return np.zeros(y.shape, dtype=np.int8), 1.0
+    codes = np.clip(np.rint(y * (QMAX / m)), -QMAX, QMAX).astype(np.int8)
+    return codes, m / (math.sqrt(hb) * QMAX)
+
+
+# --------------------------------------------------------------------------
+# Convolution on codes (conv_ref.c) and the requantize epilogue
+# --------------------------------------------------------------------------
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB = None
+
+
+def build_lib(force: bool = False) -> str:
+    out_dir = os.path.join(_HERE, "_build")
+    so = os.path.join(out_dir, "liboracle.so")
+    src = os.path.join(_HERE, "conv_ref.c")
+    if force or not os.path.exists(so) or os.path.getmtime(so) < os.path.getmtime(src):
+        os.makedirs(out_dir, exist_ok=True)
+        tmp = so + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", "-O2", "-fPIC", "-shared", "-ffp-contract=off",
+                               "-o", tmp, src])
+        os.replace(tmp, so)
+    return so
+
+
+def _lib():
+    global _LIB
+    if _LIB is None:
+        lib = ctypes.CDLL(build_lib())
+        i64 = ctypes.c_int64
+        p = ctypes.c_void_p
+        lib.oracle_conv2d_codes.argtypes = [p, i64, i64, i64, i64, p, i64, i64, i64, i64, i64,
+                                            i64, i64, i64, i64, p]
+        lib.oracle_conv2d_codes_at.argtypes = [p, i64, i64, i64, i64, p, i64, i64, i64, i64, i64,
+                                               p, i64, p]
+        _LIB = lib
+    return _LIB
+
+
+def out_hw(h, w, k, stride, pad):
+    return (h + 2 * pad - k) // stride + 1, (w + 2 * pad - k) // stride + 1
+
+
+def conv_codes(x_i8, w_int, stride: int, pad: int, window=None) -> np.ndarray:
+    """Integer accumulator sum_k x_int w_int over the unfolded patch
+    (Eqs. integer_accumulation, linear_operator). x: NHWC int8, w: OHWI int8.
+    window = (ho0, ho1, wo0, wo1) restricts the output rows/columns."""
+    x = np.ascontiguousarray(x_i8, dtype=np.int8)
+    w = np.ascontiguousarray(w_int, dtype=np.int8)
+    n, h, wd, c = x.shape
+    co, kh, kw, ci = w.shape
+    if ci != c:
+        raise ValueError("channel mismatch")
+    ho, wo = out_hw(h, wd, kh, stride, pad)
+    ho0, ho1, wo0, wo1 = window if window is not None else (0, ho, 0, wo)
+    acc = np.zeros((n, ho1 - ho0, wo1 - wo0, co), dtype=np.int64)
+    _lib().oracle_conv2d_codes(x.ctypes.data, n, h, wd, c, w.ctypes.data, co, kh, kw,
+                               stride, pad, ho0, ho1, wo0, wo1, acc.ctypes.data)
+    return acc
+
+
+def conv_codes_at(x_i8, w_int, stride: int, pad: int, pix) -> np.ndarray:
+    """The accumulator at output pixels pix[i] = (b, oy, ox): [npix, co]."""
+    x = np.ascontiguousarray(x_i8, dtype=np.int8)
+    w = np.ascontiguousarray(w_int, dtype=np.int8)
+    pix = np.ascontiguousarray(pix, dtype=np.int64).reshape(-1, 3)
+    n, h, wd, c = x.shape
+    co, kh, kw, _ = w.shape
+    acc = np.zeros((pix.shape[0], co), dtype=np.int64)
+    _lib().oracle_conv2d_codes_at(x.ctypes.data, n, h, wd, c, w.ctypes.data, co, kh, kw,
+                                  stride, pad, pix.ctypes.data, pix.shape[0], acc.ctypes.data)
+    return acc
+
+
+def epilogue_int(acc, p: Prepared) -> np.ndarray:
+    """Integer transition of Eq. (integer_hadamard_transition) with the bias of
+    Eq. (supp_bias_quantization) added first (R5):
+        a = acc + b_int;  v = H~_out (M (.) a);  u = phi(v);
+        x_next = clamp(round(H~_in,next(u) / 2^n), -127, 127)."""
+    a = np.asarray(acc, dtype=np.int64) + p.b_int
+    t = p.M * a
+    v = transform_int(t, p.hb_out) if p.hb_out else t
+    u = np.maximum(v, 0) if p.act == "relu" else v
+    w = transform_int(u, p.hb_next) if p.hb_next else u
+    return np.clip(rshift_rne(w, p.n), -QMAX, QMAX).astype(np.int8)
+
+
+def epilogue_f32(acc, p: Prepared) -> np.ndarray:
+    """Dequantized output: y = H_out (s_A (.) a) (WH) or s_A (.) a (DH), then phi;
+    with deq_c = s_x s_w,c / gamma_out the WH form is H~_out (deq (.) a)."""
+    a = np.asarray(acc, dtype=np.int64) + p.b_int
+    t = p.deq * a.astype(np.float64)
+    v = transform_real(t, p.hb_out, normalize=False) if p.hb_out else t
+    return np.maximum(v, 0.0) if p.act == "relu" else v
+
+
+def conv_layer(x_op, p: Prepared, window=None):
+    """One prepared layer on its INT8 operand: conv + epilogue."""
+    acc = conv_codes(x_op, p.w_int, p.stride, p.pad, window)
+    return epilogue_f32(acc, p) if p.out_f32 else epilogue_int(acc, p)
+
+
+# --------------------------------------------------------------------------
+# Layer stacking by the static profile mask (Sec. layer-wise selection,
+# Table integer_transitions)
+# --------------------------------------------------------------------------
+
+
+def layer_operand(x, x_kind: str, s_in: float, form: str, hb_in: int, s_x: float):
+    """The INT8 operand a layer consumes from its input.
+    x_kind: 'operand' (already the operand), 'i8' (original-basis codes at
+    s_in) or 'f16' (real values). DH applies the input transform (hb_in);
+    WH only rescales (identity transform)."""
+    hb = hb_in if form == "DH" else 1
+    if x_kind == "operand":
+        return np.asarray(x, dtype=np.int8)
+    if x_kind == "f16":
+        return quantize_act_f16(x, hb, s_x)
+    if x_kind == "i8":
+        if form == "WH" and float(np.float32(s_in)) == float(np.float32(s_x)):
+            return np.asarray(x, dtype=np.int8)
+        return quantize_act_i8(x, hb, s_in, s_x)
+    raise ValueError(x_kind)
+
+
+def prepare_chain(layers, params, scales, plan, out_f32_last=False):
+    """layers: LayerSpec-like objects; params: [(w, b)]; scales: [{'s_x','s_out'}];
+    plan: per layer the fused next-layer DH block (0 = none)."""
+    preps = []
+    for i, (L, (w, b), sc) in enumerate(zip(layers, params, scales)):
+        last = i == len(layers) - 1
+        preps.append(prepare_layer(w, b, L.form, L.hb_in, L.hb_out, sc["s_x"], sc["s_out"],
+                                   L.act, plan[i], out_f32_last and last, L.stride, L.pad))
+    return preps
+
+
+def chain_forward(layers, preps, plan, x, x_kind, s_in):
+    """Run a chain on the oracle. Returns the list of per-layer outputs."""
+    outs = []
+    cur, kind, s_cur = x, x_kind, s_in
+    for i, (L, p) in enumerate(zip(layers, preps)):
+        op = layer_operand(cur, kind, s_cur, L.form, L.hb_in, p.s_x)
+        y = conv_layer(op, p)
+        outs.append(y)
+        fused = plan[i] != 0
+        cur, s_cur = y, p.s_y
+        kind = "operand" if (fused or (i + 1 < len(layers) and layers[i + 1].form == "WH")) else "i8"
+    return outs
+
+
+# --------------------------------------------------------------------------
+# Real-valued model (fp64): the function the quantized operator approximates
+# --------------------------------------------------------------------------
+
+
+def conv_real(x, w_ohwi, b, stride: int, pad: int) -> np.ndarray:
+    """Y = X W^T + b on unfolded patches (Eq. supp_linear_operator), fp64,
+    with a library matmul per kernel tap."""
+    x = np.asarray(x, dtype=np.float64)
+    w = np.asarray(w_ohwi, dtype=np.float64)
+    n, h, wd, c = x.shape
+    co, kh, kw, _ = w.shape
+    ho, wo = out_hw(h, wd, kh, stride, pad)
+    xp = np.zeros((n, h + 2 * pad, wd + 2 * pad, c))
+    xp[:, pad:pad + h, pad:pad + wd, :] = x
+    y = np.zeros((n, ho, wo, co))
+    for ky in range(kh):
+        for kx in range(kw):
+            patch = xp[:, ky:ky + stride * (ho - 1) + 1:stride, kx:kx + stride * (wo - 1) + 1:stride, :]
+            y += patch @ w[:, ky, kx, :].T
+    if b is not None:
+        y += np.asarray(b, dtype=np.float64)
+    return y
+
+
+def calibrate_chain(layers, params, x_real, plan, first_wh_scale=None):
+    """Static scales from the real-valued model (QAT-style frozen scales,
+    Sec. quantization-aware training): per layer, s_x = max-abs of the
+    operand in its quantizer's basis / 127, and s_out = the scale of what the
+    layer emits (the next operand when fused or next is WH, the
+    original-basis intermediate otherwise, or the final output)."""
+    scales = []
+    x = np.asarray(x_real, dtype=np.float64)
+    reals = []
+    for i, (L, (w, b)) in enumerate(zip(layers, params)):
+        if L.form == "DH":
+            s_x = symmetric_scale(transform_real(x, L.hb_in))
+        else:
+            s_x = symmetric_scale(x) if (i or first_wh_scale is None) else first_wh_scale
+        y = conv_real(x, w, b, L.stride, L.pad)
+        xn = np.maximum(y, 0.0) if L.act == "relu" else y
+        reals.append((x, xn))
+        scales.append({"s_x": float(np.float32(s_x))})
+        x = xn
+    for i, L in enumerate(layers):
+        xn = reals[i][1]
+        if plan[i]:
+            s_out = symmetric_scale(transform_real(xn, plan[i]))
+        else:
+            s_out = symmetric_scale(xn)
+        scales[i]["s_out"] = float(np.float32(s_out))
+    return scales
+
+
+# --------------------------------------------------------------------------
+# Diagnostics: Eqs. (excess_kurtosis, sqnr, hadamard_sensitivity)
+# --------------------------------------------------------------------------
+
+
+def excess_kurtosis(x) -> float:
+    x = np.asarray(x, dtype=np.float64).ravel()
+    mu = x.mean()
+    d = x - mu
+    return float(np.mean(d ** 4) / np.mean(d ** 2) ** 2 - 3.0)
+
+
+def sqnr_db(x, xhat) -> float:
+    x = np.asarray(x, dtype=np.float64)
+    e = x - np.asarray(xhat, dtype=np.float64)
+    return float(10.0 * np.log10(np.sum(x * x) / np.sum(e * e)))
+
+
+def range_expands(x, hb: int) -> bool:
+    """Indicator of Eq. (hadamard_sensitivity) for one tensor."""
+    return float(np.max(np.abs(transform_real(x, hb)))) > float(np.max(np.abs(x)))

@@ -1,0 +1,140 @@
+"""Plants plausible mistakes in the CPU oracle (on the CPU, via monkeypatch)
+and checks that at least one pin in test_oracle_pins.py catches each of
+them: a dropped term, a wrong sign or index, a transposed operand, a wrong
+normalization or rounding."""
+import math
+
+import numpy as np
+import pytest
+
+import tests.test_oracle_pins as P
+from oracle import hatq_oracle as O
+
+_orig = {k: getattr(O, k) for k in ("sylvester", "transform_real", "transform_int", "rshift_rne",
+                                    "fixed_point", "prepare_layer", "epilogue_int", "conv_codes",
+                                    "quantize_act_i8", "transform_weights", "quantize_sym",
+                                    "act_multiplier")}
+
+
+def _sylvester_bad(m):
+    H = _orig["sylvester"](m).copy()
+    if m >= 4:
+        H[-1, 1] *= -1
+    return H
+
+
+def _transform_real_bad(x, hb, normalize=True):
+    y = _orig["transform_real"](x, hb, normalize=False)
+    return y / hb if normalize and hb > 1 else y
+
+
+def _transform_int_bad(x, hb):
+    y = _orig["transform_int"](x, hb)
+    if hb > 1:
+        y = y.reshape(-1, y.shape[-1])
+        y[:, 1] = -y[:, 1]
+    return y.reshape(np.shape(x))
+
+
+def _rshift_floor(v, n):
+    return np.asarray(v, dtype=np.int64) >> n
+
+
+def _fixed_point_no_gain(rho, a_bound, gain=1):
+    return _orig["fixed_point"](rho, a_bound, 1)
+
+
+def _prepare_no_gamma_in(*a, **k):
+    p = _orig["prepare_layer"](*a, **k)
+    if getattr(p, "rho", None) is not None and p.hb_next:
+        p.rho = p.rho * math.sqrt(p.hb_next)
+    return p
+
+
+def _epilogue_m_after_h(acc, p):
+    a = np.asarray(acc, dtype=np.int64) + p.b_int
+    v = O.transform_int(a, p.hb_out) if p.hb_out else a
+    t = p.M * v
+    u = np.maximum(t, 0) if p.act == "relu" else t
+    w = O.transform_int(u, p.hb_next) if p.hb_next else u
+    return np.clip(O.rshift_rne(w, p.n), -127, 127).astype(np.int8)
+
+
+def _epilogue_no_bias(acc, p):
+    class Q:
+        pass
+    q = Q()
+    q.__dict__.update(p.__dict__)
+    q.b_int = np.zeros_like(p.b_int)
+    return _orig["epilogue_int"](acc, q)
+
+
+def _conv_swap(x, w, stride, pad, window=None):
+    return _orig["conv_codes"](x, w, pad if pad else stride, stride, window)
+
+
+def _act_mult_no_sqrt(hb, s_in, s_x):
+    rho = float(np.float32(s_in)) / float(np.float32(s_x))
+    M, n = O.fixed_point([rho], [127 * hb], 1)
+    return int(M[0]), n
+
+
+def _wh_wrong_axis(w_ohwi, b, form, hb_in, hb_out):
+    if form == "WH":
+        w = np.asarray(w_ohwi, dtype=np.float64)
+        hb = min(hb_out, w.shape[-1] & -w.shape[-1])
+        return O.transform_real(w, hb), O.transform_real(np.asarray(b, np.float64), hb_out)
+    return _orig["transform_weights"](w_ohwi, b, form, hb_in, hb_out)
+
+
+def _quantize_floor(x, s):
+    return np.clip(np.floor(np.asarray(x, dtype=np.float64) / s), -127, 127).astype(np.int64)
+
+
+MUTATIONS = {
+    "sylvester_sign": ("sylvester", _sylvester_bad),
+    "normalize_by_m": ("transform_real", _transform_real_bad),
+    "int_transform_sign": ("transform_int", _transform_int_bad),
+    "shift_floor": ("rshift_rne", _rshift_floor),
+    "fixed_point_gain_dropped": ("fixed_point", _fixed_point_no_gain),
+    "gamma_in_dropped": ("prepare_layer", _prepare_no_gamma_in),
+    "M_after_H_out": ("epilogue_int", _epilogue_m_after_h),
+    "bias_dropped": ("epilogue_int", _epilogue_no_bias),
+    "conv_stride_pad_swapped": ("conv_codes", _conv_swap),
+    "act_requant_no_sqrt": ("act_multiplier", _act_mult_no_sqrt),
+    "wh_transform_wrong_axis": ("transform_weights", _wh_wrong_axis),
+    "quantizer_floor": ("quantize_sym", _quantize_floor),
+}
+
+
+def _pins():
+    """Every pin test, expanded over its parametrization."""
+    out = []
+    for name in dir(P):
+        if not name.startswith("test_"):
+            continue
+        fn = getattr(P, name)
+        marks = getattr(fn, "pytestmark", [])
+        params = [m for m in marks if m.name == "parametrize"]
+        if not params:
+            out.append((name, fn, {}))
+            continue
+        m = params[0]
+        argnames = [a.strip() for a in m.args[0].split(",")] if isinstance(m.args[0], str) else list(m.args[0])
+        for vals in m.args[1]:
+            vals = vals if len(argnames) > 1 else (vals,)
+            out.append((name, fn, dict(zip(argnames, vals))))
+    return out
+
+
+@pytest.mark.parametrize("mutation", sorted(MUTATIONS))
+def test_planted_mistake_is_caught(mutation, monkeypatch):
+    attr, bad = MUTATIONS[mutation]
+    monkeypatch.setattr(O, attr, bad)
+    caught = []
+    for name, fn, kw in _pins():
+        try:
+            fn(**kw)
+        except (Exception, pytest.fail.Exception):  # a failed pin or an error in the mutated oracle
+            caught.append(name)
+    assert caught, f"no pin catches the planted mistake {mutation}"

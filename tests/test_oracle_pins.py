@@ -1,0 +1,398 @@
+"""Pins for the CPU oracle: each check compares the oracle with something
+other than itself (a closed form, an identity of the paper, a worked table,
+brute force, exact rational arithmetic)."""
+import json
+import math
+import os
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+from oracle import hatq_oracle as O
+from synth import inputs as I
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def popcount_sign(m):
+    """Closed form of the Sylvester matrix: H~[i][j] = (-1)^popcount(i & j)."""
+    i = np.arange(m)[:, None]
+    j = np.arange(m)[None, :]
+    pc = np.vectorize(lambda v: bin(int(v)).count("1"))(i & j)
+    return np.where(pc % 2 == 0, 1, -1)
+
+
+# ---------------------------------------------------------------- Hadamard (T1)
+
+@pytest.mark.parametrize("m", [1, 2, 4, 8, 16, 32, 64, 128, 256])
+def test_sylvester_orthogonal_closed_form(m):
+    H = O.sylvester(m)
+    assert np.array_equal(H @ H.T, m * np.eye(m, dtype=np.int64))          # Eq. supp_hadamard_properties
+    assert np.array_equal(H, popcount_sign(m))
+    assert np.all(H[0] == 1) and np.all(H[:, 0] == 1)                        # constant basis h0 first
+    assert np.array_equal(H, H.T)
+
+
+def test_sylvester_h4_golden():
+    rows = [l.split() for l in open(os.path.join(GOLDEN, "sylvester_h4.txt")) if not l.startswith("#")]
+    ref = np.array([[int(v) for v in r] for r in rows if r])
+    assert np.array_equal(O.sylvester(4), ref)
+
+
+def test_sylvester_rejects_non_power_of_two():
+    with pytest.raises(ValueError):
+        O.sylvester(12)
+
+
+@pytest.mark.parametrize("c,hb", [(128, 128), (192, 64), (320, 64), (224, 32), (64, 16)])
+def test_blockdiag_orthonormal_and_transforms(c, hb):
+    T = O.blockdiag_transform(c, hb)
+    assert np.allclose(T @ T.T, np.eye(c), atol=1e-13)
+    rng = np.random.default_rng(c + hb)
+    x = rng.standard_normal((5, c))
+    # ordered-loop transform == dense Kronecker matrix product
+    assert np.allclose(O.transform_real(x, hb), x @ T, atol=1e-12)
+    xi = rng.integers(-127, 128, size=(7, c))
+    Hc = np.kron(np.eye(c // hb, dtype=np.int64), popcount_sign(hb))
+    assert np.array_equal(O.transform_int(xi, hb), xi @ Hc.T)
+
+
+def test_parseval():                                                          # T4
+    x = I.activations((1, 4, 4, 192), seed=5).astype(np.float64)
+    y = O.transform_real(x, 64)
+    assert np.allclose(np.sum(y * y), np.sum(x * x), rtol=1e-12)
+
+
+@pytest.mark.parametrize("hb", [16, 64, 128])
+def test_coherent_mean_accumulation(hb):                                      # T3, Eq. hadamard_mean_accumulation
+    mu = 0.731
+    x = np.full((3, hb), mu)
+    y = O.transform_real(x, hb)
+    assert np.allclose(y[:, 0], math.sqrt(hb) * mu, rtol=1e-14)
+    assert np.allclose(y[:, 1:], 0.0, atol=1e-13)
+    yi = O.transform_int(np.full((2, hb), 5), hb)
+    assert np.all(yi[:, 0] == 5 * hb) and np.all(yi[:, 1:] == 0)
+
+
+def test_coherent_mean_general_vector():
+    """y0 = C / sqrt(m) * mean(x) for any vector (unpadded: sqrt(C) * mean)."""
+    rng = np.random.default_rng(3)
+    x = rng.standard_normal((10, 64)) + 2.0
+    y = O.transform_real(x, 64)
+    assert np.allclose(y[:, 0], math.sqrt(64) * x.mean(axis=1), rtol=1e-12)
+
+
+# ------------------------------------------------------- function preservation (T2)
+
+def _rel(a, b):
+    return float(np.max(np.abs(a - b)) / np.max(np.abs(b)))
+
+
+@pytest.mark.parametrize("k,stride,pad,c_in,c_out,hb", [(1, 1, 0, 64, 32, 64), (3, 1, 1, 32, 48, 32),
+                                                        (5, 2, 2, 64, 16, 16)])
+def test_dh_function_preservation(k, stride, pad, c_in, c_out, hb):
+    """Eq. hadamard_linear_equivalence: (X H_in)(W H_in)^T = X W^T."""
+    x = I.activations((2, 9, 7, c_in), seed=11).astype(np.float64)
+    w = I.weights(c_out, k, k, c_in, seed=12).astype(np.float64)
+    b = I.bias(c_out, seed=13).astype(np.float64)
+    wp, bb = O.transform_weights(w, b, "DH", hb, 0)
+    y_ref = O.conv_real(x, w, b, stride, pad)
+    y_dh = O.conv_real(O.transform_real(x, hb), wp, bb, stride, pad)
+    assert _rel(y_dh, y_ref) < 1e-12
+
+
+@pytest.mark.parametrize("c_out,hb", [(64, 64), (96, 32), (128, 128)])
+def test_wh_function_preservation(c_out, hb):
+    """Eq. supp_padded_wh: (X W_bar^T + b_bar) T_out^T = X W^T + b."""
+    x = I.activations((1, 6, 6, 16), seed=21).astype(np.float64)
+    w = I.weights(c_out, 3, 3, 16, seed=22).astype(np.float64)
+    b = I.bias(c_out, seed=23).astype(np.float64)
+    wbar, bbar = O.transform_weights(w, b, "WH", 0, hb)
+    acc = O.conv_real(x, wbar, bbar, 1, 1)
+    y_wh = O.transform_real(acc, hb)
+    assert _rel(y_wh, O.conv_real(x, w, b, 1, 1)) < 1e-12
+    # and b_bar is b mapped into the output Hadamard basis: b_bar T_out^T = b
+    assert np.allclose(O.transform_real(bbar, hb), b, atol=1e-14)
+
+
+# ------------------------------------------------------------ direct conv (T5)
+
+def im2col_conv(x, w, stride, pad):
+    """Independent formulation: explicit patch matrix times weight matrix."""
+    n, h, wd, c = x.shape
+    co, kh, kw, _ = w.shape
+    ho = (h + 2 * pad - kh) // stride + 1
+    wo = (wd + 2 * pad - kw) // stride + 1
+    rows = []
+    for b in range(n):
+        for oy in range(ho):
+            for ox in range(wo):
+                patch = []
+                for ky in range(kh):
+                    for kx in range(kw):
+                        iy, ix = oy * stride + ky - pad, ox * stride + kx - pad
+                        if 0 <= iy < h and 0 <= ix < wd:
+                            patch.extend(int(v) for v in x[b, iy, ix])
+                        else:
+                            patch.extend([0] * c)
+                rows.append(patch)
+    A = np.array(rows, dtype=np.int64)
+    B = w.reshape(co, -1).astype(np.int64)
+    return (A @ B.T).reshape(n, ho, wo, co)
+
+
+@pytest.mark.parametrize("shape,co,k,stride,pad", [((1, 8, 8, 3), 5, 5, 2, 2), ((2, 7, 5, 16), 8, 3, 1, 1),
+                                                   ((1, 6, 6, 32), 4, 1, 1, 0), ((1, 9, 8, 8), 3, 5, 2, 2),
+                                                   ((1, 5, 5, 4), 2, 3, 2, 0)])
+def test_conv_codes_brute_force(shape, co, k, stride, pad):
+    x = I.uniform_codes(shape, seed=31)
+    w = I.uniform_codes((co, k, k, shape[3]), seed=32)
+    ref = im2col_conv(x, w, stride, pad)
+    got = O.conv_codes(x, w, stride, pad)
+    assert np.array_equal(got, ref)
+    ho, wo = ref.shape[1:3]
+    win = O.conv_codes(x, w, stride, pad, window=(1, ho, 0, max(1, wo - 1)))
+    assert np.array_equal(win, ref[:, 1:ho, 0:max(1, wo - 1)])
+    pix = np.array([[b, oy, ox] for b in range(shape[0]) for oy in range(ho) for ox in range(wo)])
+    at = O.conv_codes_at(x, w, stride, pad, pix)
+    assert np.array_equal(at, ref.reshape(-1, co))
+
+
+def test_conv_codes_extreme_values():
+    x = np.full((1, 4, 4, 64), -127, dtype=np.int8)
+    w = np.full((2, 3, 3, 64), 127, dtype=np.int8)
+    acc = O.conv_codes(x, w, 1, 1)
+    assert acc[0, 1, 1, 0] == -127 * 127 * 9 * 64
+    assert acc[0, 0, 0, 0] == -127 * 127 * 4 * 64
+
+
+# ------------------------------------------------------- rounding / fixed point (T6)
+
+def test_rshift_rne_matches_exact_rationals():
+    rng = np.random.default_rng(7)
+    v = np.concatenate([rng.integers(-2 ** 40, 2 ** 40, size=2000),
+                        np.array([5, -5, 3, -3, 7, -7, 1, -1, 0, 2 ** 41 + 2 ** 9, -(2 ** 41) - 2 ** 9])])
+    for n in [0, 1, 2, 3, 10, 20]:
+        got = O.rshift_rne(v, n)
+        ref = [O.round_half_even_fraction(Fraction(int(a), 2 ** n)) for a in v]
+        assert list(got) == ref
+
+
+def test_round_half_even_fraction_ties():
+    assert [O.round_half_even_fraction(Fraction(k, 2)) for k in (-5, -3, -1, 1, 3, 5)] == [-2, -2, 0, 0, 2, 2]
+
+
+def test_fixed_point_rule_is_maximal_and_accurate():
+    rng = np.random.default_rng(9)
+    rho = rng.lognormal(-6, 2, size=64)
+    a_bound = rng.integers(10 ** 5, 10 ** 8, size=64)
+    for gain in (1, 64, 64 * 64):
+        M, n = O.fixed_point(rho, a_bound, gain)
+        for r, m in zip(rho, M):
+            assert abs(Fraction(int(m)) - Fraction(float(r)) * 2 ** n) <= Fraction(1, 2)
+        assert max(M) < 2 ** 31 and max(int(m) * int(a) for m, a in zip(M, a_bound)) * gain < 2 ** 62
+        if n < 62:  # n + 1 must violate a bound
+            M2 = [int(np.rint(math.ldexp(float(r), n + 1))) for r in rho]
+            assert max(M2) >= 2 ** 31 or max(m * int(a) for m, a in zip(M2, a_bound)) * gain >= 2 ** 62
+
+
+def test_fixed_point_precision_floor():
+    with pytest.raises(OverflowError):
+        O.fixed_point([1e-9], [2 ** 30], 2 ** 28)
+
+
+def test_dynamic_multiplier_exact():
+    for maxy in (1, 3, 127, 1000, 8191, 127 * 64):
+        M, n = O.dynamic_multiplier(maxy, 64)
+        assert abs(Fraction(M) - Fraction(127 * 2 ** n, maxy)) <= Fraction(1, 2)
+        y = np.array([maxy, -maxy, 0])
+        codes = np.clip(O.rshift_rne(M * y, n), -127, 127)
+        assert list(codes) == [127, -127, 0]
+
+
+# --------------------------------------------------------------- quantizers
+
+def test_symmetric_quantizer():                                                # Eq. symmetric_q
+    x = I.activations((1, 8, 8, 32), seed=41).astype(np.float64)
+    s = O.symmetric_scale(x)
+    q = O.quantize_sym(x, s)
+    assert np.max(np.abs(q)) == 127 and q.min() >= -127
+    assert np.max(np.abs(q * s - x)) <= s / 2 + 1e-12
+    assert O.symmetric_scale(np.zeros(5)) == 1.0
+
+
+def test_quantize_act_f16_is_quantized_transform():
+    x = I.activations_f16((1, 4, 4, 128), seed=42)
+    y = O.transform_real(x.astype(np.float64), 128)
+    s = O.symmetric_scale(y)
+    q = O.quantize_act_f16(x, 128, s).astype(np.int64)
+    assert np.max(np.abs(q * s - y)) <= float(np.float32(s)) / 2 * (1 + 1e-6)
+
+
+def test_quantize_act_i8_close_to_real_rescale():
+    x = I.activations_i8((1, 6, 6, 192), seed=43, s_in=0.05)
+    s_in = 0.05
+    y = O.transform_real(x.astype(np.float64) * float(np.float32(s_in)), 64)
+    s_x = float(np.float32(O.symmetric_scale(y)))
+    q = O.quantize_act_i8(x, 64, s_in, s_x).astype(np.int64)
+    exact = np.clip(np.rint(y / s_x), -127, 127)
+    diff = np.abs(q - exact)
+    assert diff.max() <= 1 and np.mean(diff > 0) < 1e-3
+
+
+def test_quantize_act_dynamic():
+    x = I.activations_i8((1, 5, 5, 64), seed=44, s_in=0.05)
+    codes, s_used = O.quantize_act_dynamic_i8(x, 64, 0.05)
+    assert np.max(np.abs(codes.astype(int))) == 127
+    y = O.transform_real(x.astype(np.float64) * float(np.float32(0.05)), 64)
+    assert math.isclose(s_used, np.max(np.abs(y)) / 127, rel_tol=1e-6)
+    assert np.max(np.abs(codes * s_used - y)) <= s_used * 0.5001
+    z, s0 = O.quantize_act_dynamic_i8(np.zeros((1, 2, 2, 64), np.int8), 64, 0.05)
+    assert s0 == 1.0 and not z.any()
+    xf = I.activations_f16((1, 3, 3, 128), seed=45)
+    cf, sf = O.quantize_act_dynamic_f16(xf, 128)
+    assert np.max(np.abs(cf.astype(int))) == 127
+    assert math.isclose(sf, np.max(np.abs(O.transform_real(xf.astype(np.float64), 128))) / 127, rel_tol=1e-12)
+
+
+# ---------------------------------------------------- integer transitions (golden table)
+
+def test_transition_gammas_match_paper_table():
+    tab = json.load(open(os.path.join(GOLDEN, "transitions.json")))["transitions"]
+    m = 64
+    val = {"1": 1.0, "sqrt(m)": math.sqrt(m)}
+    w = I.weights(m, 1, 1, m, seed=50)
+    for row in tab:
+        form = row["from"]
+        hb_next = m if row["to"] == "DH" else 0
+        p = O.prepare_layer(w, None, form, m if form == "DH" else 0, m if form == "WH" else 0,
+                            s_x=0.02, s_y=0.03, act="none", hb_next=hb_next, out_f32=False,
+                            stride=1, pad=0)
+        alpha = val[row["gamma_out"]] * val[row["gamma_in"]]
+        expect = (float(np.float32(0.02)) * p.s_w) / (alpha * float(np.float32(0.03)))
+        assert np.allclose(p.rho, expect, rtol=1e-15)
+        assert (p.hb_out > 0) == (row["H_out"] == "H")
+        assert (p.hb_next > 0) == (row["H_in"] == "H")
+
+
+def _exact_transition(acc, p, rho_exact):
+    """x_next = clamp(rint(H_in phi(H_out(rho (.) a)))) in exact rationals, from
+    the real ratio rho (not M): the integer path may differ only through the
+    M/2^n approximation of rho."""
+    a = acc + p.b_int
+    out = np.zeros(a.shape, dtype=np.int64)
+    flat = a.reshape(-1, a.shape[-1])
+    Hout = O.sylvester(p.hb_out) if p.hb_out else None
+    Hin = O.sylvester(p.hb_next) if p.hb_next else None
+    res = []
+    for row in flat:
+        t = [Fraction(float(r)) * int(v) for r, v in zip(rho_exact, row)]
+        if Hout is not None:
+            b = p.hb_out
+            t = [sum(int(Hout[j % b][i]) * t[(j // b) * b + i] for i in range(b)) for j in range(len(t))]
+        if p.act == "relu":
+            t = [max(v, Fraction(0)) for v in t]
+        if Hin is not None:
+            b = p.hb_next
+            t = [sum(int(Hin[j % b][i]) * t[(j // b) * b + i] for i in range(b)) for j in range(len(t))]
+        res.append([max(-127, min(127, O.round_half_even_fraction(v))) for v in t])
+    out[...] = np.array(res).reshape(a.shape)
+    return out
+
+
+@pytest.mark.parametrize("form,hb_next,act", [("DH", 0, "none"), ("DH", 16, "relu"), ("WH", 0, "relu"),
+                                              ("WH", 16, "relu")])
+def test_integer_transition_vs_exact_rational(form, hb_next, act):
+    c = 32
+    w = I.weights(c, 3, 3, 16, seed=60)
+    b = I.bias(c, seed=61)
+    x = I.activations_i8((1, 4, 4, 16), seed=62, s_in=0.05)
+    def prep(s_y):
+        return O.prepare_layer(w, b, form, 16 if form == "DH" else 0, 16 if form == "WH" else 0,
+                               s_x=0.05, s_y=s_y, act=act, hb_next=hb_next, out_f32=False, stride=1, pad=1)
+    p1 = prep(1.0)
+    acc = O.conv_codes(x, p1.w_int, 1, 1)
+    z = p1.rho * (acc + p1.b_int)                    # real-valued transition at s_y = 1
+    z = O.transform_real(z, p1.hb_out, normalize=False) if p1.hb_out else z
+    z = np.maximum(z, 0) if act == "relu" else z
+    z = O.transform_real(z, hb_next, normalize=False) if hb_next else z
+    p = prep(float(np.max(np.abs(z))) / 110.0)
+    got = O.epilogue_int(acc, p).astype(np.int64)
+    ref = _exact_transition(acc, p, p.rho)
+    d = np.abs(got - ref)
+    assert d.max() <= 1 and np.mean(d > 0) < 0.01
+    assert np.mean(np.abs(ref) == 127) < 0.5                      # not saturated everywhere
+
+
+@pytest.mark.parametrize("form", ["DH", "WH"])
+def test_quantized_layer_approximates_real_layer(form):
+    """End-to-end pin: dequantized integer output vs the fp64 real model."""
+    c_in, c_out, hb = 64, 64, 64
+    x_real = I.activations((1, 10, 10, c_in), seed=70).astype(np.float64)
+    w = I.weights(c_out, 3, 3, c_in, seed=71)
+    b = I.bias(c_out, seed=72)
+    y_ref = np.maximum(O.conv_real(x_real, w, b, 1, 1), 0)
+    s_x = O.symmetric_scale(O.transform_real(x_real, hb)) if form == "DH" else O.symmetric_scale(x_real)
+    s_y = O.symmetric_scale(y_ref)
+    p = O.prepare_layer(w, b, form, hb if form == "DH" else 0, hb if form == "WH" else 0, s_x, s_y,
+                        "relu", 0, False, 1, 1)
+    op = O.quantize_act_f16(x_real.astype(np.float16), hb if form == "DH" else 1, s_x)
+    y = O.conv_layer(op, p).astype(np.float64) * p.s_y
+    # WH keeps the outlier-heavy activations in the original domain (input
+    # SQNR alone is ~24.5 dB here); DH quantizes them in the Hadamard domain.
+    floor = 28.0 if form == "DH" else 20.0
+    assert O.sqnr_db(y_ref, y) > floor
+    pf = O.prepare_layer(w, b, form, hb if form == "DH" else 0, hb if form == "WH" else 0, s_x, s_y,
+                         "relu", 0, True, 1, 1)
+    yf = O.conv_layer(op, pf)
+    assert O.sqnr_db(y_ref, yf) > floor
+
+
+def test_chain_mixed_forms_tracks_real_model():
+    """A small DH/WH chain with fused and unfused transitions stays close to
+    the real-valued model (Table integer_transitions end to end)."""
+    from synth.configs import layer, plan_chain, ChainSpec
+    layers = (layer("a", 16, 64, 3, 1, 1, "WH", "relu", hb_out=64),
+              layer("b", 64, 64, 3, 2, 1, "DH", "relu", hb_in=64),
+              layer("c", 64, 128, 3, 1, 1, "WH", "relu", hb_out=128),
+              layer("d", 128, 32, 1, 1, 0, "DH", "none", hb_in=128))
+    ch = ChainSpec("t", layers, 1, 12, 12, "i8", 0.05, 80, 81)
+    plan = plan_chain(ch)
+    assert plan == [64, 0, 0, 0]                        # WH(64)->DH(64) fused; WH(128)->DH(128) not
+    x = I.activations_i8((1, 12, 12, 16), seed=80, s_in=0.05)
+    params = [(I.weights(L.c_out, L.k, L.k, L.c_in, 90 + i), I.bias(L.c_out, 95 + i)) for i, L in enumerate(layers)]
+    x_real = x.astype(np.float64) * float(np.float32(0.05))
+    scales = O.calibrate_chain(layers, params, x_real, plan)
+    preps = O.prepare_chain(layers, params, scales, plan)
+    outs = O.chain_forward(layers, preps, plan, x, "i8", 0.05)
+    ref = x_real
+    for L, (w, b) in zip(layers, params):
+        ref = O.conv_real(ref, w, b, L.stride, L.pad)
+        ref = np.maximum(ref, 0) if L.act == "relu" else ref
+    got = outs[-1].astype(np.float64) * preps[-1].s_y
+    assert O.sqnr_db(ref, got) > 15.0
+
+
+# ------------------------------------------------------- method diagnostics (T9)
+
+def test_hadamard_domain_improves_tensorwise_sqnr_and_kurtosis():
+    """Sec. transform-domain motivation: on outlier-heavy activations the
+    Hadamard domain has lower excess kurtosis and higher per-tensor INT8 SQNR."""
+    x = I.activations((1, 16, 16, 128), seed=0).astype(np.float64)
+    y = O.transform_real(x, 128)
+    qx = O.quantize_sym(x, O.symmetric_scale(x)) * O.symmetric_scale(x)
+    qy = O.quantize_sym(y, O.symmetric_scale(y)) * O.symmetric_scale(y)
+    assert O.sqnr_db(y, qy) > O.sqnr_db(x, qx)
+    assert O.excess_kurtosis(y) < O.excess_kurtosis(x)
+
+
+def test_range_expansion_indicator():
+    """Eq. hadamard_sensitivity: a nonnegative, nonzero-mean tensor (ReLU
+    output) expands under the transform; a zero-mean outlier tensor shrinks."""
+    rng = np.random.default_rng(1)
+    relu_like = np.maximum(rng.standard_normal((64, 64)) + 1.0, 0)
+    assert O.range_expands(relu_like, 64)
+    spiky = rng.standard_normal((64, 64)) * 0.1
+    spiky[:, 3] = 50.0 * np.sign(rng.standard_normal(64))
+    assert not O.range_expands(spiky, 64)
