@@ -1,0 +1,217 @@
+/*
+ * hatq.h - C ABI of the Hadamard-domain INT8 convolution library (libhatq.so).
+ *
+ * The operator is HaTQ's layer in integer-only form ("Hadamard-Domain Model
+ * Quantization for Learned Image Coding"): a convolution unfolded as the
+ * linear operator Y = X W^T (Eq. linear_operator) whose operands are quantized
+ * in a Hadamard basis, either double-Hadamard (DH: activations and weights
+ * transformed along C_in, Eq. double_hadamard_quantization) or weight-only
+ * (WH: weights transformed along C_out and the output basis restored after
+ * accumulation, Eq. weight_only_hadamard_quantization), with INT8 codes,
+ * int32 accumulation (Eq. integer_accumulation) and fixed-point
+ * requantization (Eqs. integer_fixed_point_scale, integer_hadamard_transition).
+ *
+ * Conventions shared by every entry point
+ *  - Layout: activations NHWC (C contiguous), weights OHWI, all C-contiguous.
+ *  - Ownership: the caller allocates and owns every buffer; no entry point
+ *    allocates device memory. Device pointers must be 16-byte aligned.
+ *  - An empty batch (n == 0) is a valid no-op; its pointers may be NULL.
+ *  - Streams: device work is enqueued on `stream` (a cudaStream_t; NULL is the
+ *    legacy default stream) and is asynchronous unless stated otherwise.
+ *  - Errors: argument, shape, alignment and overflow errors are returned
+ *    before anything is launched; a CUDA launch error returns HATQ_ERR_CUDA.
+ *    Kernels that wait on barriers wait a bounded time; an expired wait
+ *    records an error word that hatq_sync_status() reports as
+ *    HATQ_ERR_TIMEOUT. hatq_last_error() gives a message for the calling
+ *    thread's last failure.
+ *  - Codes are symmetric INT8 in [-127, 127] (Eq. symmetric_q with b = 8);
+ *    round() is round-half-to-even everywhere.
+ *  - Hadamard transforms are block-diagonal Sylvester transforms
+ *    I_{C/hb} (x) H_hb along the channel axis (Eq. supp_sylvester), hb a power
+ *    of two dividing the channel count; the unnormalized transform H~ uses
+ *    only additions and subtractions, its 1/sqrt(hb) is folded into scales.
+ */
+#ifndef HATQ_H
+#define HATQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *hatq_stream;   /* same type as cudaStream_t */
+
+typedef enum {
+    HATQ_OK = 0,
+    HATQ_ERR_INVALID_ARG = 1,   /* bad pointer, shape, alignment or value */
+    HATQ_ERR_UNSUPPORTED = 2,   /* valid by the paper but not implemented here */
+    HATQ_ERR_OVERFLOW = 3,      /* int32 accumulator or int64 requant bound violated */
+    HATQ_ERR_CUDA = 4,          /* a CUDA runtime/driver call failed */
+    HATQ_ERR_TIMEOUT = 5        /* a bounded device-side wait expired */
+} hatq_status;
+
+typedef enum { HATQ_DH = 0, HATQ_WH = 1 } hatq_form;
+typedef enum { HATQ_ACT_NONE = 0, HATQ_ACT_RELU = 1 } hatq_act;
+
+/* What a layer input holds (hatq_layer, hatq_quantize_act). */
+typedef enum {
+    HATQ_IN_OPERAND = 0,  /* INT8 codes already in this layer's operand basis and scale */
+    HATQ_IN_I8 = 1,       /* INT8 codes in the original basis at scale s_in */
+    HATQ_IN_F16 = 2       /* IEEE fp16 real values (FP16 entry) */
+} hatq_input_kind;
+
+/* One convolution (Eq. linear_operator with D = C_in Kh Kw). */
+typedef struct {
+    int c_in, c_out;      /* channels; c_out % 16 == 0 */
+    int kh, kw;           /* kernel size */
+    int stride, pad;      /* stride >= 1, symmetric zero padding */
+    int form;             /* hatq_form, from the static profile mask (Eq. layerwise_hadamard_selection) */
+    int hb_in;            /* DH: Hadamard block along c_in (16..256, power of two); 0 for WH */
+    int hb_out;           /* WH: Hadamard block along c_out (16..128); 0 for DH */
+} hatq_conv_desc;
+
+/*
+ * A prepared layer (Sec. deployment realization: transformed weights are
+ * input-independent and stored after offline transformation).
+ * The caller sets the six device pointers (sizes from hatq_prepared_sizes)
+ * before hatq_prepare_weights fills them; every other field is written by
+ * the library. opaque[] holds the library's tensor-memory-access descriptor
+ * of w_f16 and must not be modified.
+ */
+typedef struct {
+    hatq_conv_desc d;
+    int act;              /* hatq_act */
+    int hb_next;          /* block of the next layer's DH transform applied in this epilogue, 0 = none */
+    int out_f32;          /* 1: dequantized float32 output; 0: INT8 codes at s_y */
+    int shift;            /* shared right shift n (Eq. integer_fixed_point_scale) */
+    int k_pad;            /* packed reduction length = columns of w_i8 / w_f16 */
+    int gather;           /* 1: small-channel layer (c_in % 16 != 0), reduction packed densely */
+    float s_x;            /* scale of the INT8 operand this layer consumes */
+    float s_y;            /* scale of the INT8 codes it emits */
+    int8_t *w_i8;         /* [c_out][k_pad] weight codes w_int, K order (kh, kw, c_in) */
+    uint16_t *w_f16;      /* [c_out][k_pad] the same codes as IEEE fp16 (exact), tensor-core operand */
+    int32_t *b_int;       /* [c_out] bias codes, Eq. supp_bias_quantization */
+    int32_t *mult;        /* [c_out] multipliers M_c, Eq. integer_fixed_point_scale */
+    float *deq;           /* [c_out] s_x s_w,c / gamma_out (float32 output mode) */
+    float *s_w;           /* [c_out] per-output-channel weight scales */
+    uint64_t opaque[16];
+} hatq_prepared;
+
+/*
+ * Device buffer sizes of a prepared layer: w_elems = c_out * k_pad (elements
+ * of w_i8 and of w_f16), ch_elems = c_out (b_int, mult, deq, s_w).
+ * Returns HATQ_ERR_INVALID_ARG / HATQ_ERR_UNSUPPORTED for a bad descriptor.
+ */
+hatq_status hatq_prepared_sizes(const hatq_conv_desc *d, size_t *w_elems, size_t *ch_elems);
+
+/*
+ * Offline weight preparation (Eqs. double_hadamard_quantization,
+ * supp_padded_wh_parameters, supp_bias_quantization, integer_fixed_point_scale;
+ * Table integer_transitions).
+ *   w_ohwi  host float32 [c_out][kh][kw][c_in]; bias host float32 [c_out] or NULL.
+ *   s_x     scale of the INT8 operand the layer consumes (DH: in the input
+ *           Hadamard basis; WH: original basis).
+ *   s_y     scale of the INT8 codes the layer emits (ignored when out_f32).
+ *   act     activation phi applied in the epilogue (positively homogeneous).
+ *   hb_next block of the next layer's DH input transform to apply after phi
+ *           (DH-to-DH / WH-to-DH transitions), 0 for none.
+ *   out     caller-owned struct with its device pointers set.
+ * DH: W' = W (I (x) T_in) along c_in; WH: W_bar = T_out^T W along c_out and
+ * b_bar = b T_out. Per output channel s_w = max|W'|/127, w_int = round(W'/s_w),
+ * b_int = round(b_bar/(s_x s_w)), rho_c = s_x s_w,c / (gamma_out gamma_in s_y),
+ * M_c = round(rho_c 2^n) with the shared n chosen as the largest in [0, 62]
+ * such that all M_c < 2^31 and max_c M_c A_c g_out g_next < 2^62 (A_c the
+ * worst-case |accumulator|, g the unnormalized transform gains); fewer than
+ * 16 multiplier bits returns HATQ_ERR_OVERFLOW. Real arithmetic is fp64 in a
+ * fixed summation order. Synchronizes `stream` before returning.
+ */
+hatq_status hatq_prepare_weights(const hatq_conv_desc *d, const float *w_ohwi, const float *bias,
+                                 float s_x, float s_y, int act, int hb_next, int out_f32,
+                                 hatq_prepared *out, hatq_stream stream);
+
+/*
+ * The arithmetic of hatq_prepare_weights into caller-owned HOST buffers, with
+ * no device involved (for serializing prepared layers and for checking the
+ * offline step): w_i8 / w_f16 [c_out][k_pad], b_int / mult / deq / s_w
+ * [c_out], *shift = n. Same arguments, rules and errors as
+ * hatq_prepare_weights.
+ */
+hatq_status hatq_prepare_weights_host(const hatq_conv_desc *d, const float *w_ohwi, const float *bias,
+                                      float s_x, float s_y, int act, int hb_next, int out_f32,
+                                      int8_t *w_i8, uint16_t *w_f16, int32_t *b_int, int32_t *mult,
+                                      float *deq, float *s_w, int *shift);
+
+/*
+ * Online activation transform + quantization (the activation side of
+ * Eq. double_hadamard_quantization; Eq. symmetric_q; INT8 entry per
+ * Eq. supp_general_input_transition).
+ *   x       device NHWC, int8 codes at scale s_in (x_kind = HATQ_IN_I8) or
+ *           fp16 values (HATQ_IN_F16); n*h*w*c elements, c % 16 == 0.
+ *   hb      block of the unnormalized transform along c: 1 (no transform,
+ *           plain requantization) or a power of two in 2..256 dividing c.
+ *   s_out   > 0: static output scale; <= 0: dynamic per-tensor scale from the
+ *           transformed tensor's max-abs (two passes), written to *s_used.
+ *   y       device NHWC int8 codes of Q(x T) at scale s_out (or *s_used).
+ *   s_used  device float, required in dynamic mode, may be NULL otherwise.
+ *   workspace  device, >= 32 bytes, required in dynamic mode (reset each call).
+ * FP16 entry: y = clamp(round((H~ x) / (sqrt(hb) s_out))) with an fp32
+ * butterfly. INT8 entry: v = H~ x exactly in integers,
+ * y = clamp(round(M_q v / 2^n_q)) with M_q / 2^n_q ~ s_in / (sqrt(hb) s_out).
+ */
+hatq_status hatq_quantize_act(const void *x, int x_kind, float s_in, int n, int h, int w, int c,
+                              int hb, float s_out, int8_t *y, float *s_used, void *workspace,
+                              hatq_stream stream);
+
+/*
+ * Convolution on INT8 operands with the fused requantize epilogue
+ * (Eqs. integer_accumulation, integer_hadamard_transition):
+ *   a = sum_k x_int w_int + b_int                    (exact integer)
+ *   INT8 output:  y = clamp(round(H~_next phi(H~_out (M (.) a)) / 2^n))
+ *   float output: y = phi(H~_out (deq (.) a))        (float32, no rounding)
+ * where H~_out is applied for WH layers and H~_next when hb_next > 0.
+ *   x   device NHWC int8 [n][h][w][c_in], the layer's operand (basis and scale s_x).
+ *   y   device NHWC [n][ho][wo][c_out], int8 or float32 (L->out_f32),
+ *       ho = (h + 2 pad - kh) / stride + 1 (floor), likewise wo.
+ * The reduction runs on the tensor cores with the codes held exactly as fp16
+ * operands and fp32 partial sums that stay below 2^24 in magnitude, moved to
+ * int32 every 1024 reduction elements, so the accumulator is exact.
+ */
+hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prepared *L,
+                           void *y, hatq_stream stream);
+
+/*
+ * One layer in one call: the activation transform/quantize of
+ * hatq_quantize_act when x is not yet the layer's operand (DH: transform with
+ * hb_in; WH: requantize to s_x when s_in != s_x), then hatq_conv2d_i8.
+ *   x_kind   hatq_input_kind of x; s_in its scale for HATQ_IN_I8.
+ *   scratch  device buffer for the INT8 operand when one is produced,
+ *            >= n*h*w*c_in bytes (may be NULL when none is needed).
+ */
+hatq_status hatq_layer(const void *x, int x_kind, float s_in, int n, int h, int w,
+                       const hatq_prepared *L, void *y, void *scratch, size_t scratch_bytes,
+                       hatq_stream stream);
+
+/* Number of kernel launches hatq_layer / hatq_conv2d_i8 make for these
+ * arguments (for launch accounting), or -1 for invalid arguments. */
+int hatq_layer_launches(int x_kind, float s_in, const hatq_prepared *L);
+
+/* Message describing the calling thread's most recent failure ("" if none). */
+const char *hatq_last_error(void);
+
+/* Synchronizes `stream`, then reads and clears the device error word of the
+ * current device: HATQ_ERR_TIMEOUT if a bounded wait expired, HATQ_ERR_CUDA
+ * on an asynchronous CUDA error, HATQ_OK otherwise. The error word is sticky:
+ * while it is set, convolution blocks that have not started return at once,
+ * so work enqueued after a failure produces no output until it is read. */
+hatq_status hatq_sync_status(hatq_stream stream);
+
+/* Library version, (major << 16) | minor. */
+int hatq_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HATQ_H */

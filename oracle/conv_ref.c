@@ -15,8 +15,33 @@
  * wt : OHWI int8, shape [co][kh][kw][c]
  * acc: int64, shape [n][ho1-ho0][wo1-wo0][co] (an output window; the full
  *      output is ho0 = wo0 = 0, ho1 = Ho, wo1 = Wo)
+ *
+ * When built with OpenMP the output rows are shared among threads; every sum
+ * is an exact integer, so the result does not depend on the thread count.
  */
 #include <stdint.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* Threads the direct convolution may use (1 without OpenMP). */
+int oracle_max_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+void oracle_set_threads(int t)
+{
+#ifdef _OPENMP
+    if (t > 0) omp_set_num_threads(t);
+#else
+    (void)t;
+#endif
+}
 
 void oracle_conv2d_codes(const int8_t *x, int64_t n, int64_t h, int64_t w, int64_t c,
                          const int8_t *wt, int64_t co, int64_t kh, int64_t kw,
@@ -25,6 +50,7 @@ void oracle_conv2d_codes(const int8_t *x, int64_t n, int64_t h, int64_t w, int64
                          int64_t *acc)
 {
     int64_t nho = ho1 - ho0, nwo = wo1 - wo0;
+#pragma omp parallel for collapse(2) schedule(dynamic, 1)
     for (int64_t b = 0; b < n; ++b)
         for (int64_t oy = ho0; oy < ho1; ++oy)
             for (int64_t ox = wo0; ox < wo1; ++ox) {
@@ -55,6 +81,7 @@ void oracle_conv2d_codes_at(const int8_t *x, int64_t n, int64_t h, int64_t w, in
                             const int64_t *pix, int64_t npix, int64_t *acc)
 {
     (void)n;
+#pragma omp parallel for schedule(dynamic, 16)
     for (int64_t i = 0; i < npix; ++i) {
         int64_t b = pix[3 * i], oy = pix[3 * i + 1], ox = pix[3 * i + 2];
         for (int64_t o = 0; o < co; ++o) {

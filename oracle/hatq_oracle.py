@@ -312,8 +312,9 @@ def build_lib(force: bool = False) -> str:
     if force or not os.path.exists(so) or os.path.getmtime(so) < os.path.getmtime(src):
         os.makedirs(out_dir, exist_ok=True)
         tmp = so + f".tmp{os.getpid()}"
-        subprocess.check_call(["gcc", "-O2", "-fPIC", "-shared", "-ffp-contract=off",
-                               "-o", tmp, src])
+        base = ["gcc", "-O2", "-fPIC", "-shared", "-ffp-contract=off", "-o", tmp, src]
+        if subprocess.run(base[:1] + ["-fopenmp"] + base[1:], capture_output=True).returncode != 0:
+            subprocess.check_call(base)
         os.replace(tmp, so)
     return so
 
@@ -328,8 +329,19 @@ def _lib():
                                             i64, i64, i64, i64, p]
         lib.oracle_conv2d_codes_at.argtypes = [p, i64, i64, i64, i64, p, i64, i64, i64, i64, i64,
                                                p, i64, p]
+        lib.oracle_max_threads.restype = ctypes.c_int
+        lib.oracle_set_threads.argtypes = [ctypes.c_int]
         _LIB = lib
     return _LIB
+
+
+def max_threads() -> int:
+    """Threads the direct convolution uses (OpenMP; 1 without it)."""
+    return int(_lib().oracle_max_threads())
+
+
+def set_threads(t: int) -> None:
+    _lib().oracle_set_threads(int(t))
 
 
 def out_hw(h, w, k, stride, pad):

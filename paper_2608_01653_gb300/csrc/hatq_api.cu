@@ -1,0 +1,533 @@
+// Host side of libhatq: the C ABI declared in include/hatq.h.
+//
+// Offline weight preparation follows Eqs. (double_hadamard_quantization,
+// supp_padded_wh_parameters, supp_bias_quantization, integer_fixed_point_scale)
+// and Table integer_transitions of the HaTQ paper; every real-valued step is
+// fp64 with a fixed summation order (for output j of a block transform:
+// acc = 0; acc += +-x_i for i = 0..hb-1; then acc / sqrt(hb)), so the result
+// does not depend on the compiler or the machine.
+#include <cuda_fp16.h>
+
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "hatq.h"
+#include "hatq_internal.h"
+
+namespace {
+
+thread_local std::string g_msg;
+
+hatq_status fail(hatq_status st, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_msg = buf;
+    return st;
+}
+
+hatq_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(HATQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Device error word written by kernels (bounded-wait expiry, bound checks).
+__device__ int g_err_word;
+
+int *err_word() {
+    static int *ptrs[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    if (!ptrs[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_err_word) != cudaSuccess) return nullptr;
+        ptrs[dev] = static_cast<int *>(p);
+    }
+    return ptrs[dev];
+}
+
+bool pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+int sylvester_sign(int i, int j) { return (__builtin_popcount((unsigned)(i & j)) & 1) ? -1 : 1; }
+
+// ------------------------------------------------------------ tensor maps
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        cudaDriverEntryPointQueryResult q;
+        void *p = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+// ------------------------------------------------------------ geometry
+
+struct Geometry {
+    int gather, cin_pad, k_pad, n_t, G;
+};
+
+hatq_status check_desc(const hatq_conv_desc *d) {
+    if (!d) return fail(HATQ_ERR_INVALID_ARG, "null descriptor");
+    if (d->c_in < 1 || d->c_out < 32 || d->c_out % 32)
+        return fail(HATQ_ERR_UNSUPPORTED, "c_in >= 1 and c_out a positive multiple of 32 are required (c_in=%d c_out=%d)",
+                    d->c_in, d->c_out);
+    if (d->kh < 1 || d->kw < 1 || d->kh > 16 || d->kw > 16) return fail(HATQ_ERR_INVALID_ARG, "kernel size out of range");
+    if (d->stride < 1 || d->stride > 2) return fail(HATQ_ERR_UNSUPPORTED, "stride must be 1 or 2");
+    if (d->pad < 0 || d->pad >= d->kh || d->pad >= d->kw) return fail(HATQ_ERR_INVALID_ARG, "padding out of range");
+    if (d->form == HATQ_DH) {
+        if (d->hb_out != 0) return fail(HATQ_ERR_INVALID_ARG, "a DH layer has no output block");
+        if (!pow2(d->hb_in) || d->hb_in < 2 || d->hb_in > 256 || d->c_in % d->hb_in)
+            return fail(HATQ_ERR_INVALID_ARG, "DH block hb_in must be a power of two in 2..256 dividing c_in");
+        if (d->c_in % 16) return fail(HATQ_ERR_UNSUPPORTED, "a DH layer needs c_in % 16 == 0");
+    } else if (d->form == HATQ_WH) {
+        if (d->hb_in != 0) return fail(HATQ_ERR_INVALID_ARG, "a WH layer has no input block");
+        if (!pow2(d->hb_out) || d->hb_out < 2 || d->hb_out > 128 || d->c_out % d->hb_out)
+            return fail(HATQ_ERR_INVALID_ARG, "WH block hb_out must be a power of two in 2..128 dividing c_out");
+    } else {
+        return fail(HATQ_ERR_INVALID_ARG, "unknown form %d", d->form);
+    }
+    return HATQ_OK;
+}
+
+bool fusable(int hb_out, int hb_next) {
+    if (hb_out == 0 || hb_next == 0) return (hb_out > hb_next ? hb_out : hb_next) <= 128;
+    return hb_out <= 64 && hb_next <= 64;
+}
+
+hatq_status geometry(const hatq_conv_desc *d, int hb_next, Geometry *g) {
+    g->gather = d->c_in % 16 != 0;
+    g->cin_pad = (d->c_in + 63) / 64 * 64;
+    g->k_pad = g->gather ? (d->kh * d->kw * d->c_in + 63) / 64 * 64 : d->kh * d->kw * g->cin_pad;
+    const int hb_out = d->form == HATQ_WH ? d->hb_out : 0;
+    int G = 32;
+    if (hb_out > G) G = hb_out;
+    if (hb_next > G) G = hb_next;
+    g->G = G;
+    g->n_t = 0;
+    for (int nt = 256; nt >= G; nt -= 16)
+        if (nt % G == 0 && d->c_out % nt == 0) { g->n_t = nt; break; }
+    if (!g->n_t) return fail(HATQ_ERR_UNSUPPORTED, "no output-channel tile for c_out=%d with group %d", d->c_out, G);
+    return HATQ_OK;
+}
+
+// ------------------------------------------------------------ fixed point (M, n)
+
+// Largest n in [0, 62] with all M_c = rint(rho_c 2^n) < 2^31 and
+// max_c(M_c A_c) * gain < 2^62; fewer than 16 bits in max M is an error.
+hatq_status fixed_point(const std::vector<double> &rho, const std::vector<long long> &abound, long long gain,
+                        std::vector<int32_t> &M, int &shift) {
+    for (double r : rho)
+        if (!(r >= 0.0) || !std::isfinite(r)) return fail(HATQ_ERR_INVALID_ARG, "scale ratio must be finite and >= 0");
+    M.assign(rho.size(), 0);
+    for (int n = 62; n >= 0; --n) {
+        bool ok = true;
+        long long mmax = 0;
+        unsigned __int128 worst = 0;
+        std::vector<long long> m(rho.size());
+        for (size_t c = 0; c < rho.size() && ok; ++c) {
+            const double v = std::nearbyint(std::ldexp(rho[c], n));
+            if (v >= 2147483648.0) { ok = false; break; }
+            m[c] = (long long)v;
+            if (m[c] > mmax) mmax = m[c];
+            const unsigned __int128 w = (unsigned __int128)m[c] * (unsigned __int128)abound[c];
+            if (w > worst) worst = w;
+        }
+        if (!ok) continue;
+        if (worst * (unsigned __int128)gain >= ((unsigned __int128)1 << 62)) continue;
+        if (mmax < (1LL << 15)) return fail(HATQ_ERR_OVERFLOW, "fewer than 16 bits of multiplier precision");
+        for (size_t c = 0; c < rho.size(); ++c) M[c] = (int32_t)m[c];
+        shift = n;
+        return HATQ_OK;
+    }
+    return fail(HATQ_ERR_OVERFLOW, "no shift satisfies the multiplier and overflow bounds");
+}
+
+// Normalized transform of one contiguous hb-block x into y (element j at
+// y[j * ystep]) in the fixed order: acc = 0; acc += +-x_i, i = 0..hb-1; acc / sqrt(hb).
+void block_transform(const double *x, double *y, int hb, long long ystep) {
+    const double sq = std::sqrt((double)hb);
+    for (int j = 0; j < hb; ++j) {
+        double acc = 0.0;
+        for (int i = 0; i < hb; ++i) acc += sylvester_sign(i, j) > 0 ? x[i] : -x[i];
+        y[j * ystep] = acc / sq;
+    }
+}
+
+uint16_t f16_bits(int v) {
+    const __half h = __float2half_rn((float)v);
+    uint16_t b;
+    std::memcpy(&b, &h, 2);
+    return b;
+}
+
+void choose_mtile(int ho, int wo, int stride, int *tw, int *th) {
+    long long best = -1;
+    for (int t = 128; t >= 8; t >>= 1) {
+        const int h = 128 / t;
+        if (t * stride > 256 || h * stride > 256) continue;
+        const long long area = (long long)((wo + t - 1) / t) * t * (long long)((ho + h - 1) / h) * h;
+        if (best < 0 || area < best) { best = area; *tw = t; *th = h; }
+    }
+}
+
+hatq_status validate_prepare(const hatq_conv_desc *d, const float *w_ohwi, float s_x, float s_y, int act,
+                                    int hb_next, int out_f32, Geometry *g) {
+    hatq_status st = check_desc(d);
+    if (st != HATQ_OK) return st;
+    if (!w_ohwi) return fail(HATQ_ERR_INVALID_ARG, "null weights");
+    if (!(s_x > 0.f) || !std::isfinite(s_x)) return fail(HATQ_ERR_INVALID_ARG, "s_x must be positive");
+    if (!out_f32 && (!(s_y > 0.f) || !std::isfinite(s_y))) return fail(HATQ_ERR_INVALID_ARG, "s_y must be positive");
+    if (act != HATQ_ACT_NONE && act != HATQ_ACT_RELU) return fail(HATQ_ERR_INVALID_ARG, "unknown activation");
+    if (hb_next != 0 && (!pow2(hb_next) || hb_next < 2 || hb_next > 128 || d->c_out % hb_next))
+        return fail(HATQ_ERR_INVALID_ARG, "hb_next must be 0 or a power of two in 2..128 dividing c_out");
+    if (out_f32 && hb_next) return fail(HATQ_ERR_INVALID_ARG, "a float32 output has no next-layer transform");
+    const int hb_out = d->form == HATQ_WH ? d->hb_out : 0;
+    if (!fusable(hb_out, hb_next))
+        return fail(HATQ_ERR_UNSUPPORTED, "output block %d and next-layer block %d cannot both be applied in the epilogue",
+                    hb_out, hb_next);
+    return geometry(d, hb_next, g);
+}
+
+}  // namespace
+
+extern "C" {
+
+int hatq_version(void) { return (0 << 16) | 1; }
+
+const char *hatq_last_error(void) { return g_msg.c_str(); }
+
+hatq_status hatq_prepared_sizes(const hatq_conv_desc *d, size_t *w_elems, size_t *ch_elems) {
+    hatq_status st = check_desc(d);
+    if (st != HATQ_OK) return st;
+    Geometry g;
+    if ((st = geometry(d, 0, &g)) != HATQ_OK) return st;
+    if (w_elems) *w_elems = (size_t)d->c_out * g.k_pad;
+    if (ch_elems) *ch_elems = (size_t)d->c_out;
+    return HATQ_OK;
+}
+
+hatq_status hatq_prepare_weights_host(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                      float s_y, int act, int hb_next, int out_f32, int8_t *w_i8_out,
+                                      uint16_t *w_f16_out, int32_t *b_int_out, int32_t *mult_out, float *deq_out,
+                                      float *s_w_out, int *shift_out) {
+    Geometry g;
+    hatq_status st = validate_prepare(d, w_ohwi, s_x, s_y, act, hb_next, out_f32, &g);
+    if (st != HATQ_OK) return st;
+    if (!w_i8_out || !w_f16_out || !b_int_out || !mult_out || !deq_out || !s_w_out || !shift_out)
+        return fail(HATQ_ERR_INVALID_ARG, "null output buffer");
+    const int co = d->c_out, ci = d->c_in, taps = d->kh * d->kw;
+    const long long per_o = (long long)taps * ci;
+    // 1. Hadamard-domain weights and bias (fp64)
+    std::vector<double> wp((size_t)co * per_o);
+    std::vector<double> bbar(co, 0.0);
+    if (bias)
+        for (int o = 0; o < co; ++o) bbar[o] = (double)bias[o];
+    if (d->form == HATQ_DH) {
+        const int hb = d->hb_in;
+        for (long long r = 0; r < (long long)co * taps; ++r)
+            for (int blk = 0; blk < ci / hb; ++blk) {
+                double x[256];
+                for (int i = 0; i < hb; ++i) x[i] = (double)w_ohwi[r * ci + blk * hb + i];
+                block_transform(x, &wp[r * ci + blk * hb], hb, 1);
+            }
+    } else {
+        const int hb = d->hb_out;
+        for (long long t = 0; t < per_o; ++t)            // (tap, ci) column, transform along c_out
+            for (int blk = 0; blk < co / hb; ++blk) {
+                double x[128];
+                for (int i = 0; i < hb; ++i) x[i] = (double)w_ohwi[(long long)(blk * hb + i) * per_o + t];
+                block_transform(x, &wp[(long long)(blk * hb) * per_o + t], hb, per_o);
+            }
+        std::vector<double> b0 = bbar;
+        for (int blk = 0; blk < co / hb; ++blk) block_transform(&b0[blk * hb], &bbar[blk * hb], hb, 1);
+    }
+    // 2. channel-wise symmetric weight quantization, bias codes, bounds
+    std::vector<double> s_a(co), rho(co);
+    std::vector<long long> abound(co);
+    std::memset(w_i8_out, 0, (size_t)co * g.k_pad);
+    for (size_t k = 0; k < (size_t)co * g.k_pad; ++k) w_f16_out[k] = f16_bits(0);
+    const double sx = (double)s_x, sy = (double)s_y;
+    for (int o = 0; o < co; ++o) {
+        const double *row = &wp[(size_t)o * per_o];
+        double m = 0.0;
+        for (long long k = 0; k < per_o; ++k) m = std::fmax(m, std::fabs(row[k]));
+        const double sw = m > 0.0 ? m / 127.0 : 1.0;
+        long long sum_abs = 0;
+        for (int tap = 0; tap < taps; ++tap)
+            for (int c = 0; c < ci; ++c) {
+                double q = std::nearbyint(row[(long long)tap * ci + c] / sw);
+                q = q < -127.0 ? -127.0 : (q > 127.0 ? 127.0 : q);
+                const int qi = (int)q;
+                sum_abs += qi < 0 ? -qi : qi;
+                const long long k = g.gather ? (long long)tap * ci + c : (long long)tap * g.cin_pad + c;
+                w_i8_out[(size_t)o * g.k_pad + k] = (int8_t)qi;
+                w_f16_out[(size_t)o * g.k_pad + k] = f16_bits(qi);
+            }
+        s_a[o] = sx * sw;
+        const double bq = std::nearbyint(bbar[o] / s_a[o]);
+        if (!(std::fabs(bq) < 1073741824.0)) return fail(HATQ_ERR_OVERFLOW, "bias code of channel %d out of range", o);
+        b_int_out[o] = (int32_t)bq;
+        abound[o] = 127LL * sum_abs + (long long)std::llabs((long long)b_int_out[o]);
+        if (abound[o] >= (1LL << 31)) return fail(HATQ_ERR_OVERFLOW, "int32 accumulator bound exceeded in channel %d", o);
+        s_w_out[o] = (float)sw;
+    }
+    // 3. requantization (Eq. integer_fixed_point_scale; gammas of Table integer_transitions)
+    const double g_out = d->form == HATQ_WH ? std::sqrt((double)d->hb_out) : 1.0;
+    const double g_in = hb_next ? std::sqrt((double)hb_next) : 1.0;
+    for (int o = 0; o < co; ++o) deq_out[o] = (float)(s_a[o] / g_out);
+    *shift_out = 0;
+    if (out_f32) {
+        for (int o = 0; o < co; ++o) mult_out[o] = 0;
+        return HATQ_OK;
+    }
+    const double alpha = g_out * g_in;
+    for (int o = 0; o < co; ++o) rho[o] = s_a[o] / (alpha * sy);
+    const long long gain = (long long)(d->form == HATQ_WH ? d->hb_out : 1) * (hb_next ? hb_next : 1);
+    std::vector<int32_t> mult;
+    int shift = 0;
+    if ((st = fixed_point(rho, abound, gain, mult, shift)) != HATQ_OK) return st;
+    for (int o = 0; o < co; ++o) mult_out[o] = mult[o];
+    *shift_out = shift;
+    return HATQ_OK;
+}
+
+hatq_status hatq_prepare_weights(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                 float s_y, int act, int hb_next, int out_f32, hatq_prepared *out,
+                                 hatq_stream stream) {
+    Geometry g;
+    hatq_status st = validate_prepare(d, w_ohwi, s_x, s_y, act, hb_next, out_f32, &g);
+    if (st != HATQ_OK) return st;
+    if (!out) return fail(HATQ_ERR_INVALID_ARG, "null output struct");
+    if (!out->w_i8 || !out->w_f16 || !out->b_int || !out->mult || !out->deq || !out->s_w)
+        return fail(HATQ_ERR_INVALID_ARG, "prepared-layer device buffers must be set before preparation");
+    if (!aligned16(out->w_i8) || !aligned16(out->w_f16) || !aligned16(out->b_int) || !aligned16(out->mult) ||
+        !aligned16(out->deq) || !aligned16(out->s_w))
+        return fail(HATQ_ERR_INVALID_ARG, "prepared-layer device buffers must be 16-byte aligned");
+    const int co = d->c_out;
+    std::vector<int8_t> w_i8((size_t)co * g.k_pad);
+    std::vector<uint16_t> w_f16((size_t)co * g.k_pad);
+    std::vector<int32_t> b_int(co), mult(co);
+    std::vector<float> deq(co), s_w(co);
+    int shift = 0;
+    st = hatq_prepare_weights_host(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, w_i8.data(), w_f16.data(),
+                                   b_int.data(), mult.data(), deq.data(), s_w.data(), &shift);
+    if (st != HATQ_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    if ((e = cudaMemcpyAsync(out->w_i8, w_i8.data(), w_i8.size(), cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->w_f16, w_f16.data(), w_f16.size() * 2, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->b_int, b_int.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->mult, mult.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->deq, deq.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->s_w, s_w.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return cuda_fail(e, "upload of prepared weights");
+    if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return cuda_fail(e, "upload of prepared weights");
+    // weight tensor map: [c_out][k_pad] fp16, 64 x n_t box, 128-byte swizzle
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return fail(HATQ_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    CUtensorMap tm;
+    const cuuint64_t dims[2] = {(cuuint64_t)g.k_pad, (cuuint64_t)co};
+    const cuuint64_t strides[1] = {(cuuint64_t)g.k_pad * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)g.n_t};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(&tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, out->w_f16, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "weight tensor map encoding failed (%d)", (int)r);
+    static_assert(sizeof(CUtensorMap) <= sizeof(out->opaque), "opaque area too small");
+    std::memcpy(out->opaque, &tm, sizeof tm);
+
+    out->d = *d;
+    out->act = act;
+    out->hb_next = hb_next;
+    out->out_f32 = out_f32 ? 1 : 0;
+    out->shift = shift;
+    out->k_pad = g.k_pad;
+    out->gather = g.gather;
+    out->s_x = s_x;
+    out->s_y = out_f32 ? 0.f : s_y;
+    return HATQ_OK;
+}
+
+hatq_status hatq_quantize_act(const void *x, int x_kind, float s_in, int n, int h, int w, int c, int hb, float s_out,
+                              int8_t *y, float *s_used, void *workspace, hatq_stream stream) {
+    if (n == 0 && h >= 0 && w >= 0 && c >= 0) return HATQ_OK;        // empty batch: nothing to do
+    if (!x || !y) return fail(HATQ_ERR_INVALID_ARG, "null input or output");
+    if (!aligned16(x) || !aligned16(y)) return fail(HATQ_ERR_INVALID_ARG, "input and output must be 16-byte aligned");
+    if (x_kind != HATQ_IN_I8 && x_kind != HATQ_IN_F16) return fail(HATQ_ERR_INVALID_ARG, "x_kind must be I8 or F16");
+    if (n < 0 || h < 0 || w < 0 || c < 16 || c % 16) return fail(HATQ_ERR_INVALID_ARG, "shape must be n,h,w >= 0, c % 16 == 0");
+    if (!pow2(hb) || hb > 256 || c % hb) return fail(HATQ_ERR_INVALID_ARG, "hb must be a power of two <= 256 dividing c");
+    const bool dynamic = !(s_out > 0.f);
+    if (x_kind == HATQ_IN_I8 && !(s_in > 0.f)) return fail(HATQ_ERR_INVALID_ARG, "s_in must be positive");
+    if (dynamic && (!s_used || !workspace)) return fail(HATQ_ERR_INVALID_ARG, "dynamic mode needs s_used and workspace");
+    if (dynamic && !aligned16(workspace)) return fail(HATQ_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+    const long long total = (long long)n * h * w * c;
+    hatq::ActQuantArgs a{};
+    a.x = x;
+    a.y = y;
+    a.total = total;
+    a.hb = hb;
+    a.f16 = x_kind == HATQ_IN_F16;
+    a.err = err_word();
+    if (!a.err) return fail(HATQ_ERR_CUDA, "no CUDA device");
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (total == 0) return HATQ_OK;
+    cudaError_t e;
+    if (dynamic) {
+        a.dyn = static_cast<hatq::DynParams *>(workspace);
+        e = hatq::launch_act_dynamic(a, s_in, s_used, s);
+    } else {
+        if (a.f16) {
+            a.inv = (float)(1.0 / (std::sqrt((double)hb) * (double)s_out));
+        } else {
+            const double rho = (double)s_in / (std::sqrt((double)hb) * (double)s_out);
+            std::vector<int32_t> M;
+            int shift = 0;
+            hatq_status st = fixed_point({rho}, {127LL * hb}, 1, M, shift);
+            if (st != HATQ_OK) return st;
+            a.mult = M[0];
+            a.shift = shift;
+        }
+        e = hatq::launch_act_quant(a, s);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "activation quantization launch");
+    return HATQ_OK;
+}
+
+hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prepared *L, void *y, hatq_stream stream) {
+    if (!L) return fail(HATQ_ERR_INVALID_ARG, "null layer");
+    if (n == 0 && h >= 1 && w >= 1) return HATQ_OK;                    // empty batch: nothing to do
+    if (!x || !y) return fail(HATQ_ERR_INVALID_ARG, "null argument");
+    if (!aligned16(x) || !aligned16(y)) return fail(HATQ_ERR_INVALID_ARG, "input and output must be 16-byte aligned");
+    const hatq_conv_desc *d = &L->d;
+    hatq_status st = check_desc(d);
+    if (st != HATQ_OK) return st;
+    if (n < 0 || h < 1 || w < 1) return fail(HATQ_ERR_INVALID_ARG, "bad input shape");
+    const int ho = (h + 2 * d->pad - d->kh) / d->stride + 1;
+    const int wo = (w + 2 * d->pad - d->kw) / d->stride + 1;
+    if (h + 2 * d->pad < d->kh || w + 2 * d->pad < d->kw || ho < 1 || wo < 1)
+        return fail(HATQ_ERR_INVALID_ARG, "input smaller than the kernel");
+    if ((long long)n * h * w * d->c_in >= (1LL << 40)) return fail(HATQ_ERR_UNSUPPORTED, "input too large");
+    if (n == 0) return HATQ_OK;
+    Geometry g;
+    if ((st = geometry(d, L->hb_next, &g)) != HATQ_OK) return st;
+    if (g.k_pad != L->k_pad || g.gather != L->gather) return fail(HATQ_ERR_INVALID_ARG, "prepared layer is inconsistent");
+    if ((long long)n * ((ho + 0) * (long long)wo) > (1LL << 31)) return fail(HATQ_ERR_UNSUPPORTED, "too many output pixels");
+
+    hatq::ConvArgs a{};
+    a.n = n; a.h = h; a.w = w; a.c = d->c_in;
+    a.ho = ho; a.wo = wo; a.co = d->c_out;
+    a.kh = d->kh; a.kw = d->kw; a.stride = d->stride; a.pad = d->pad;
+    choose_mtile(ho, wo, d->stride, &a.tw, &a.th);
+    a.tiles_w = (wo + a.tw - 1) / a.tw;
+    a.tiles_h = (ho + a.th - 1) / a.th;
+    if ((long long)n * a.tiles_w * a.tiles_h >= (1LL << 31)) return fail(HATQ_ERR_UNSUPPORTED, "grid too large");
+    a.n_t = g.n_t;
+    a.num_kb = g.k_pad / 64;
+    a.cin_kb = g.cin_pad / 64;
+    a.gather = g.gather;
+    a.chunk_kb = 16;
+    a.b_bytes = a.n_t * 128;
+    a.raw_bytes = g.gather ? 0 : 8192;
+    a.stage_bytes = 16384 + a.b_bytes + a.raw_bytes;
+    const int smem_cap = 227 * 1024 - 1024 - 256;
+    a.stages = smem_cap / a.stage_bytes;
+    if (a.stages > 8) a.stages = 8;
+    if (a.stages < 2) return fail(HATQ_ERR_UNSUPPORTED, "tile does not fit in shared memory");
+    int pc = 32;
+    while (pc < a.n_t) pc <<= 1;
+    a.part_col = pc;
+    a.tmem_cols = a.num_kb > a.chunk_kb ? 2 * pc : pc;
+    a.x = x;
+    a.b_int = L->b_int;
+    a.mult = L->mult;
+    a.deq = L->deq;
+    a.shift = L->shift;
+    a.hb_out = d->form == HATQ_WH ? d->hb_out : 0;
+    a.hb_next = L->hb_next;
+    a.act = L->act;
+    a.out_f32 = L->out_f32;
+    a.y = y;
+    a.err = err_word();
+    if (!a.err) return fail(HATQ_ERR_CUDA, "no CUDA device");
+    const int smem_bytes = a.stages * a.stage_bytes + 1024 + 8 * (3 * a.stages + 3) + 16;
+
+    CUtensorMap tmB, tmA;
+    std::memcpy(&tmB, L->opaque, sizeof tmB);
+    if (!g.gather) {
+        EncodeTiledFn enc = encode_fn();
+        if (!enc) return fail(HATQ_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+        const cuuint64_t dims[4] = {(cuuint64_t)d->c_in, (cuuint64_t)w, (cuuint64_t)h, (cuuint64_t)n};
+        const cuuint64_t strides[3] = {(cuuint64_t)d->c_in, (cuuint64_t)w * d->c_in, (cuuint64_t)h * w * d->c_in};
+        const cuuint32_t box[4] = {64, (cuuint32_t)(a.tw * d->stride), (cuuint32_t)(a.th * d->stride), 1};
+        const cuuint32_t estr[4] = {1, (cuuint32_t)d->stride, (cuuint32_t)d->stride, 1};
+        CUresult r = enc(&tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<int8_t *>(x), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "activation tensor map encoding failed (%d)", (int)r);
+    } else {
+        tmA = tmB;
+    }
+    cudaError_t e = hatq::launch_conv(tmA, tmB, a, smem_bytes, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "convolution launch");
+    return HATQ_OK;
+}
+
+int hatq_layer_launches(int x_kind, float s_in, const hatq_prepared *L) {
+    if (!L) return -1;
+    if (x_kind == HATQ_IN_OPERAND) return 1;
+    if (x_kind == HATQ_IN_I8) return (L->d.form == HATQ_WH && s_in == L->s_x) ? 1 : 2;
+    if (x_kind == HATQ_IN_F16) return 2;
+    return -1;
+}
+
+hatq_status hatq_layer(const void *x, int x_kind, float s_in, int n, int h, int w, const hatq_prepared *L, void *y,
+                       void *scratch, size_t scratch_bytes, hatq_stream stream) {
+    if (!L) return fail(HATQ_ERR_INVALID_ARG, "null layer");
+    if (n == 0 && h >= 1 && w >= 1) return HATQ_OK;                    // empty batch: nothing to do
+    if (!x || !y) return fail(HATQ_ERR_INVALID_ARG, "null argument");
+    const hatq_conv_desc *d = &L->d;
+    if (x_kind == HATQ_IN_OPERAND || (x_kind == HATQ_IN_I8 && d->form == HATQ_WH && s_in == L->s_x))
+        return hatq_conv2d_i8(static_cast<const int8_t *>(x), n, h, w, L, y, stream);
+    if (x_kind != HATQ_IN_I8 && x_kind != HATQ_IN_F16) return fail(HATQ_ERR_INVALID_ARG, "unknown input kind %d", x_kind);
+    const size_t need = (size_t)n * h * w * d->c_in;
+    if (!scratch || scratch_bytes < need) return fail(HATQ_ERR_INVALID_ARG, "scratch must hold %zu bytes", need);
+    if (d->c_in % 16) return fail(HATQ_ERR_UNSUPPORTED, "an input transform needs c_in % 16 == 0");
+    const int hb = d->form == HATQ_DH ? d->hb_in : 1;
+    hatq_status st = hatq_quantize_act(x, x_kind, s_in, n, h, w, d->c_in, hb, L->s_x, static_cast<int8_t *>(scratch),
+                                       nullptr, nullptr, stream);
+    if (st != HATQ_OK) return st;
+    return hatq_conv2d_i8(static_cast<const int8_t *>(scratch), n, h, w, L, y, stream);
+}
+
+hatq_status hatq_sync_status(hatq_stream stream) {
+    cudaError_t e = cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronization");
+    int *p = err_word();
+    if (!p) return fail(HATQ_ERR_CUDA, "no CUDA device");
+    int v = 0;
+    if ((e = cudaMemcpy(&v, p, sizeof v, cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(e, "error word read");
+    if (v != 0) {
+        const int zero = 0;
+        cudaMemcpy(p, &zero, sizeof zero, cudaMemcpyHostToDevice);
+        if (v == hatq::kErrWaitTimeout) return fail(HATQ_ERR_TIMEOUT, "a device-side bounded wait expired");
+        return fail(HATQ_ERR_OVERFLOW, "a device-side bound check failed (code %d)", v);
+    }
+    return HATQ_OK;
+}
+
+}  // extern "C"

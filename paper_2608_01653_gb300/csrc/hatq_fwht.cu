@@ -1,0 +1,307 @@
+// Online activation transform + INT8 quantization (the activation side of
+// HaTQ's double-Hadamard operator, Eq. double_hadamard_quantization, with the
+// butterfly evaluation of the Sylvester transform, Eq. supp_sylvester, and
+// the normalization folded into the quantization scale, as the deployment
+// realization of the supplementary material describes).
+//
+// Memory-bound: every element is read once and written once. A warp owns a
+// contiguous 512-element span of the flattened NHWC tensor (16 elements per
+// lane, one 16-byte load for INT8, two for FP16), so any Hadamard block
+// (hb <= 256, hb | C, 16 | C) lies inside one warp: the first log2(min(hb,16))
+// butterfly stages run inside a lane, the rest across lanes with __shfl_xor.
+//
+// INT8 entry: the integer butterfly runs on packed int16 pairs (|partial| <=
+// 127 * 2^s < 2^15 for hb <= 256, so 16-bit lanes are exact), then
+// y = clamp(round_half_even(M_q v / 2^n_q)).
+// FP16 entry: fp32 butterfly, y = clamp(rint(v * inv)), inv = 1/(sqrt(hb) s).
+#include <cuda_fp16.h>
+
+#include "hatq_internal.h"
+
+namespace hatq {
+namespace {
+
+constexpr int kThreads = 256;
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+    uint32_t d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+    return d;
+}
+
+// 16 int8 codes -> 8 registers, register k = (element 2k | element 2k+1 << 16),
+// sign-extended to int16 (prmt selector bit 3 replicates the byte's sign).
+__device__ __forceinline__ void unpack_i8x16(const int4 raw, uint32_t (&r)[8]) {
+    const uint32_t w[4] = {(uint32_t)raw.x, (uint32_t)raw.y, (uint32_t)raw.z, (uint32_t)raw.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        r[2 * i] = prmt(w[i], 0u, 0x9180u);
+        r[2 * i + 1] = prmt(w[i], 0u, 0xB3A2u);
+    }
+}
+
+// Sylvester butterfly over 16 packed elements of one lane plus the
+// cross-lane stages; afterwards each element holds (H~_hb x)_j.
+__device__ __forceinline__ void butterfly_i16(uint32_t (&r)[8], int hb, int lane) {
+    if (hb >= 2) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const uint32_t sw = prmt(r[k], 0u, 0x1032u);
+            r[k] = prmt(__vadd2(r[k], sw), __vsub2(r[k], sw), 0x5410u);
+        }
+    }
+    if (hb >= 4) {
+#pragma unroll
+        for (int k = 0; k < 8; k += 2) {
+            const uint32_t a = r[k], b = r[k + 1];
+            r[k] = __vadd2(a, b);
+            r[k + 1] = __vsub2(a, b);
+        }
+    }
+    if (hb >= 8) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            if (k & 2) continue;
+            const uint32_t a = r[k], b = r[k + 2];
+            r[k] = __vadd2(a, b);
+            r[k + 2] = __vsub2(a, b);
+        }
+    }
+    if (hb >= 16) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const uint32_t a = r[k], b = r[k + 4];
+            r[k] = __vadd2(a, b);
+            r[k + 4] = __vsub2(a, b);
+        }
+    }
+#pragma unroll
+    for (int m = 1; m < 16; m <<= 1) {
+        if (16 * m >= hb) break;
+        const bool upper = (lane & m) != 0;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const uint32_t p = __shfl_xor_sync(0xffffffffu, r[k], m);
+            r[k] = upper ? __vsub2(p, r[k]) : __vadd2(r[k], p);
+        }
+    }
+}
+
+__device__ __forceinline__ void butterfly_f32(float (&f)[16], int hb, int lane) {
+#pragma unroll
+    for (int h = 1; h < 16; h <<= 1) {
+        if (h >= hb) break;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            if (i & h) continue;
+            const float a = f[i], b = f[i + h];
+            f[i] = a + b;
+            f[i + h] = a - b;
+        }
+    }
+#pragma unroll
+    for (int m = 1; m < 16; m <<= 1) {
+        if (16 * m >= hb) break;
+        const bool upper = (lane & m) != 0;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const float p = __shfl_xor_sync(0xffffffffu, f[i], m);
+            f[i] = upper ? p - f[i] : f[i] + p;
+        }
+    }
+}
+
+// round(P / 2^n) half to even, clamped to [-127, 127].
+__device__ __forceinline__ int requant(long long P, int n) {
+    long long q = P;
+    if (n > 0) q = (P + ((1LL << (n - 1)) - 1) + ((P >> n) & 1)) >> n;
+    q = q < -127 ? -127 : (q > 127 ? 127 : q);
+    return (int)q;
+}
+
+__device__ __forceinline__ int clamp127(int v) { return v < -127 ? -127 : (v > 127 ? 127 : v); }
+
+__device__ __forceinline__ uint32_t pack4(int a, int b, int c, int d) {
+    return (uint32_t)(a & 0xff) | ((uint32_t)(b & 0xff) << 8) | ((uint32_t)(c & 0xff) << 16) |
+           ((uint32_t)(d & 0xff) << 24);
+}
+
+__device__ __forceinline__ int lo16(uint32_t r) { return (int)(short)(r & 0xffffu); }
+__device__ __forceinline__ int hi16(uint32_t r) { return ((int)r) >> 16; }
+
+__device__ __forceinline__ void load_f16x16(const __half *p, float (&f)[16]) {
+    const int4 a = __ldg(reinterpret_cast<const int4 *>(p));
+    const int4 b = __ldg(reinterpret_cast<const int4 *>(p) + 1);
+    const uint32_t w[8] = {(uint32_t)a.x, (uint32_t)a.y, (uint32_t)a.z, (uint32_t)a.w,
+                           (uint32_t)b.x, (uint32_t)b.y, (uint32_t)b.z, (uint32_t)b.w};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        __half2 h2 = *reinterpret_cast<const __half2 *>(&w[i]);
+        const float2 v = __half22float2(h2);
+        f[2 * i] = v.x;
+        f[2 * i + 1] = v.y;
+    }
+}
+
+// MODE 0: static scale. MODE 1: scale from the dynamic parameter block.
+// MODE 2: max-abs pass of the dynamic mode (no store).
+template <bool F16, int MODE>
+__global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
+    const int lane = threadIdx.x & 31;
+    const long long warp = ((long long)blockIdx.x * kThreads + threadIdx.x) >> 5;
+    const long long nwarps = ((long long)gridDim.x * kThreads) >> 5;
+    const long long tiles = (a.total + 511) >> 9;
+    long long mult = a.mult;
+    int shift = a.shift;
+    float inv = a.inv;
+    if (MODE == 1) {
+        mult = a.dyn->mult;
+        shift = a.dyn->shift;
+        inv = a.dyn->inv;
+    }
+    uint32_t local_max = 0;
+    float local_maxf = 0.f;
+    for (long long t = warp; t < tiles; t += nwarps) {
+        const long long e0 = (t << 9) + lane * 16;
+        const bool valid = e0 < a.total;
+        if (!F16) {
+            int4 raw = make_int4(0, 0, 0, 0);
+            if (valid) raw = __ldg(reinterpret_cast<const int4 *>(static_cast<const int8_t *>(a.x) + e0));
+            uint32_t r[8];
+            unpack_i8x16(raw, r);
+            butterfly_i16(r, a.hb, lane);
+            if (MODE == 2) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const uint32_t m0 = (uint32_t)abs(lo16(r[k])), m1 = (uint32_t)abs(hi16(r[k]));
+                    local_max = max(local_max, max(m0, m1));
+                }
+            } else if (valid) {
+                uint32_t o[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const uint32_t r0 = r[2 * i], r1 = r[2 * i + 1];
+                    o[i] = pack4(requant(mult * lo16(r0), shift), requant(mult * hi16(r0), shift),
+                                 requant(mult * lo16(r1), shift), requant(mult * hi16(r1), shift));
+                }
+                *reinterpret_cast<int4 *>(a.y + e0) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
+            }
+        } else {
+            float f[16];
+            if (valid) {
+                load_f16x16(static_cast<const __half *>(a.x) + e0, f);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) f[i] = 0.f;
+            }
+            butterfly_f32(f, a.hb, lane);
+            if (MODE == 2) {
+#pragma unroll
+                for (int i = 0; i < 16; ++i) local_maxf = fmaxf(local_maxf, fabsf(f[i]));
+            } else if (valid) {
+                uint32_t o[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    o[i] = pack4(clamp127(__float2int_rn(f[4 * i] * inv)), clamp127(__float2int_rn(f[4 * i + 1] * inv)),
+                                 clamp127(__float2int_rn(f[4 * i + 2] * inv)), clamp127(__float2int_rn(f[4 * i + 3] * inv)));
+                *reinterpret_cast<int4 *>(a.y + e0) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
+            }
+        }
+    }
+    if (MODE == 2) {
+        uint32_t m = F16 ? __float_as_uint(local_maxf) : local_max;   // nonnegative floats order as integers
+        m = __reduce_max_sync(0xffffffffu, m);
+        if (lane == 0 && m) atomicMax(&a.dyn->maxbits, m);
+    }
+}
+
+// round(num / den) half to even for num, den > 0.
+__device__ long long div_rne(unsigned long long num, unsigned long long den) {
+    unsigned long long q = num / den, r = num % den;
+    if (2 * r > den || (2 * r == den && (q & 1))) ++q;
+    return (long long)q;
+}
+
+// Dynamic parameters from the max-abs: INT8 entry uses the exact rational
+// rho = 127 / max|v| (the 1/sqrt(hb) and s_in cancel), M = round(rho 2^n) with
+// the largest n such that M < 2^31 and M 127 hb < 2^62; the scan starts at
+// n = 55 (127 * 2^55 < 2^63), and every n > 39 fails M < 2^31 for the
+// max |v| <= 127 * 256 of this operator, so the result equals a scan from 62.
+__global__ void act_dyn_params_kernel(DynParams *p, int f16, int hb, float s_in, float *s_used, int *err) {
+    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    const unsigned int mb = p->maxbits;
+    const double sq = sqrt((double)hb);
+    if (mb == 0) {
+        p->mult = 0; p->shift = 0; p->inv = 0.f;
+        if (s_used) *s_used = 1.0f;
+        return;
+    }
+    if (f16) {
+        const float m = __uint_as_float(mb);
+        p->inv = 127.0f / m;
+        p->mult = 0; p->shift = 0;
+        if (s_used) *s_used = (float)((double)m / (sq * 127.0));
+        return;
+    }
+    int found = -1;
+    long long M = 0;
+    for (int n = 55; n >= 0; --n) {
+        const long long m = div_rne(127ull << n, (unsigned long long)mb);
+        if (m >= (1LL << 31)) continue;
+        const unsigned long long worst = (unsigned long long)m * 127ull * (unsigned long long)hb;
+        if (worst >= (1ull << 62)) continue;
+        found = n; M = m;
+        break;
+    }
+    if (found < 0 || M < (1LL << 15)) {
+        atomicExch(err, kErrBounds);
+        found = 0; M = 0;
+    }
+    p->mult = M;
+    p->shift = found;
+    p->inv = 0.f;
+    if (s_used) *s_used = (float)(((double)s_in * (double)mb) / (sq * 127.0));
+}
+
+int num_sms() {
+    static int sms = 0;
+    if (!sms) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (sms <= 0) sms = 148;
+    }
+    return sms;
+}
+
+int grid_for(long long total) {
+    const long long tiles = (total + 511) / 512;
+    const long long want = (tiles + 7) / 8;           // 8 warps per block
+    const long long cap = (long long)num_sms() * 8;   // 8 resident blocks of 256 threads per SM
+    return (int)(want < 1 ? 1 : (want < cap ? want : cap));
+}
+
+}  // namespace
+
+cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s) {
+    const int grid = grid_for(a.total);
+    if (a.f16) act_quant_kernel<true, 0><<<grid, kThreads, 0, s>>>(a);
+    else act_quant_kernel<false, 0><<<grid, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_act_dynamic(const ActQuantArgs &a, float s_in, float *s_used, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(a.dyn, 0, sizeof(DynParams), s);
+    if (e != cudaSuccess) return e;
+    const int grid = grid_for(a.total);
+    if (a.f16) act_quant_kernel<true, 2><<<grid, kThreads, 0, s>>>(a);
+    else act_quant_kernel<false, 2><<<grid, kThreads, 0, s>>>(a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    act_dyn_params_kernel<<<1, 32, 0, s>>>(a.dyn, a.f16, a.hb, s_in, s_used, a.err);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (a.f16) act_quant_kernel<true, 1><<<grid, kThreads, 0, s>>>(a);
+    else act_quant_kernel<false, 1><<<grid, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace hatq

@@ -1,0 +1,68 @@
+// Internal interface between the host side of libhatq (hatq_api.cu) and the
+// kernel translation units. Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace hatq {
+
+// Error word codes written by kernels (read back by hatq_sync_status).
+enum : int { kErrNone = 0, kErrWaitTimeout = 1, kErrBounds = 2 };
+
+// ---------------------------------------------------------------- quantize
+struct ActQuantArgs {
+    const void *x;        // int8 or fp16 NHWC
+    int8_t *y;
+    long long total;      // elements, multiple of 16
+    int hb;               // 1..256
+    int f16;              // input is fp16
+    long long mult;       // static INT8 entry: M_q
+    int shift;            //                    n_q
+    float inv;            // static FP16 entry: 1 / (sqrt(hb) s_out)
+    // dynamic mode: device parameter block written by the parameter kernel
+    struct DynParams *dyn;
+    int *err;
+};
+
+// Device-side parameters of the dynamic-scale mode (lives in the caller's workspace).
+struct DynParams {
+    unsigned int maxbits;   // max |H~ x| (integer, or fp32 bits for FP16 entry)
+    int shift;
+    long long mult;
+    float inv;
+    float pad_;
+    unsigned long long reserved;
+};
+
+cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s);
+cudaError_t launch_act_dynamic(const ActQuantArgs &a, float s_in, float *s_used, cudaStream_t s);
+
+// ---------------------------------------------------------------- conv
+struct ConvArgs {
+    int n, h, w, c;
+    int ho, wo, co;
+    int kh, kw, stride, pad;
+    int tw, th, tiles_w, tiles_h;    // output tile: tw x th pixels (tw * th == 128)
+    int n_t;                         // output channels per tile
+    int num_kb;                      // 64-wide reduction blocks
+    int cin_kb;                      // reduction blocks per kernel tap (tiled loader)
+    int gather;                      // small-channel loader
+    int chunk_kb;                    // reduction blocks per exact fp32 chunk
+    int stages;
+    int tmem_cols, part_col;
+    int stage_bytes, b_bytes, raw_bytes;
+    const int8_t *x;
+    const int32_t *b_int;
+    const int32_t *mult;
+    const float *deq;
+    int shift, hb_out, hb_next, act, out_f32;
+    void *y;
+    int *err;
+};
+
+cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const ConvArgs &a,
+                        int smem_bytes, cudaStream_t s);
+
+}  // namespace hatq

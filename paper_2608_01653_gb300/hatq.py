@@ -1,0 +1,278 @@
+"""Thin Python binding of libhatq (include/hatq.h): argument marshalling only.
+
+Every computation runs inside libhatq's CUDA kernels (or, for the offline
+weight preparation, its host code). PyTorch supplies device memory and the
+current stream. There is no CPU fallback: if the library cannot be built or
+loaded, or no CUDA device is present, the calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import re
+from dataclasses import dataclass
+
+import numpy as np
+
+from . import build as _build
+
+OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_OVERFLOW, ERR_CUDA, ERR_TIMEOUT = range(6)
+DH, WH = 0, 1
+ACT_NONE, ACT_RELU = 0, 1
+IN_OPERAND, IN_I8, IN_F16 = 0, 1, 2
+
+_ACTS = {"none": ACT_NONE, "relu": ACT_RELU}
+_FORMS = {"DH": DH, "WH": WH}
+
+
+class HatqError(RuntimeError):
+    def __init__(self, status, message):
+        super().__init__(f"hatq status {status}: {message}")
+        self.status = status
+
+
+class ConvDesc(ctypes.Structure):
+    _fields_ = [("c_in", ctypes.c_int), ("c_out", ctypes.c_int), ("kh", ctypes.c_int), ("kw", ctypes.c_int),
+                ("stride", ctypes.c_int), ("pad", ctypes.c_int), ("form", ctypes.c_int),
+                ("hb_in", ctypes.c_int), ("hb_out", ctypes.c_int)]
+
+
+class PreparedStruct(ctypes.Structure):
+    _fields_ = [("d", ConvDesc), ("act", ctypes.c_int), ("hb_next", ctypes.c_int), ("out_f32", ctypes.c_int),
+                ("shift", ctypes.c_int), ("k_pad", ctypes.c_int), ("gather", ctypes.c_int),
+                ("s_x", ctypes.c_float), ("s_y", ctypes.c_float),
+                ("w_i8", ctypes.c_void_p), ("w_f16", ctypes.c_void_p), ("b_int", ctypes.c_void_p),
+                ("mult", ctypes.c_void_p), ("deq", ctypes.c_void_p), ("s_w", ctypes.c_void_p),
+                ("opaque", ctypes.c_uint64 * 16)]
+
+
+_LIB = None
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+_F = ctypes.c_float
+
+
+def load(build: bool = True) -> ctypes.CDLL:
+    """Load libhatq.so (building it in-tree first if it is missing or stale)."""
+    global _LIB
+    if _LIB is None:
+        path = _build.build() if build else _build.LIB
+        lib = ctypes.CDLL(path)
+        sig = {
+            "hatq_prepared_sizes": (_I, [ctypes.POINTER(ConvDesc), ctypes.POINTER(ctypes.c_size_t),
+                                         ctypes.POINTER(ctypes.c_size_t)]),
+            "hatq_prepare_weights": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _I, _I, _I,
+                                          ctypes.POINTER(PreparedStruct), _P]),
+            "hatq_prepare_weights_host": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _I, _I, _I,
+                                               _P, _P, _P, _P, _P, _P, ctypes.POINTER(_I)]),
+            "hatq_quantize_act": (_I, [_P, _I, _F, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P]),
+            "hatq_conv2d_i8": (_I, [_P, _I, _I, _I, ctypes.POINTER(PreparedStruct), _P, _P]),
+            "hatq_layer": (_I, [_P, _I, _F, _I, _I, _I, ctypes.POINTER(PreparedStruct), _P, _P,
+                                ctypes.c_size_t, _P]),
+            "hatq_layer_launches": (_I, [_I, _F, ctypes.POINTER(PreparedStruct)]),
+            "hatq_last_error": (ctypes.c_char_p, []),
+            "hatq_sync_status": (_I, [_P]),
+            "hatq_version": (_I, []),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _LIB = lib
+    return _LIB
+
+
+def declared_functions(header_path: str | None = None):
+    """Names of the functions include/hatq.h declares."""
+    import os
+    header_path = header_path or os.path.join(_build.INCLUDE, "hatq.h")
+    text = open(header_path).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(hatq_[a-z0-9_]+)\s*\(", text)))
+
+
+def last_error() -> str:
+    return load().hatq_last_error().decode()
+
+
+def _check(status):
+    if status != OK:
+        raise HatqError(status, last_error())
+
+
+def _torch():
+    import torch
+    if not torch.cuda.is_available():
+        raise RuntimeError("libhatq needs a CUDA device; none is available")
+    return torch
+
+
+def _stream(stream):
+    torch = _torch()
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _ptr(t):
+    return ctypes.c_void_p(t.data_ptr()) if t is not None else None
+
+
+def make_desc(c_in, c_out, k, stride, pad, form, hb_in=0, hb_out=0, kw=None) -> ConvDesc:
+    form = _FORMS.get(form, form)
+    return ConvDesc(c_in, c_out, k, k if kw is None else kw, stride, pad, form, hb_in, hb_out)
+
+
+def desc_from_spec(spec) -> ConvDesc:
+    """A ConvDesc from a layer description with c_in, c_out, k, stride, pad, form, hb_in, hb_out."""
+    return make_desc(spec.c_in, spec.c_out, spec.k, spec.stride, spec.pad, spec.form, spec.hb_in, spec.hb_out)
+
+
+def prepared_sizes(desc: ConvDesc):
+    w = ctypes.c_size_t()
+    c = ctypes.c_size_t()
+    _check(load().hatq_prepared_sizes(ctypes.byref(desc), ctypes.byref(w), ctypes.byref(c)))
+    return w.value, c.value
+
+
+@dataclass
+class HostPrepared:
+    w_i8: np.ndarray
+    w_f16: np.ndarray
+    b_int: np.ndarray
+    mult: np.ndarray
+    deq: np.ndarray
+    s_w: np.ndarray
+    shift: int
+
+
+def prepare_weights_host(desc: ConvDesc, w_ohwi, bias, s_x, s_y, act="none", hb_next=0, out_f32=False):
+    """hatq_prepare_weights_host: the offline preparation into host arrays."""
+    w_elems, ch = prepared_sizes(desc)
+    w = np.ascontiguousarray(w_ohwi, dtype=np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    out = HostPrepared(np.zeros(w_elems, np.int8), np.zeros(w_elems, np.uint16), np.zeros(ch, np.int32),
+                       np.zeros(ch, np.int32), np.zeros(ch, np.float32), np.zeros(ch, np.float32), 0)
+    shift = ctypes.c_int()
+    _check(load().hatq_prepare_weights_host(
+        ctypes.byref(desc), w.ctypes.data, None if b is None else b.ctypes.data, float(s_x), float(s_y),
+        _ACTS.get(act, act), int(hb_next), int(bool(out_f32)), out.w_i8.ctypes.data, out.w_f16.ctypes.data,
+        out.b_int.ctypes.data, out.mult.ctypes.data, out.deq.ctypes.data, out.s_w.ctypes.data, ctypes.byref(shift)))
+    out.shift = shift.value
+    k_pad = w_elems // desc.c_out
+    out.w_i8 = out.w_i8.reshape(desc.c_out, k_pad)
+    out.w_f16 = out.w_f16.reshape(desc.c_out, k_pad)
+    return out
+
+
+class PreparedLayer:
+    """A prepared layer: device buffers (torch tensors) plus the C struct."""
+
+    def __init__(self, desc: ConvDesc, device="cuda"):
+        torch = _torch()
+        w_elems, ch = prepared_sizes(desc)
+        self.desc = desc
+        self.w_i8 = torch.zeros(w_elems, dtype=torch.int8, device=device)
+        self.w_f16 = torch.zeros(w_elems, dtype=torch.float16, device=device)
+        self.b_int = torch.zeros(ch, dtype=torch.int32, device=device)
+        self.mult = torch.zeros(ch, dtype=torch.int32, device=device)
+        self.deq = torch.zeros(ch, dtype=torch.float32, device=device)
+        self.s_w = torch.zeros(ch, dtype=torch.float32, device=device)
+        self.struct = PreparedStruct()
+        self.struct.w_i8 = self.w_i8.data_ptr()
+        self.struct.w_f16 = self.w_f16.data_ptr()
+        self.struct.b_int = self.b_int.data_ptr()
+        self.struct.mult = self.mult.data_ptr()
+        self.struct.deq = self.deq.data_ptr()
+        self.struct.s_w = self.s_w.data_ptr()
+
+    @property
+    def c_in(self):
+        return self.desc.c_in
+
+    @property
+    def c_out(self):
+        return self.desc.c_out
+
+    @property
+    def out_f32(self):
+        return bool(self.struct.out_f32)
+
+    @property
+    def s_x(self):
+        return float(self.struct.s_x)
+
+    @property
+    def s_y(self):
+        return float(self.struct.s_y)
+
+    def out_shape(self, n, h, w):
+        d = self.desc
+        return (n, (h + 2 * d.pad - d.kh) // d.stride + 1, (w + 2 * d.pad - d.kw) // d.stride + 1, d.c_out)
+
+
+def prepare_weights(desc: ConvDesc, w_ohwi, bias, s_x, s_y, act="none", hb_next=0, out_f32=False,
+                    stream=None, device="cuda") -> PreparedLayer:
+    """hatq_prepare_weights: offline transform, quantize and pack into device buffers."""
+    L = PreparedLayer(desc, device)
+    w = np.ascontiguousarray(w_ohwi, dtype=np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    _check(load().hatq_prepare_weights(ctypes.byref(desc), w.ctypes.data, None if b is None else b.ctypes.data,
+                                       float(s_x), float(s_y), _ACTS.get(act, act), int(hb_next),
+                                       int(bool(out_f32)), ctypes.byref(L.struct), _stream(stream)))
+    return L
+
+
+def quantize_act(x, x_kind, s_in, hb, s_out, y=None, s_used=None, workspace=None, stream=None):
+    """hatq_quantize_act on a CUDA NHWC tensor (int8 codes or fp16 values).
+    s_out <= 0 selects the dynamic mode (s_used: 1-element float32 CUDA tensor)."""
+    torch = _torch()
+    n, h, w, c = x.shape
+    if y is None:
+        y = torch.empty((n, h, w, c), dtype=torch.int8, device=x.device)
+    if s_out <= 0:
+        if s_used is None:
+            s_used = torch.empty(1, dtype=torch.float32, device=x.device)
+        if workspace is None:
+            workspace = torch.empty(64, dtype=torch.uint8, device=x.device)
+    _check(load().hatq_quantize_act(_ptr(x), int(x_kind), float(s_in), n, h, w, c, int(hb), float(s_out), _ptr(y),
+                                    _ptr(s_used), _ptr(workspace), _stream(stream)))
+    return (y, s_used) if s_out <= 0 else y
+
+
+def conv2d_i8(x, L: PreparedLayer, y=None, stream=None):
+    """hatq_conv2d_i8: convolution + fused requantize epilogue on the INT8 operand x (NHWC)."""
+    torch = _torch()
+    n, h, w, c = x.shape
+    if c != L.c_in:
+        raise ValueError("channel mismatch")
+    if y is None:
+        y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32 if L.out_f32 else torch.int8, device=x.device)
+    _check(load().hatq_conv2d_i8(_ptr(x), n, h, w, ctypes.byref(L.struct), _ptr(y), _stream(stream)))
+    return y
+
+
+def layer(x, x_kind, s_in, L: PreparedLayer, y=None, scratch=None, stream=None):
+    """hatq_layer: input transform/quantize (when needed) + conv in one call."""
+    torch = _torch()
+    n, h, w, c = x.shape
+    if y is None:
+        y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32 if L.out_f32 else torch.int8, device=x.device)
+    nbytes = 0
+    if layer_launches(x_kind, s_in, L) > 1:
+        if scratch is None:
+            scratch = torch.empty(n * h * w * c, dtype=torch.int8, device=x.device)
+        nbytes = scratch.numel() * scratch.element_size()
+    _check(load().hatq_layer(_ptr(x), int(x_kind), float(s_in), n, h, w, ctypes.byref(L.struct), _ptr(y),
+                             _ptr(scratch), nbytes, _stream(stream)))
+    return y
+
+
+def layer_launches(x_kind, s_in, L: PreparedLayer) -> int:
+    return int(load().hatq_layer_launches(int(x_kind), float(s_in), ctypes.byref(L.struct)))
+
+
+def sync_status(stream=None):
+    _check(load().hatq_sync_status(_stream(stream)))
+
+
+def version() -> int:
+    return int(load().hatq_version())

@@ -1,0 +1,130 @@
+"""C-ABI checks that need no GPU: the library builds and loads, exports every
+function include/hatq.h declares, validates arguments on the host, and its
+offline weight preparation (hatq_prepare_weights_host) reproduces the CPU
+oracle bit for bit (codes, bias codes, multipliers, shift)."""
+import ctypes
+import json
+import os
+
+import numpy as np
+import pytest
+
+from oracle import hatq_oracle as O
+from paper_2608_01653_gb300 import hatq as H
+from synth import configs as C
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    return H.load()
+
+
+def test_exports_every_declared_function(lib):
+    names = H.declared_functions()
+    assert "hatq_conv2d_i8" in names and "hatq_prepare_weights" in names
+    assert "hatq_quantize_act" in names and "hatq_layer" in names
+    for name in names:
+        assert hasattr(lib, name), f"libhatq.so does not export {name}"
+
+
+def test_version_and_last_error(lib):
+    assert H.version() == 1
+    d = H.make_desc(64, 48, 3, 1, 1, "DH", hb_in=64)          # c_out not a multiple of 32
+    with pytest.raises(H.HatqError) as e:
+        H.prepared_sizes(d)
+    assert e.value.status == H.ERR_UNSUPPORTED and "c_out" in H.last_error()
+
+
+@pytest.mark.parametrize("desc,k_pad", [
+    (H.make_desc(192, 192, 5, 2, 2, "DH", hb_in=64), 25 * 192),
+    (H.make_desc(3, 192, 5, 2, 2, "WH", hb_out=64), 128),       # small-channel packing 75 -> 128
+    (H.make_desc(32, 224, 3, 1, 1, "DH", hb_in=32), 9 * 64),    # c_in padded to 64 per tap
+    (H.make_desc(224, 128, 3, 1, 1, "WH", hb_out=128), 9 * 256),
+    (H.make_desc(128, 128, 1, 1, 0, "DH", hb_in=128), 128),
+])
+def test_prepared_sizes(desc, k_pad):
+    w, c = H.prepared_sizes(desc)
+    assert c == desc.c_out and w == desc.c_out * k_pad
+
+
+@pytest.mark.parametrize("bad", [
+    dict(c_in=192, c_out=192, k=5, stride=3, pad=2, form="DH", hb_in=64),     # stride 3
+    dict(c_in=192, c_out=192, k=5, stride=2, pad=2, form="DH", hb_in=48),     # block not a power of two
+    dict(c_in=192, c_out=192, k=5, stride=2, pad=2, form="DH", hb_in=128),    # block does not divide c_in
+    dict(c_in=192, c_out=192, k=5, stride=2, pad=2, form="WH", hb_out=256),   # WH block too large
+    dict(c_in=192, c_out=192, k=5, stride=2, pad=5, form="DH", hb_in=64),     # pad >= k
+    dict(c_in=3, c_out=192, k=5, stride=2, pad=2, form="DH", hb_in=2),        # DH with c_in % 16
+    dict(c_in=192, c_out=192, k=5, stride=2, pad=2, form="XX", hb_in=64),
+])
+def test_invalid_descriptors_rejected(bad):
+    form = {"DH": H.DH, "WH": H.WH}.get(bad.pop("form"), 7)
+    d = H.make_desc(form=form, **bad)
+    with pytest.raises(H.HatqError) as e:
+        H.prepared_sizes(d)
+    assert e.value.status in (H.ERR_INVALID_ARG, H.ERR_UNSUPPORTED)
+
+
+def test_prepare_rejects_unfusable_pair_and_bad_scales():
+    d = H.make_desc(64, 128, 3, 1, 1, "WH", hb_out=128)
+    w = np.zeros((128, 3, 3, 64), np.float32)
+    with pytest.raises(H.HatqError) as e:
+        H.prepare_weights_host(d, w, None, 0.1, 0.1, "relu", hb_next=128)
+    assert e.value.status == H.ERR_UNSUPPORTED
+    with pytest.raises(H.HatqError):
+        H.prepare_weights_host(d, w, None, -1.0, 0.1)
+    with pytest.raises(H.HatqError):
+        H.prepare_weights_host(d, w, None, 0.1, 0.1, out_f32=True, hb_next=64)
+
+
+def _oracle_packed(p, desc, k_pad):
+    """The oracle's OHWI codes laid out in the library's packed reduction order."""
+    co, kh, kw, ci = p.w_int.shape
+    out = np.zeros((co, k_pad), np.int8)
+    if ci % 16:
+        out[:, :kh * kw * ci] = p.w_int.reshape(co, -1)
+    else:
+        cin_pad = (ci + 63) // 64 * 64
+        tmp = np.zeros((co, kh * kw, cin_pad), np.int8)
+        tmp[:, :, :ci] = p.w_int.reshape(co, kh * kw, ci)
+        out[:] = tmp.reshape(co, -1)
+    return out
+
+
+def _all_layers():
+    calib = json.load(open(os.path.join(GOLDEN, "calibration.json")))["configs"]
+    for cname in ("cfg0", "cfg1", "cfg2", "cfg3"):
+        cfg = C.CONFIGS[cname]
+        for ch in cfg.chains:
+            plan = C.plan_chain(ch)
+            params = C.chain_params(ch)
+            for i, L in enumerate(ch.layers):
+                last = i == len(ch.layers) - 1
+                yield (f"{cname}/{ch.name}/{L.name}", L, params[i], calib[cname][ch.name][i], plan[i],
+                       ch.out_f32 and last)
+
+
+@pytest.mark.parametrize("case", list(_all_layers()), ids=lambda c: c[0])
+def test_host_prepare_matches_oracle_bit_exact(case):
+    name, L, (w, b), sc, hb_next, out_f32 = case
+    desc = H.desc_from_spec(L)
+    got = H.prepare_weights_host(desc, w, b, sc["s_x"], sc["s_out"], L.act, hb_next, out_f32)
+    ref = O.prepare_layer(w, b, L.form, L.hb_in, L.hb_out, sc["s_x"], sc["s_out"], L.act, hb_next, out_f32,
+                          L.stride, L.pad)
+    assert np.array_equal(got.w_i8, _oracle_packed(ref, desc, got.w_i8.shape[1]))
+    assert np.array_equal(got.w_f16.view(np.float16).astype(np.int64), got.w_i8.astype(np.int64))
+    assert np.array_equal(got.b_int, ref.b_int)
+    assert np.array_equal(got.s_w, ref.s_w.astype(np.float32))
+    if out_f32:
+        assert np.array_equal(got.deq, ref.deq.astype(np.float32))
+    else:
+        assert got.shift == ref.n
+        assert np.array_equal(got.mult.astype(np.int64), ref.M)
+
+
+def test_host_prepare_zero_weights_and_no_bias():
+    d = H.make_desc(64, 64, 1, 1, 0, "DH", hb_in=64)
+    w = np.zeros((64, 1, 1, 64), np.float32)
+    got = H.prepare_weights_host(d, w, None, 0.1, 0.1)
+    assert not got.w_i8.any() and np.all(got.s_w == 1.0) and not got.b_int.any()
