@@ -51,9 +51,12 @@ def parse():
     p.add_argument("--steps", type=int, default=10)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--workload", default="cfg4", choices=["cfg4", "cfg2", "cfg1", "fwht"])
+    p.add_argument("--workload", default="cfg4", choices=["cfg4", "cfg2", "cfg1", "fwht"],
+                   help="fwht: the INT8 transform+requantize pass alone on the config-4 ga2 input")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--layer", default="", help="time one layer of the config-4 chains (e.g. ga2, h1, s0a)")
+    p.add_argument("--batch", type=int, default=8, help="batch for --layer / the FWHT pass")
     return p.parse_args()
 
 
@@ -189,6 +192,72 @@ def workload_name(cfg):
     return f"{cfg.name}: {cfg.description}"
 
 
+# ------------------------------------------------------------------ single-kernel modes
+
+def time_events(fn, steps, warmup):
+    import torch
+    for _ in range(max(3, warmup)):
+        fn()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(steps):
+        fn()
+    e1.record()
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / steps
+
+
+def run_layer_mode(args, cfg, scales):
+    """One conv layer of the config-4 chains on a synthetic INT8 operand."""
+    import torch
+    from paper_2608_01653_gb300 import hatq as H
+    H.load()
+    for ch in cfg.chains:
+        for i, L in enumerate(ch.layers):
+            if L.name == args.layer:
+                n, h, w = ch.with_batch(args.batch, ch.h, ch.w, 0).shapes()[i]
+                params = C.chain_params(ch)[i]
+                hb_next = C.plan_chain(ch)[i]
+                sc = scales[ch.name][i]
+                P = H.prepare_weights(H.desc_from_spec(L), params[0], params[1], sc["s_x"], sc["s_out"], L.act,
+                                      hb_next, False)
+                x = torch.from_numpy(I.activations_i8((n, h, w, L.c_in), seed=5, s_in=0.05)).cuda()
+                y = torch.empty(P.out_shape(n, h, w), dtype=torch.int8, device="cuda")
+                ms = time_events(lambda: H.conv2d_i8(x, P, y=y), args.steps, args.warmup)
+                H.sync_status()
+                flops = 2 * L.macs(n, h, w)
+                peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
+                peak = peaks.get("bf16_tflops", FALLBACK_BF16_TFLOPS)
+                tf = flops / (ms / 1000) / 1e12
+                print(json.dumps({"mode": "layer", "layer": L.name, "chain": ch.name, "batch": n, "in_hw": [h, w],
+                                  "c_in": L.c_in, "c_out": L.c_out, "k": L.k, "stride": L.stride, "form": L.form,
+                                  "hb_next": hb_next, "ms": ms, "tflops": tf, "peak_bf16_burst": peak,
+                                  "frac": tf / peak}), flush=True)
+                return
+    raise SystemExit(f"unknown layer {args.layer}")
+
+
+def run_fwht_mode(args):
+    """The INT8-entry transform + requantize pass (hb 64) on an NHWC tensor
+    shaped like the config-4 ga2 input: 1 byte read + 1 byte written per element."""
+    import torch
+    from paper_2608_01653_gb300 import hatq as H
+    H.load()
+    shape = (args.batch, 1080, 1920, 192)
+    x = torch.from_numpy(I.uniform_codes(shape, seed=9)).cuda()
+    y = torch.empty_like(x)
+    ms = time_events(lambda: H.quantize_act(x, H.IN_I8, 0.05, 64, 0.07, y=y), args.steps, args.warmup)
+    H.sync_status()
+    nbytes = 2 * x.numel()
+    peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
+    peak = peaks.get("hbm_gbs", FALLBACK_HBM_GBS)
+    gbs = nbytes / (ms / 1000) / 1e9
+    print(json.dumps({"mode": "fwht", "shape": list(shape), "hb": 64, "ms": ms, "GB/s": gbs, "peak_hbm_gbs": peak,
+                      "frac": gbs / peak}), flush=True)
+
+
 # ------------------------------------------------------------------ GPU arm
 
 def main():
@@ -199,6 +268,12 @@ def main():
     cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht") else args.workload)
     if args.impl == "reference":
         run_reference(args, cfg, scales)
+        return
+    if args.layer:
+        run_layer_mode(args, cfg, scales)
+        return
+    if args.workload == "fwht":
+        run_fwht_mode(args)
         return
 
     import torch

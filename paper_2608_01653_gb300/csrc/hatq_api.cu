@@ -51,6 +51,8 @@ int *err_word() {
     return ptrs[dev];
 }
 
+constexpr int kTileRows = 128;
+
 bool pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 int sylvester_sign(int i, int j) { return (__builtin_popcount((unsigned)(i & j)) & 1) ? -1 : 1; }
@@ -444,9 +446,16 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     a.b_bytes = a.n_t * 128;
     a.raw_bytes = g.gather ? 0 : 8192;
     a.stage_bytes = 16384 + a.b_bytes + a.raw_bytes;
-    const int smem_cap = 227 * 1024 - 1024 - 256;
+    // reserve room for barriers, the gather table, epilogue constants and the input window
+    int win_reserve = 0;
+    if (g.gather) {
+        const int wh = (a.th - 1) * d->stride + d->kh, ww = (a.tw - 1) * d->stride + d->kw;
+        win_reserve = (wh * ww * d->c_in + 127) & ~127;
+    }
+    const int smem_cap = 227 * 1024 - 1024 - 1024 - 256 - 3 * 1024 - 128 - (g.gather ? g.k_pad * 4 : 0) - win_reserve;
     a.stages = smem_cap / a.stage_bytes;
     if (a.stages > 8) a.stages = 8;
+    if (g.gather && a.stages > 4) a.stages = 4;
     if (a.stages < 2) return fail(HATQ_ERR_UNSUPPORTED, "tile does not fit in shared memory");
     int pc = 32;
     while (pc < a.n_t) pc <<= 1;
@@ -464,7 +473,18 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     a.y = y;
     a.err = err_word();
     if (!a.err) return fail(HATQ_ERR_CUDA, "no CUDA device");
-    const int smem_bytes = a.stages * a.stage_bytes + 1024 + 8 * (3 * a.stages + 3) + 16;
+    // dynamic shared memory: [stages][barriers | gather table | constants | window]
+    const int bar_bytes = 8 * (3 * a.stages + 3) + 16;
+    const int table_bytes = g.gather ? a.num_kb * 64 * 4 : 0;
+    a.const_off = (bar_bytes + table_bytes + 127) & ~127;
+    a.win_off = a.const_off + 3 * 256 * 4;
+    a.win_h = (a.th - 1) * d->stride + d->kh;
+    a.win_w = (a.tw - 1) * d->stride + d->kw;
+    const int win_bytes = g.gather ? (a.win_h * a.win_w * d->c_in + 127) & ~127 : 0;
+    const int smem_bytes = a.stages * a.stage_bytes + 1024 + a.win_off + win_bytes;
+    const int out_stage = kTileRows * (a.n_t * (L->out_f32 ? 4 : 1) + 16);
+    if (out_stage > a.stages * a.stage_bytes) return fail(HATQ_ERR_UNSUPPORTED, "output tile does not fit the stage buffers");
+    if (smem_bytes > 227 * 1024 - 1024) return fail(HATQ_ERR_UNSUPPORTED, "shared memory budget exceeded (%d bytes)", smem_bytes);
 
     CUtensorMap tmB, tmA;
     std::memcpy(&tmB, L->opaque, sizeof tmB);

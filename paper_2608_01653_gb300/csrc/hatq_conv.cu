@@ -24,8 +24,11 @@
 //   warp 1     TMEM allocation; lane 0 issues the MMAs and commits.
 //   warps 2-3  converters: INT8 box -> fp16 operand tile in the 128B-swizzled
 //              K-major layout the MMA descriptor expects (or, for small c_in,
-//              a direct gather of the packed reduction from global memory).
-//   warps 4-7  drain fp32 chunk sums into the int32 partial; final epilogue.
+//              a gather from the tile's input window staged in shared memory).
+//   warps 4-7  drain fp32 chunk sums into the int32 partial.
+//   all warps  final epilogue once the last MMA completed: warps w and w+4
+//              share TMEM lane quadrant w%4 and split the column groups; the
+//              output tile is staged in shared memory and copied out coalesced.
 // Every mbarrier wait is bounded: on expiry the kernel records an error word,
 // raises a CTA-wide abort flag and unwinds (waiting, again bounded, for its own
 // MMAs and copies) before freeing TMEM.
@@ -189,9 +192,20 @@ __device__ __forceinline__ uint32_t sw128_offset(int row, int chunk) {
 // ------------------------------------------------------------------ epilogue math
 
 __device__ __forceinline__ int requant8(long long v, int n) {
-    long long q = v;
-    if (n > 0) q = (v + ((1LL << (n - 1)) - 1) + ((v >> n) & 1)) >> n;
-    return (int)(q < -127 ? -127 : (q > 127 ? 127 : q));
+    // round(v / 2^n) half to even, clamped to [-127, 127]: v + 2^(n-1) - 1 + bit_n(v), then >> n.
+    int q;
+    if (n >= 32) {
+        // |v| < 2^62, so the shifted value fits in 32 bits.
+        const long long u = v + ((1LL << (n - 1)) - 1) + ((int)((unsigned long long)v >> n) & 1);
+        q = (int)(u >> n);
+    } else if (n > 0) {
+        const long long u = v + ((1LL << (n - 1)) - 1) + ((v >> n) & 1);
+        const long long w = u >> n;
+        q = w < -127 ? -127 : (w > 127 ? 127 : (int)w);
+    } else {
+        q = v < -127 ? -127 : (v > 127 ? 127 : (int)v);
+    }
+    return q < -127 ? -127 : (q > 127 ? 127 : q);
 }
 
 template <int G, int HB, typename T>
@@ -223,15 +237,17 @@ __device__ __forceinline__ void fwht(T (&t)[G], int hb) {
 }
 
 struct EpiCtx {
+    const int *b_int;    // this tile's bias codes, multipliers and dequant factors (shared memory)
+    const int *mult;
+    const float *deq;
     uint32_t t_acc;      // TMEM address of this warp's lanes, column 0 of the accumulator
     uint32_t t_part;     // ... of the int32 partial region
     bool has_part;
-    int n0;              // first output channel of the tile
-    long long pix;       // output pixel index (flat NHWC row) or -1 if outside the image
+    uint8_t *row;        // this thread's row of the shared-memory output tile
 };
 
 // Exact int32 accumulator of 16 columns starting at tile column `col`, bias included.
-__device__ __forceinline__ void load_acc16(const EpiCtx &e, const ConvArgs &a, int col, int (&v)[16]) {
+__device__ __forceinline__ void load_acc16(const EpiCtx &e, int col, int (&v)[16]) {
     uint32_t r[16];
     tmem_ld16(e.t_acc + col, r);
     if (e.has_part) {
@@ -245,31 +261,31 @@ __device__ __forceinline__ void load_acc16(const EpiCtx &e, const ConvArgs &a, i
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[i] = __float2int_rn(__uint_as_float(r[i]));
     }
-    const int4 *bp = reinterpret_cast<const int4 *>(a.b_int + e.n0 + col);
+    const int4 *bp = reinterpret_cast<const int4 *>(e.b_int + col);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const int4 b = __ldg(bp + i);
+        const int4 b = bp[i];
         v[4 * i] += b.x; v[4 * i + 1] += b.y; v[4 * i + 2] += b.z; v[4 * i + 3] += b.w;
     }
 }
 
-// t = M (.) a for 16 columns.
-__device__ __forceinline__ void scale_i64(const ConvArgs &a, int ch0, const int (&v)[16], long long *t) {
-    const int4 *mp = reinterpret_cast<const int4 *>(a.mult + ch0);
+// t = M (.) a for 16 columns starting at tile column col.
+__device__ __forceinline__ void scale_i64(const EpiCtx &e, int col, const int (&v)[16], long long *t) {
+    const int4 *mp = reinterpret_cast<const int4 *>(e.mult + col);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const int4 m = __ldg(mp + i);
+        const int4 m = mp[i];
         t[4 * i] = (long long)m.x * v[4 * i];
         t[4 * i + 1] = (long long)m.y * v[4 * i + 1];
         t[4 * i + 2] = (long long)m.z * v[4 * i + 2];
         t[4 * i + 3] = (long long)m.w * v[4 * i + 3];
     }
 }
-__device__ __forceinline__ void scale_f32(const ConvArgs &a, int ch0, const int (&v)[16], float *t) {
-    const float4 *dp = reinterpret_cast<const float4 *>(a.deq + ch0);
+__device__ __forceinline__ void scale_f32(const EpiCtx &e, int col, const int (&v)[16], float *t) {
+    const float4 *dp = reinterpret_cast<const float4 *>(e.deq + col);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const float4 d = __ldg(dp + i);
+        const float4 d = dp[i];
         t[4 * i] = d.x * (float)v[4 * i];
         t[4 * i + 1] = d.y * (float)v[4 * i + 1];
         t[4 * i + 2] = d.z * (float)v[4 * i + 2];
@@ -277,10 +293,10 @@ __device__ __forceinline__ void scale_f32(const ConvArgs &a, int ch0, const int 
     }
 }
 
+// Requantized codes of G columns starting at tile column col, written to this
+// thread's row of the shared-memory output tile (copied out coalesced later).
 template <int G>
-__device__ __forceinline__ void store_codes(const ConvArgs &a, long long pix, int ch0, const long long (&t)[G]) {
-    if (pix < 0) return;
-    int8_t *dst = static_cast<int8_t *>(a.y) + pix * a.co + ch0;
+__device__ __forceinline__ void store_codes(const ConvArgs &a, uint8_t *row, int col, const long long (&t)[G]) {
 #pragma unroll
     for (int i = 0; i < G / 16; ++i) {
         uint32_t w[4];
@@ -291,32 +307,29 @@ __device__ __forceinline__ void store_codes(const ConvArgs &a, long long pix, in
                    ((uint32_t)(requant8(t[b + 2], a.shift) & 0xff) << 16) |
                    ((uint32_t)(requant8(t[b + 3], a.shift) & 0xff) << 24);
         }
-        reinterpret_cast<int4 *>(dst)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
+        reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
     }
 }
 template <int G>
-__device__ __forceinline__ void store_f32(const ConvArgs &a, long long pix, int ch0, const float (&t)[G]) {
-    if (pix < 0) return;
-    float *dst = static_cast<float *>(a.y) + pix * a.co + ch0;
+__device__ __forceinline__ void store_f32(uint8_t *row, int col, const float (&t)[G]) {
 #pragma unroll
     for (int i = 0; i < G / 4; ++i)
-        reinterpret_cast<float4 *>(dst)[i] = make_float4(t[4 * i], t[4 * i + 1], t[4 * i + 2], t[4 * i + 3]);
+        reinterpret_cast<float4 *>(row + 4 * col)[i] = make_float4(t[4 * i], t[4 * i + 1], t[4 * i + 2], t[4 * i + 3]);
 }
 
-template <typename T>
-__device__ __forceinline__ T relu(T v) { return v > T(0) ? v : T(0); }
+__device__ __forceinline__ long long relu(long long v) { return ((int)(v >> 32)) < 0 ? 0LL : v; }
+__device__ __forceinline__ float relu(float v) { return fmaxf(v, 0.f); }
 
 // One group of G <= 64 columns held entirely in registers.
 template <int G>
 __device__ __forceinline__ void epi_group(const EpiCtx &e, const ConvArgs &a, int col) {
-    const int ch0 = e.n0 + col;
     if (!a.out_f32) {
         long long t[G];
 #pragma unroll
         for (int q = 0; q < G / 16; ++q) {
             int v[16];
-            load_acc16(e, a, col + 16 * q, v);
-            scale_i64(a, ch0 + 16 * q, v, t + 16 * q);
+            load_acc16(e, col + 16 * q, v);
+            scale_i64(e, col + 16 * q, v, t + 16 * q);
         }
         if (a.hb_out) fwht<G>(t, a.hb_out);
         if (a.act) {
@@ -324,21 +337,21 @@ __device__ __forceinline__ void epi_group(const EpiCtx &e, const ConvArgs &a, in
             for (int i = 0; i < G; ++i) t[i] = relu(t[i]);
         }
         if (a.hb_next) fwht<G>(t, a.hb_next);
-        store_codes<G>(a, e.pix, ch0, t);
+        store_codes<G>(a, e.row, col, t);
     } else {
         float t[G];
 #pragma unroll
         for (int q = 0; q < G / 16; ++q) {
             int v[16];
-            load_acc16(e, a, col + 16 * q, v);
-            scale_f32(a, ch0 + 16 * q, v, t + 16 * q);
+            load_acc16(e, col + 16 * q, v);
+            scale_f32(e, col + 16 * q, v, t + 16 * q);
         }
         if (a.hb_out) fwht<G>(t, a.hb_out);
         if (a.act) {
 #pragma unroll
             for (int i = 0; i < G; ++i) t[i] = relu(t[i]);
         }
-        store_f32<G>(a, e.pix, ch0, t);
+        store_f32<G>(e.row, col, t);
     }
 }
 
@@ -346,7 +359,6 @@ __device__ __forceinline__ void epi_group(const EpiCtx &e, const ConvArgs &a, in
 // H~_128 [x_lo; x_hi] = [H~_64 (x_lo + x_hi); H~_64 (x_lo - x_hi)], evaluated
 // as two register-resident passes of 64 outputs each.
 __device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a, int col) {
-    const int ch0 = e.n0 + col;
     const bool pre_relu = a.act && a.hb_out == 0;     // phi before H~_next
     const bool post_relu = a.act && a.hb_out != 0;    // phi after H~_out
 #pragma unroll 1
@@ -357,12 +369,12 @@ __device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a,
             for (int q = 0; q < 4; ++q) {
                 int v[16];
                 long long x[16];
-                load_acc16(e, a, col + 16 * q, v);
-                scale_i64(a, ch0 + 16 * q, v, x);
+                load_acc16(e, col + 16 * q, v);
+                scale_i64(e, col + 16 * q, v, x);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) s[16 * q + i] = pre_relu ? relu(x[i]) : x[i];
-                load_acc16(e, a, col + 64 + 16 * q, v);
-                scale_i64(a, ch0 + 64 + 16 * q, v, x);
+                load_acc16(e, col + 64 + 16 * q, v);
+                scale_i64(e, col + 64 + 16 * q, v, x);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) {
                     const long long x1 = pre_relu ? relu(x[i]) : x[i];
@@ -374,19 +386,19 @@ __device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a,
 #pragma unroll
                 for (int i = 0; i < 64; ++i) s[i] = relu(s[i]);
             }
-            store_codes<64>(a, e.pix, ch0 + 64 * pass, s);
+            store_codes<64>(a, e.row, col + 64 * pass, s);
         } else {
             float s[64];
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 int v[16];
                 float x[16];
-                load_acc16(e, a, col + 16 * q, v);
-                scale_f32(a, ch0 + 16 * q, v, x);
+                load_acc16(e, col + 16 * q, v);
+                scale_f32(e, col + 16 * q, v, x);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) s[16 * q + i] = x[i];
-                load_acc16(e, a, col + 64 + 16 * q, v);
-                scale_f32(a, ch0 + 64 + 16 * q, v, x);
+                load_acc16(e, col + 64 + 16 * q, v);
+                scale_f32(e, col + 64 + 16 * q, v, x);
 #pragma unroll
                 for (int i = 0; i < 16; ++i) s[16 * q + i] = pass == 0 ? s[16 * q + i] + x[i] : s[16 * q + i] - x[i];
             }
@@ -395,7 +407,7 @@ __device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a,
 #pragma unroll
                 for (int i = 0; i < 64; ++i) s[i] = relu(s[i]);
             }
-            store_f32<64>(a, e.pix, ch0 + 64 * pass, s);
+            store_f32<64>(e.row, col + 64 * pass, s);
         }
     }
 }
@@ -456,6 +468,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                      "r"(a.tmem_cols)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    // per-tile bias codes, multipliers and dequant factors for the epilogue,
+    // staged once (128-byte aligned, read with 16-byte vector loads)
+    int *cb = reinterpret_cast<int *>(bar_area + a.const_off);
+    for (int c = threadIdx.x; c < a.n_t; c += kThreads) {
+        cb[c] = a.b_int[n0 + c];
+        cb[256 + c] = a.mult[n0 + c];
+        reinterpret_cast<float *>(cb)[512 + c] = a.deq[n0 + c];
     }
     tc_fence_before();
     __syncthreads();
@@ -530,100 +550,163 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------------------------------------------------- converters
         constexpr int kPasses = 512 / kConvThreads;   // 128 rows x 4 quarters per 64-wide block
         const int ct = threadIdx.x - 64;              // 0..kConvThreads-1
-        int g_iy0[kPasses], g_ix0[kPasses];
-        const long long g_base = (long long)img * a.h * a.w * a.c;
-        if (a.gather) {
+        if (!a.gather) {
+            for (int kb = 0; kb < a.num_kb; ++kb) {
+                const int s = kb % S, r = kb / S;
+                if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) break;
+                uint8_t *st = smem + (size_t)s * a.stage_bytes;
+                const uint8_t *raw = st + 16384 + a.b_bytes;
+                int4 v[kPasses];                       // all loads first, then convert and store
+#pragma unroll
+                for (int p = 0; p < kPasses; ++p) {
+                    const int idx = p * kConvThreads + ct;
+                    v[p] = *reinterpret_cast<const int4 *>(raw + (idx >> 2) * 64 + (idx & 3) * 16);
+                }
+#pragma unroll
+                for (int p = 0; p < kPasses; ++p) {
+                    const int idx = p * kConvThreads + ct;
+                    const int m = idx >> 2, q = idx & 3;    // row, 16-element quarter of the 64-wide block
+                    uint32_t h[8];
+                    i8x4_to_f16x4((uint32_t)v[p].x, h[0], h[1]);
+                    i8x4_to_f16x4((uint32_t)v[p].y, h[2], h[3]);
+                    i8x4_to_f16x4((uint32_t)v[p].z, h[4], h[5]);
+                    i8x4_to_f16x4((uint32_t)v[p].w, h[6], h[7]);
+                    *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
+                    *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
+                }
+                fence_proxy_async_smem();
+                mbar_arrive(conv_bar(s));
+            }
+        } else {
+            // Small-channel layer: the tile's input window ((th-1)s+kh rows of
+            // (tw-1)s+kw pixels, zero outside the image) is copied to shared
+            // memory with coalesced byte loads, then the packed reduction index
+            // k = (ky, kx, ci) is gathered from it through a per-CTA offset table.
+            int *tab = reinterpret_cast<int *>(bar_area + 8 * (3 * S + 3) + 16);
+            uint8_t *win = bar_area + a.win_off;
+            const int taps = a.kh * a.kw;
+            for (int k = ct; k < a.num_kb * kBlockK; k += kConvThreads) {
+                const int tap = k / a.c, ci = k - tap * a.c;
+                const int ky = tap / a.kw, kx = tap - ky * a.kw;
+                tab[k] = tap < taps ? (ky * a.win_w + kx) * a.c + ci : -1;
+            }
+            {
+                const int ix_lo = wo0 * a.stride - a.pad;
+                const int row_b = a.win_w * a.c;
+                const int b_lo = max(0, -ix_lo) * a.c, b_hi = min(a.win_w, a.w - ix_lo) * a.c;
+                for (int r = 0; r < a.win_h; ++r) {
+                    const int iy = ho0 * a.stride - a.pad + r;
+                    const bool row_in = iy >= 0 && iy < a.h;
+                    const int8_t *src = a.x + (((long long)img * a.h + (row_in ? iy : 0)) * a.w + ix_lo) * a.c;
+                    for (int b = ct; b < row_b; b += kConvThreads)
+                        win[r * row_b + b] = (row_in && b >= b_lo && b < b_hi) ? (uint8_t)__ldg(src + b) : (uint8_t)0;
+                }
+            }
+            asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");
+            int rb[kPasses];
 #pragma unroll
             for (int p = 0; p < kPasses; ++p) {
                 const int m = (p * kConvThreads + ct) >> 2;
-                const int oy = ho0 + m / a.tw, ox = wo0 + m % a.tw;
-                g_iy0[p] = oy * a.stride - a.pad;
-                g_ix0[p] = ox * a.stride - a.pad;
+                rb[p] = ((m / a.tw) * a.stride * a.win_w + (m % a.tw) * a.stride) * a.c;
             }
-        }
-        for (int kb = 0; kb < a.num_kb; ++kb) {
-            const int s = kb % S, r = kb / S;
-            if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) break;
-            uint8_t *st = smem + (size_t)s * a.stage_bytes;
-            const uint8_t *raw = st + 16384 + a.b_bytes;
+            for (int kb = 0; kb < a.num_kb; ++kb) {
+                const int s = kb % S, r = kb / S;
+                if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) break;
+                uint8_t *st = smem + (size_t)s * a.stage_bytes;
 #pragma unroll
-            for (int p = 0; p < kPasses; ++p) {
-                const int idx = p * kConvThreads + ct;
-                const int m = idx >> 2, q = idx & 3;    // row, 16-element quarter of the 64-wide block
-                uint32_t w4[4];
-                if (!a.gather) {
-                    const int4 v = *reinterpret_cast<const int4 *>(raw + m * 64 + q * 16);
-                    w4[0] = (uint32_t)v.x; w4[1] = (uint32_t)v.y; w4[2] = (uint32_t)v.z; w4[3] = (uint32_t)v.w;
-                } else {
-                    int8_t b[16];
+                for (int p = 0; p < kPasses; ++p) {
+                    const int idx = p * kConvThreads + ct;
+                    const int m = idx >> 2, q = idx & 3;
+                    uint32_t w4[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
-                        const int k = kb * kBlockK + q * 16 + j;
-                        const int tap = k / a.c, ci = k - tap * a.c;
-                        const int ky = tap / a.kw, kx = tap - ky * a.kw;
-                        const int iy = g_iy0[p] + ky, ix = g_ix0[p] + kx;
-                        int8_t val = 0;
-                        if (ky < a.kh && iy >= 0 && iy < a.h && ix >= 0 && ix < a.w)
-                            val = a.x[g_base + ((long long)iy * a.w + ix) * a.c + ci];
-                        b[j] = val;
+                        const int off = tab[kb * kBlockK + q * 16 + j];
+                        const uint32_t b = off >= 0 ? (uint32_t)win[rb[p] + off] : 0u;
+                        w4[j >> 2] |= b << (8 * (j & 3));
                     }
+                    uint32_t h[8];
 #pragma unroll
-                    for (int j = 0; j < 4; ++j)
-                        w4[j] = (uint32_t)(uint8_t)b[4 * j] | ((uint32_t)(uint8_t)b[4 * j + 1] << 8) |
-                                ((uint32_t)(uint8_t)b[4 * j + 2] << 16) | ((uint32_t)(uint8_t)b[4 * j + 3] << 24);
+                    for (int j = 0; j < 4; ++j) i8x4_to_f16x4(w4[j], h[2 * j], h[2 * j + 1]);
+                    *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
+                    *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
                 }
-                uint32_t h[8];
-#pragma unroll
-                for (int j = 0; j < 4; ++j) i8x4_to_f16x4(w4[j], h[2 * j], h[2 * j + 1]);
-                *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
-                *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
+                fence_proxy_async_smem();
+                mbar_arrive(conv_bar(s));
             }
-            fence_proxy_async_smem();
-            mbar_arrive(conv_bar(s));
         }
     } else {
-        // ---------------------------------------------------------- drain + epilogue
-        const int quad = warp & 3;                 // TMEM lane quadrant this warp may access
+        // ---------------------------------------------------------- drains (chunk sums -> int32 partial)
+        const uint32_t t_acc = tmem + ((uint32_t)((warp & 3) * 32) << 16);
+        const uint32_t t_part = t_acc + (uint32_t)a.part_col;
+        for (int ch = 0; ch + 1 < nchunks; ++ch) {
+            if (!mbar_wait(acc_full, ch & 1, abort_flag, a.err)) break;
+            tc_fence_after();
+            for (int col = 0; col < a.n_t; col += 32) {
+                uint32_t r[32];
+                tmem_ld32(t_acc + col, r);
+                if (ch > 0) {
+                    uint32_t p[32];
+                    tmem_ld32(t_part + col, p);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) r[i] = (uint32_t)(__float2int_rn(__uint_as_float(r[i])) + (int)p[i]);
+                } else {
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) r[i] = (uint32_t)__float2int_rn(__uint_as_float(r[i]));
+                }
+                tmem_st32(t_part + col, r);
+            }
+            tmem_wait_st();
+            tc_fence_before();
+            mbar_arrive(acc_empty);
+        }
+    }
+
+    // -------------------------------------------------------------- final epilogue, all eight warps
+    // Warps w and w+4 share TMEM lane quadrant w%4 and split the column groups.
+    // mma_done completes exactly once, after the last MMA (and hence after the
+    // last drain, which the MMA issuer waited for).
+    __syncwarp();
+    bool fin = mbar_wait(mma_done, 0, abort_flag, a.err);
+    fin = __all_sync(0xffffffffu, fin);
+    tc_fence_after();
+    const int esz = a.out_f32 ? 4 : 1;
+    const int row_bytes = a.n_t * esz, row_stride = row_bytes + 16;
+    if (fin) {
+        const int quad = warp & 3;
         const int row = quad * 32 + lane;
         EpiCtx e;
+        e.b_int = cb;
+        e.mult = cb + 256;
+        e.deq = reinterpret_cast<const float *>(cb + 512);
         e.t_acc = tmem + ((uint32_t)(quad * 32) << 16);
         e.t_part = e.t_acc + (uint32_t)a.part_col;
-        e.n0 = n0;
-        const int oy = ho0 + row / a.tw, ox = wo0 + row % a.tw;
-        e.pix = (oy < a.ho && ox < a.wo) ? ((long long)img * a.ho + oy) * a.wo + ox : -1;
-        bool ok = true;
-        for (int ch = 0; ch < nchunks; ++ch) {
-            if (!mbar_wait(acc_full, ch & 1, abort_flag, a.err)) { ok = false; break; }
-            tc_fence_after();
-            if (ch + 1 < nchunks) {
-                for (int col = 0; col < a.n_t; col += 32) {
-                    uint32_t r[32];
-                    tmem_ld32(e.t_acc + col, r);
-                    if (ch > 0) {
-                        uint32_t p[32];
-                        tmem_ld32(e.t_part + col, p);
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) r[i] = (uint32_t)(__float2int_rn(__uint_as_float(r[i])) + (int)p[i]);
-                    } else {
-                        tmem_wait_ld();
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) r[i] = (uint32_t)__float2int_rn(__uint_as_float(r[i]));
-                    }
-                    tmem_st32(e.t_part + col, r);
-                }
-                tmem_wait_st();
-                tc_fence_before();
-                mbar_arrive(acc_empty);
-            }
+        e.has_part = nchunks > 1;
+        // output tile staged in the (now idle) pipeline buffers, rows padded by
+        // 16 bytes so 8 consecutive rows fall in 8 different bank groups
+        e.row = smem + (size_t)row * row_stride;
+        const int G = max(32, max(a.hb_out, a.hb_next));
+        const int mine = warp >> 2;                // warps 4-7 take even groups, 0-3 odd
+        int gi = 0;
+        for (int col = 0; col < a.n_t; col += G, ++gi) {
+            if ((gi & 1) != (mine ^ 1)) continue;
+            if (G == 32) epi_group<32>(e, a, col);
+            else if (G == 64) epi_group<64>(e, a, col);
+            else epi_group128(e, a, col);
         }
-        if (ok) {
-            e.has_part = nchunks > 1;
-            const int G = max(32, max(a.hb_out, a.hb_next));
-            for (int col = 0; col < a.n_t; col += G) {
-                if (G == 32) epi_group<32>(e, a, col);
-                else if (G == 64) epi_group<64>(e, a, col);
-                else epi_group128(e, a, col);
+    }
+    __syncthreads();
+    if (*abort_flag == 0) {
+        // coalesced copy-out: consecutive threads write consecutive 16-byte chunks
+        const int cpr = row_bytes >> 4;
+        for (int j = threadIdx.x; j < kTileM * cpr; j += kThreads) {
+            const int r = j / cpr, c = j - r * cpr;
+            const int oy = ho0 + r / a.tw, ox = wo0 + r % a.tw;
+            if (oy < a.ho && ox < a.wo) {
+                const long long pix = ((long long)img * a.ho + oy) * a.wo + ox;
+                const int4 v = *reinterpret_cast<const int4 *>(smem + (size_t)r * row_stride + c * 16);
+                *reinterpret_cast<int4 *>(static_cast<uint8_t *>(a.y) + (pix * a.co + n0) * esz + c * 16) = v;
             }
         }
     }

@@ -129,20 +129,6 @@ __device__ __forceinline__ uint32_t pack4(int a, int b, int c, int d) {
 __device__ __forceinline__ int lo16(uint32_t r) { return (int)(short)(r & 0xffffu); }
 __device__ __forceinline__ int hi16(uint32_t r) { return ((int)r) >> 16; }
 
-__device__ __forceinline__ void load_f16x16(const __half *p, float (&f)[16]) {
-    const int4 a = __ldg(reinterpret_cast<const int4 *>(p));
-    const int4 b = __ldg(reinterpret_cast<const int4 *>(p) + 1);
-    const uint32_t w[8] = {(uint32_t)a.x, (uint32_t)a.y, (uint32_t)a.z, (uint32_t)a.w,
-                           (uint32_t)b.x, (uint32_t)b.y, (uint32_t)b.z, (uint32_t)b.w};
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        __half2 h2 = *reinterpret_cast<const __half2 *>(&w[i]);
-        const float2 v = __half22float2(h2);
-        f[2 * i] = v.x;
-        f[2 * i + 1] = v.y;
-    }
-}
-
 // MODE 0: static scale. MODE 1: scale from the dynamic parameter block.
 // MODE 2: max-abs pass of the dynamic mode (no store).
 template <bool F16, int MODE>
@@ -161,14 +147,32 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
     }
     uint32_t local_max = 0;
     float local_maxf = 0.f;
+    // Software pipelining: the loads of this warp's next tile are in flight
+    // while the current tile is transformed and stored.
+    int4 cur0 = make_int4(0, 0, 0, 0), cur1 = make_int4(0, 0, 0, 0);
+    auto load_tile = [&](long long t, int4 &v0, int4 &v1) {
+        const long long e0 = (t << 9) + lane * 16;
+        v0 = make_int4(0, 0, 0, 0);
+        v1 = make_int4(0, 0, 0, 0);
+        if (t < tiles && e0 < a.total) {
+            if (!F16) {
+                v0 = __ldg(reinterpret_cast<const int4 *>(static_cast<const int8_t *>(a.x) + e0));
+            } else {
+                const int4 *p = reinterpret_cast<const int4 *>(static_cast<const __half *>(a.x) + e0);
+                v0 = __ldg(p);
+                v1 = __ldg(p + 1);
+            }
+        }
+    };
+    load_tile(warp, cur0, cur1);
     for (long long t = warp; t < tiles; t += nwarps) {
+        int4 nxt0, nxt1;
+        load_tile(t + nwarps, nxt0, nxt1);
         const long long e0 = (t << 9) + lane * 16;
         const bool valid = e0 < a.total;
         if (!F16) {
-            int4 raw = make_int4(0, 0, 0, 0);
-            if (valid) raw = __ldg(reinterpret_cast<const int4 *>(static_cast<const int8_t *>(a.x) + e0));
             uint32_t r[8];
-            unpack_i8x16(raw, r);
+            unpack_i8x16(cur0, r);
             butterfly_i16(r, a.hb, lane);
             if (MODE == 2) {
 #pragma unroll
@@ -188,11 +192,13 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
             }
         } else {
             float f[16];
-            if (valid) {
-                load_f16x16(static_cast<const __half *>(a.x) + e0, f);
-            } else {
+            const uint32_t w[8] = {(uint32_t)cur0.x, (uint32_t)cur0.y, (uint32_t)cur0.z, (uint32_t)cur0.w,
+                                   (uint32_t)cur1.x, (uint32_t)cur1.y, (uint32_t)cur1.z, (uint32_t)cur1.w};
 #pragma unroll
-                for (int i = 0; i < 16; ++i) f[i] = 0.f;
+            for (int i = 0; i < 8; ++i) {
+                const float2 v = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
+                f[2 * i] = v.x;
+                f[2 * i + 1] = v.y;
             }
             butterfly_f32(f, a.hb, lane);
             if (MODE == 2) {
@@ -207,6 +213,8 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
                 *reinterpret_cast<int4 *>(a.y + e0) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
             }
         }
+        cur0 = nxt0;
+        cur1 = nxt1;
     }
     if (MODE == 2) {
         uint32_t m = F16 ? __float_as_uint(local_maxf) : local_max;   // nonnegative floats order as integers

@@ -53,6 +53,8 @@ struct ConvArgs {
     int stages;
     int tmem_cols, part_col;
     int stage_bytes, b_bytes, raw_bytes;
+    int const_off;                   // offsets from the barrier area: epilogue constants,
+    int win_off, win_h, win_w;       // small-channel input window and its size
     const int8_t *x;
     const int32_t *b_int;
     const int32_t *mult;
