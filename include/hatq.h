@@ -193,6 +193,26 @@ hatq_status hatq_layer(const void *x, int x_kind, float s_in, int n, int h, int 
                        const hatq_prepared *L, void *y, void *scratch, size_t scratch_bytes,
                        hatq_stream stream);
 
+/*
+ * hatq_layer for callers that cannot allocate device memory (code running
+ * where cudaMalloc is not allowed or not available: host callbacks, plugins
+ * whose host engine owns every allocation, allocator-less embeddings). The
+ * paper has no counterpart: this only moves hatq_layer's scratch buffer.
+ * The INT8 operand that hatq_layer would stage in `scratch` is staged in a
+ * fixed device array of HATQ_NOALLOC_MAX_BYTES bytes that the library holds
+ * on every device that loads it, until the process exits. An operand larger
+ * than that (n*h*w*c_in bytes) returns HATQ_ERR_INVALID_ARG before any launch.
+ * Nothing is allocated: no cudaMalloc/cudaFree and no allocating library call.
+ * The first call on a device looks up the array's device address with that
+ * device current; make that first call before any stream capture. All calls
+ * share the array and it keeps the last call's contents; calls whose GPU work
+ * overlaps (unordered streams) race on it. Inputs and outputs are the
+ * caller's, as in hatq_layer.
+ */
+#define HATQ_NOALLOC_MAX_BYTES (32u << 20)
+hatq_status hatq_layer_noalloc(const void *x, int x_kind, float s_in, int n, int h, int w,
+                               const hatq_prepared *L, void *y, hatq_stream stream);
+
 /* Number of kernel launches hatq_layer / hatq_conv2d_i8 make for these
  * arguments (for launch accounting), or -1 for invalid arguments. */
 int hatq_layer_launches(int x_kind, float s_in, const hatq_prepared *L);

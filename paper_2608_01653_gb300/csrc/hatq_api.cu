@@ -206,6 +206,8 @@ hatq_status validate_prepare(const hatq_conv_desc *d, const float *w_ohwi, float
 
 }  // namespace
 
+hatq_status hatq::report(hatq_status st, const char *msg) { return fail(st, "%s", msg); }
+
 extern "C" {
 
 int hatq_version(void) { return (0 << 16) | 1; }

@@ -6,7 +6,12 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "hatq.h"
+
 namespace hatq {
+
+// Records `msg` as the calling thread's hatq_last_error() and returns st.
+hatq_status report(hatq_status st, const char *msg);
 
 // Error word codes written by kernels (read back by hatq_sync_status).
 enum : int { kErrNone = 0, kErrWaitTimeout = 1, kErrBounds = 2 };

@@ -276,3 +276,21 @@ def sync_status(stream=None):
 
 def version() -> int:
     return int(load().hatq_version())
+
+
+def layer_noalloc(x, x_kind, s_in, L: PreparedLayer, y=None, stream=None):
+    """hatq_layer_noalloc: hatq_layer for callers that cannot allocate device
+    memory; the staged INT8 operand lives in the library's fixed device array
+    (at most HATQ_NOALLOC_MAX_BYTES bytes, shared by all calls)."""
+    torch = _torch()
+    fn = load().hatq_layer_noalloc
+    fn.restype = _I
+    fn.argtypes = [_P, _I, _F, _I, _I, _I, ctypes.POINTER(PreparedStruct), _P, _P]
+    n, h, w, c = x.shape
+    if y is None:
+        y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32 if L.out_f32 else torch.int8, device=x.device)
+    _check(fn(_ptr(x), int(x_kind), float(s_in), n, h, w, ctypes.byref(L.struct), _ptr(y), _stream(stream)))
+    return y
+
+
+NOALLOC_MAX_BYTES = 32 << 20
