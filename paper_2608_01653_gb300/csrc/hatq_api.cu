@@ -448,21 +448,39 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     a.b_bytes = a.n_t * 128;
     a.raw_bytes = g.gather ? 0 : 8192;
     a.stage_bytes = 16384 + a.b_bytes + a.raw_bytes;
-    // reserve room for barriers, the gather table, epilogue constants and the input window
-    int win_reserve = 0;
-    if (g.gather) {
-        const int wh = (a.th - 1) * d->stride + d->kh, ww = (a.tw - 1) * d->stride + d->kw;
-        win_reserve = (wh * ww * d->c_in + 127) & ~127;
+    a.n_tiles_n = d->c_out / a.n_t;
+    {
+        const long long nt = (long long)n * a.tiles_w * a.tiles_h * a.n_tiles_n;
+        if (nt >= (1LL << 31)) return fail(HATQ_ERR_UNSUPPORTED, "too many output tiles");
+        a.num_tiles = (int)nt;
     }
-    const int smem_cap = 227 * 1024 - 1024 - 1024 - 256 - 3 * 1024 - 128 - (g.gather ? g.k_pad * 4 : 0) - win_reserve;
-    a.stages = smem_cap / a.stage_bytes;
+    // TMEM: one or two accumulator buffers of n_t fp32 columns (+ n_t int32
+    // partial columns when the reduction spans several exact chunks)
+    const bool drains = a.num_kb > a.chunk_kb;
+    a.buf_cols = a.n_t * (drains ? 2 : 1);
+    a.nbuf = 2 * a.buf_cols <= 512 ? 2 : 1;
+    a.tmem_cols = 32;
+    while (a.tmem_cols < a.nbuf * a.buf_cols) a.tmem_cols <<= 1;
+    // shared memory: [stages][output tiles][barriers | gather table | constants | window]
+    const int esz = L->out_f32 ? 4 : 1;
+    a.row_stride = a.n_t * esz + 16;                 // padded rows: 8 consecutive rows hit 8 bank groups
+    a.staging_bytes = L->out_f32 ? 0 : a.nbuf * kTileRows * a.row_stride;   // float32 output is stored directly
+    a.win_h = (a.th - 1) * d->stride + d->kh;
+    a.win_w = (a.tw - 1) * d->stride + d->kw;
+    const int win_bytes = g.gather ? (a.win_h * a.win_w * d->c_in + 127) & ~127 : 0;
+    const int table_bytes = g.gather ? a.num_kb * 64 * 4 : 0;
+    const int const_bytes = (3 * d->c_out * 4 + 127) & ~127;
+    const int fixed = 1024 /* align */ + 8 * (3 * 8 + 7) + 16 + 128 + table_bytes + const_bytes + win_bytes;
+    const int budget = 227 * 1024 - 1024 /* static */ - fixed - a.staging_bytes;
+    a.stages = budget / a.stage_bytes;
     if (a.stages > 8) a.stages = 8;
     if (g.gather && a.stages > 4) a.stages = 4;
     if (a.stages < 2) return fail(HATQ_ERR_UNSUPPORTED, "tile does not fit in shared memory");
-    int pc = 32;
-    while (pc < a.n_t) pc <<= 1;
-    a.part_col = pc;
-    a.tmem_cols = a.num_kb > a.chunk_kb ? 2 * pc : pc;
+    const int bar_bytes = 8 * (3 * a.stages + 7) + 16;
+    a.const_off = (bar_bytes + table_bytes + 127) & ~127;
+    a.win_off = a.const_off + const_bytes;
+    const int smem_bytes = a.stages * a.stage_bytes + a.staging_bytes + 1024 + a.win_off + win_bytes;
+    if (smem_bytes > 227 * 1024 - 1024) return fail(HATQ_ERR_UNSUPPORTED, "shared memory budget exceeded (%d bytes)", smem_bytes);
     a.x = x;
     a.b_int = L->b_int;
     a.mult = L->mult;
@@ -475,18 +493,6 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     a.y = y;
     a.err = err_word();
     if (!a.err) return fail(HATQ_ERR_CUDA, "no CUDA device");
-    // dynamic shared memory: [stages][barriers | gather table | constants | window]
-    const int bar_bytes = 8 * (3 * a.stages + 3) + 16;
-    const int table_bytes = g.gather ? a.num_kb * 64 * 4 : 0;
-    a.const_off = (bar_bytes + table_bytes + 127) & ~127;
-    a.win_off = a.const_off + 3 * 256 * 4;
-    a.win_h = (a.th - 1) * d->stride + d->kh;
-    a.win_w = (a.tw - 1) * d->stride + d->kw;
-    const int win_bytes = g.gather ? (a.win_h * a.win_w * d->c_in + 127) & ~127 : 0;
-    const int smem_bytes = a.stages * a.stage_bytes + 1024 + a.win_off + win_bytes;
-    const int out_stage = kTileRows * (a.n_t * (L->out_f32 ? 4 : 1) + 16);
-    if (out_stage > a.stages * a.stage_bytes) return fail(HATQ_ERR_UNSUPPORTED, "output tile does not fit the stage buffers");
-    if (smem_bytes > 227 * 1024 - 1024) return fail(HATQ_ERR_UNSUPPORTED, "shared memory budget exceeded (%d bytes)", smem_bytes);
 
     CUtensorMap tmB, tmA;
     std::memcpy(&tmB, L->opaque, sizeof tmB);

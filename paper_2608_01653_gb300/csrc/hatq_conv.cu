@@ -39,7 +39,7 @@
 namespace hatq {
 namespace {
 
-constexpr int kThreads = 256;
+constexpr int kThreads = 384;
 constexpr int kConvThreads = 64;       // converter warps 2-3
 constexpr int kBlockK = 64;            // fp16 elements per 128-byte swizzle row
 constexpr int kTileM = 128;
@@ -243,7 +243,8 @@ struct EpiCtx {
     uint32_t t_acc;      // TMEM address of this warp's lanes, column 0 of the accumulator
     uint32_t t_part;     // ... of the int32 partial region
     bool has_part;
-    uint8_t *row;        // this thread's row of the shared-memory output tile
+    uint8_t *row;        // this thread's row of the shared-memory output tile (INT8 output)
+    float *gout;         // float32 output: this thread's pixel row in global memory, or null
 };
 
 // Exact int32 accumulator of 16 columns starting at tile column `col`, bias included.
@@ -310,11 +311,13 @@ __device__ __forceinline__ void store_codes(const ConvArgs &a, uint8_t *row, int
         reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
     }
 }
+// Float32 output goes straight to global memory (no shared-memory staging).
 template <int G>
-__device__ __forceinline__ void store_f32(uint8_t *row, int col, const float (&t)[G]) {
+__device__ __forceinline__ void store_f32(float *gout, int col, const float (&t)[G]) {
+    if (!gout) return;
 #pragma unroll
     for (int i = 0; i < G / 4; ++i)
-        reinterpret_cast<float4 *>(row + 4 * col)[i] = make_float4(t[4 * i], t[4 * i + 1], t[4 * i + 2], t[4 * i + 3]);
+        reinterpret_cast<float4 *>(gout + col)[i] = make_float4(t[4 * i], t[4 * i + 1], t[4 * i + 2], t[4 * i + 3]);
 }
 
 __device__ __forceinline__ long long relu(long long v) { return ((int)(v >> 32)) < 0 ? 0LL : v; }
@@ -351,7 +354,7 @@ __device__ __forceinline__ void epi_group(const EpiCtx &e, const ConvArgs &a, in
 #pragma unroll
             for (int i = 0; i < G; ++i) t[i] = relu(t[i]);
         }
-        store_f32<G>(e.row, col, t);
+        store_f32<G>(e.gout, col, t);
     }
 }
 
@@ -407,29 +410,37 @@ __device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a,
 #pragma unroll
                 for (int i = 0; i < 64; ++i) s[i] = relu(s[i]);
             }
-            store_f32<64>(e.row, col + 64 * pass, s);
+            store_f32<64>(e.gout, col + 64 * pass, s);
         }
     }
 }
 
 // ------------------------------------------------------------------ kernel
 
+// One CTA per SM, looping over output tiles (tile t -> M tile t / n_tiles_n,
+// N tile t % n_tiles_n). The stage ring runs continuously across tiles. The
+// accumulator is double-buffered in TMEM when two buffers fit: epilogue
+// warpgroup w then takes the tiles of buffer w while the MMA issuer already
+// fills the other buffer; with one buffer both epilogue warpgroups split the
+// columns of every tile.
 __global__ void __launch_bounds__(kThreads, 1)
     conv_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const ConvArgs a) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = a.stages;
-    uint8_t *bar_area = smem + (size_t)S * a.stage_bytes;
+    uint8_t *staging = smem + (size_t)S * a.stage_bytes;
+    uint8_t *bar_area = staging + (size_t)a.staging_bytes;
     const uint32_t bar0 = smem_addr(bar_area);
-    // barriers: full[S], conv[S], empty[S], acc_full, acc_empty, mma_done
+    // barriers: full[S], conv[S], empty[S], acc_full[2], acc_empty[2], acc_free[2], mma_done
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
     auto conv_bar = [&](int s) { return bar0 + 8u * (S + s); };
     auto empty_bar = [&](int s) { return bar0 + 8u * (2 * S + s); };
-    const uint32_t acc_full = bar0 + 8u * (3 * S);
-    const uint32_t acc_empty = acc_full + 8;
-    const uint32_t mma_done = acc_full + 16;
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_area + 8 * (3 * S + 3));
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_area + 8 * (3 * S + 3) + 4);
+    auto acc_full = [&](int b) { return bar0 + 8u * (3 * S + b); };
+    auto acc_empty = [&](int b) { return bar0 + 8u * (3 * S + 2 + b); };
+    auto acc_free = [&](int b) { return bar0 + 8u * (3 * S + 4 + b); };
+    const uint32_t mma_done = bar0 + 8u * (3 * S + 6);
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_area + 8 * (3 * S + 7));
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_area + 8 * (3 * S + 7) + 4);
 
     // A failure already recorded by this launch (or an earlier, unread one)
     // ends every CTA that has not started, so a fault cannot serialize waits.
@@ -441,15 +452,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-
-    // tile coordinates
     const int tiles_per_img = a.tiles_w * a.tiles_h;
-    const int img = blockIdx.x / tiles_per_img;
-    const int rem = blockIdx.x - img * tiles_per_img;
-    const int ty = rem / a.tiles_w;
-    const int tx = rem - ty * a.tiles_w;
-    const int ho0 = ty * a.th, wo0 = tx * a.tw;
-    const int n0 = blockIdx.y * a.n_t;
+    const int nbuf = a.nbuf;
+    const int ep_count = nbuf == 2 ? 128 : 256;     // epilogue threads that arrive per buffer
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -457,8 +462,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(conv_bar(s), kConvThreads);
             mbar_init(empty_bar(s), 1);
         }
-        mbar_init(acc_full, 1);
-        mbar_init(acc_empty, 128);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(acc_full(b), 1);
+            mbar_init(acc_empty(b), ep_count);
+            mbar_init(acc_free(b), ep_count);
+        }
         mbar_init(mma_done, 1);
         *abort_flag = 0;
         fence_barrier_init();
@@ -469,13 +477,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
-    // per-tile bias codes, multipliers and dequant factors for the epilogue,
-    // staged once (128-byte aligned, read with 16-byte vector loads)
+    // bias codes, multipliers and dequant factors of all output channels,
+    // staged once per CTA (128-byte aligned, read with 16-byte vector loads)
     int *cb = reinterpret_cast<int *>(bar_area + a.const_off);
-    for (int c = threadIdx.x; c < a.n_t; c += kThreads) {
-        cb[c] = a.b_int[n0 + c];
-        cb[256 + c] = a.mult[n0 + c];
-        reinterpret_cast<float *>(cb)[512 + c] = a.deq[n0 + c];
+    for (int c = threadIdx.x; c < a.co; c += kThreads) {
+        cb[c] = a.b_int[c];
+        cb[a.co + c] = a.mult[c];
+        reinterpret_cast<float *>(cb)[2 * a.co + c] = a.deq[c];
     }
     tc_fence_before();
     __syncthreads();
@@ -483,7 +491,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = *tmem_holder;
 
     const int nchunks = (a.num_kb + a.chunk_kb - 1) / a.chunk_kb;
+    const int my_tiles = a.num_tiles > (int)blockIdx.x ? (a.num_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
+    auto tile_coords = [&](int j, int &img, int &ho0, int &wo0, int &n0) {
+        const int t = (int)blockIdx.x + j * (int)gridDim.x;
+        const int mt = t / a.n_tiles_n;
+        n0 = (t - mt * a.n_tiles_n) * a.n_t;
+        img = mt / tiles_per_img;
+        const int rem = mt - img * tiles_per_img;
+        const int ty = rem / a.tiles_w;
+        ho0 = ty * a.th;
+        wo0 = (rem - ty * a.tiles_w) * a.tw;
+    };
 
+    // Register split: warpgroup 0 (producer, MMA issuer, converters) gives
+    // registers up, the two epilogue warpgroups take them (launch: 384 x 168;
+    // after: 128 x 88 + 256 x 208 = 64512, and per scheduler 88 + 2 x 208 <= 512).
+    if (warp < 4) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 88;" ::: "memory");
     if (warp == 0) {
         // ---------------------------------------------------------- TMA producer
         if (lane == 0) {
@@ -491,20 +515,25 @@ __global__ void __launch_bounds__(kThreads, 1)
             int issued_round[8];
             for (int s = 0; s < 8; ++s) issued_round[s] = -1;
             bool ok = true;
-            for (int kb = 0; kb < a.num_kb && ok; ++kb) {
-                const int s = kb % S, r = kb / S;
-                if (!mbar_wait(empty_bar(s), (r & 1) ^ 1, abort_flag, a.err)) { ok = false; break; }
-                const uint32_t st = smem_addr(smem + (size_t)s * a.stage_bytes);
-                mbar_expect_tx(full_bar(s), tx_bytes);
-                tma_load_2d(st + 16384, &tmB, full_bar(s), kb * kBlockK, n0);
-                if (!a.gather) {
-                    const int tap = kb / a.cin_kb;
-                    const int c0 = (kb - tap * a.cin_kb) * kBlockK;
-                    const int ky = tap / a.kw, kx = tap - (tap / a.kw) * a.kw;
-                    tma_load_4d(st + 16384 + a.b_bytes, &tmA, full_bar(s), c0, wo0 * a.stride + kx - a.pad,
-                                ho0 * a.stride + ky - a.pad, img);
+            int it = 0;
+            for (int j = 0; j < my_tiles && ok; ++j) {
+                int img, ho0, wo0, n0;
+                tile_coords(j, img, ho0, wo0, n0);
+                for (int kb = 0; kb < a.num_kb; ++kb, ++it) {
+                    const int s = it % S, r = it / S;
+                    if (!mbar_wait(empty_bar(s), (r & 1) ^ 1, abort_flag, a.err)) { ok = false; break; }
+                    const uint32_t st = smem_addr(smem + (size_t)s * a.stage_bytes);
+                    mbar_expect_tx(full_bar(s), tx_bytes);
+                    tma_load_2d(st + 16384, &tmB, full_bar(s), kb * kBlockK, n0);
+                    if (!a.gather) {
+                        const int tap = kb / a.cin_kb;
+                        const int c0 = (kb - tap * a.cin_kb) * kBlockK;
+                        const int ky = tap / a.kw, kx = tap - (tap / a.kw) * a.kw;
+                        tma_load_4d(st + 16384 + a.b_bytes, &tmA, full_bar(s), c0, wo0 * a.stride + kx - a.pad,
+                                    ho0 * a.stride + ky - a.pad, img);
+                    }
+                    issued_round[s] = r;
                 }
-                issued_round[s] = r;
             }
             if (!ok) {
                 // let our own copies land before the CTA unwinds
@@ -521,25 +550,36 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             const uint32_t idesc = idesc_f16(a.n_t);
             bool ok = true;
-            for (int kb = 0; kb < a.num_kb && ok; ++kb) {
-                const int s = kb % S, r = kb / S;
-                const int ck = kb % a.chunk_kb;
-                if (ck == 0 && kb > 0) {
-                    const int ch = kb / a.chunk_kb;    // wait until chunk ch-1 was drained
-                    if (!mbar_wait(acc_empty, (ch - 1) & 1, abort_flag, a.err)) { ok = false; break; }
+            int it = 0;
+            int empty_cnt[2] = {0, 0};
+            for (int j = 0; j < my_tiles && ok; ++j) {
+                const int b = j % nbuf;
+                const uint32_t d_tmem = tmem + (uint32_t)(b * a.buf_cols);
+                if (j >= nbuf) {      // wait until the epilogue released this buffer
+                    if (!mbar_wait(acc_free(b), ((j / nbuf) - 1) & 1, abort_flag, a.err)) { ok = false; break; }
                     tc_fence_after();
                 }
-                if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
-                if (!mbar_wait(conv_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
-                tc_fence_after();
-                const uint32_t st = smem_addr(smem + (size_t)s * a.stage_bytes);
-                const uint64_t da = sdesc_sw128(st);
-                const uint64_t db = sdesc_sw128(st + 16384);
+                for (int kb = 0; kb < a.num_kb; ++kb, ++it) {
+                    const int s = it % S, r = it / S;
+                    const int ck = kb % a.chunk_kb;
+                    if (ck == 0 && kb > 0) {   // wait until the previous chunk was drained
+                        if (!mbar_wait(acc_empty(b), empty_cnt[b] & 1, abort_flag, a.err)) { ok = false; break; }
+                        ++empty_cnt[b];
+                        tc_fence_after();
+                    }
+                    if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
+                    if (!mbar_wait(conv_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t st = smem_addr(smem + (size_t)s * a.stage_bytes);
+                    const uint64_t da = sdesc_sw128(st);
+                    const uint64_t db = sdesc_sw128(st + 16384);
 #pragma unroll
-                for (int kk = 0; kk < kBlockK / 16; ++kk)   // K = 16 per instruction, 32 bytes apart
-                    umma_f16(tmem, da + (uint64_t)(2 * kk), db + (uint64_t)(2 * kk), idesc, (ck > 0 || kk > 0) ? 1u : 0u);
-                umma_commit(empty_bar(s));
-                if (ck == a.chunk_kb - 1 || kb == a.num_kb - 1) umma_commit(acc_full);
+                    for (int kk = 0; kk < kBlockK / 16; ++kk)   // K = 16 per instruction, 32 bytes apart
+                        umma_f16(d_tmem, da + (uint64_t)(2 * kk), db + (uint64_t)(2 * kk), idesc,
+                                 (ck > 0 || kk > 0) ? 1u : 0u);
+                    umma_commit(empty_bar(s));
+                    if (ck == a.chunk_kb - 1 || kb == a.num_kb - 1) umma_commit(acc_full(b));
+                }
             }
             umma_commit(mma_done);
             const long long t0 = clock64();
@@ -550,39 +590,44 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------------------------------------------------- converters
         constexpr int kPasses = 512 / kConvThreads;   // 128 rows x 4 quarters per 64-wide block
         const int ct = threadIdx.x - 64;              // 0..kConvThreads-1
+        int it = 0;
+        bool ok = true;
         if (!a.gather) {
-            for (int kb = 0; kb < a.num_kb; ++kb) {
-                const int s = kb % S, r = kb / S;
-                if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) break;
-                uint8_t *st = smem + (size_t)s * a.stage_bytes;
-                const uint8_t *raw = st + 16384 + a.b_bytes;
-                int4 v[kPasses];                       // all loads first, then convert and store
+            for (int j = 0; j < my_tiles && ok; ++j) {
+                for (int kb = 0; kb < a.num_kb; ++kb, ++it) {
+                    const int s = it % S, r = it / S;
+                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
+                    if (!ok) break;
+                    uint8_t *st = smem + (size_t)s * a.stage_bytes;
+                    const uint8_t *raw = st + 16384 + a.b_bytes;
+                    int4 v[kPasses];                       // all loads first, then convert and store
 #pragma unroll
-                for (int p = 0; p < kPasses; ++p) {
-                    const int idx = p * kConvThreads + ct;
-                    v[p] = *reinterpret_cast<const int4 *>(raw + (idx >> 2) * 64 + (idx & 3) * 16);
-                }
+                    for (int p = 0; p < kPasses; ++p) {
+                        const int idx = p * kConvThreads + ct;
+                        v[p] = *reinterpret_cast<const int4 *>(raw + (idx >> 2) * 64 + (idx & 3) * 16);
+                    }
 #pragma unroll
-                for (int p = 0; p < kPasses; ++p) {
-                    const int idx = p * kConvThreads + ct;
-                    const int m = idx >> 2, q = idx & 3;    // row, 16-element quarter of the 64-wide block
-                    uint32_t h[8];
-                    i8x4_to_f16x4((uint32_t)v[p].x, h[0], h[1]);
-                    i8x4_to_f16x4((uint32_t)v[p].y, h[2], h[3]);
-                    i8x4_to_f16x4((uint32_t)v[p].z, h[4], h[5]);
-                    i8x4_to_f16x4((uint32_t)v[p].w, h[6], h[7]);
-                    *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
-                    *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
+                    for (int p = 0; p < kPasses; ++p) {
+                        const int idx = p * kConvThreads + ct;
+                        const int m = idx >> 2, q = idx & 3;    // row, 16-element quarter of the 64-wide block
+                        uint32_t h[8];
+                        i8x4_to_f16x4((uint32_t)v[p].x, h[0], h[1]);
+                        i8x4_to_f16x4((uint32_t)v[p].y, h[2], h[3]);
+                        i8x4_to_f16x4((uint32_t)v[p].z, h[4], h[5]);
+                        i8x4_to_f16x4((uint32_t)v[p].w, h[6], h[7]);
+                        *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
+                        *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
+                    }
+                    fence_proxy_async_smem();
+                    mbar_arrive(conv_bar(s));
                 }
-                fence_proxy_async_smem();
-                mbar_arrive(conv_bar(s));
             }
         } else {
-            // Small-channel layer: the tile's input window ((th-1)s+kh rows of
+            // Small-channel layer: each tile's input window ((th-1)s+kh rows of
             // (tw-1)s+kw pixels, zero outside the image) is copied to shared
             // memory with coalesced byte loads, then the packed reduction index
             // k = (ky, kx, ci) is gathered from it through a per-CTA offset table.
-            int *tab = reinterpret_cast<int *>(bar_area + 8 * (3 * S + 3) + 16);
+            int *tab = reinterpret_cast<int *>(bar_area + 8 * (3 * S + 7) + 16);
             uint8_t *win = bar_area + a.win_off;
             const int taps = a.kh * a.kw;
             for (int k = ct; k < a.num_kb * kBlockK; k += kConvThreads) {
@@ -590,123 +635,155 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int ky = tap / a.kw, kx = tap - ky * a.kw;
                 tab[k] = tap < taps ? (ky * a.win_w + kx) * a.c + ci : -1;
             }
-            {
-                const int ix_lo = wo0 * a.stride - a.pad;
-                const int row_b = a.win_w * a.c;
-                const int b_lo = max(0, -ix_lo) * a.c, b_hi = min(a.win_w, a.w - ix_lo) * a.c;
-                for (int r = 0; r < a.win_h; ++r) {
-                    const int iy = ho0 * a.stride - a.pad + r;
-                    const bool row_in = iy >= 0 && iy < a.h;
-                    const int8_t *src = a.x + (((long long)img * a.h + (row_in ? iy : 0)) * a.w + ix_lo) * a.c;
-                    for (int b = ct; b < row_b; b += kConvThreads)
-                        win[r * row_b + b] = (row_in && b >= b_lo && b < b_hi) ? (uint8_t)__ldg(src + b) : (uint8_t)0;
-                }
-            }
-            asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");
             int rb[kPasses];
 #pragma unroll
             for (int p = 0; p < kPasses; ++p) {
                 const int m = (p * kConvThreads + ct) >> 2;
                 rb[p] = ((m / a.tw) * a.stride * a.win_w + (m % a.tw) * a.stride) * a.c;
             }
-            for (int kb = 0; kb < a.num_kb; ++kb) {
-                const int s = kb % S, r = kb / S;
-                if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) break;
-                uint8_t *st = smem + (size_t)s * a.stage_bytes;
-#pragma unroll
-                for (int p = 0; p < kPasses; ++p) {
-                    const int idx = p * kConvThreads + ct;
-                    const int m = idx >> 2, q = idx & 3;
-                    uint32_t w4[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) {
-                        const int off = tab[kb * kBlockK + q * 16 + j];
-                        const uint32_t b = off >= 0 ? (uint32_t)win[rb[p] + off] : 0u;
-                        w4[j >> 2] |= b << (8 * (j & 3));
+            // Every converter thread runs the same tile loop (also after an
+            // abort, doing no work) so both warps reach each named barrier.
+            for (int j = 0; j < my_tiles; ++j) {
+                int img, ho0, wo0, n0;
+                tile_coords(j, img, ho0, wo0, n0);
+                asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // previous window consumed
+                if (ok) {
+                    const int ix_lo = wo0 * a.stride - a.pad;
+                    const int row_b = a.win_w * a.c;
+                    const int b_lo = max(0, -ix_lo) * a.c, b_hi = min(a.win_w, a.w - ix_lo) * a.c;
+                    for (int r = 0; r < a.win_h; ++r) {
+                        const int iy = ho0 * a.stride - a.pad + r;
+                        const bool row_in = iy >= 0 && iy < a.h;
+                        const int8_t *src = a.x + (((long long)img * a.h + (row_in ? iy : 0)) * a.w + ix_lo) * a.c;
+                        for (int b = ct; b < row_b; b += kConvThreads)
+                            win[r * row_b + b] = (row_in && b >= b_lo && b < b_hi) ? (uint8_t)__ldg(src + b) : (uint8_t)0;
                     }
-                    uint32_t h[8];
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) i8x4_to_f16x4(w4[j], h[2 * j], h[2 * j + 1]);
-                    *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
-                    *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
                 }
-                fence_proxy_async_smem();
-                mbar_arrive(conv_bar(s));
+                asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // window complete
+                for (int kb = 0; kb < a.num_kb && ok; ++kb, ++it) {
+                    const int s = it % S, r = it / S;
+                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
+                    if (!ok) break;
+                    uint8_t *st = smem + (size_t)s * a.stage_bytes;
+#pragma unroll
+                    for (int p = 0; p < kPasses; ++p) {
+                        const int idx = p * kConvThreads + ct;
+                        const int m = idx >> 2, q = idx & 3;
+                        uint32_t w4[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+                        for (int jj = 0; jj < 16; ++jj) {
+                            const int off = tab[kb * kBlockK + q * 16 + jj];
+                            const uint32_t bb = off >= 0 ? (uint32_t)win[rb[p] + off] : 0u;
+                            w4[jj >> 2] |= bb << (8 * (jj & 3));
+                        }
+                        uint32_t h[8];
+#pragma unroll
+                        for (int jj = 0; jj < 4; ++jj) i8x4_to_f16x4(w4[jj], h[2 * jj], h[2 * jj + 1]);
+                        *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
+                        *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
+                    }
+                    fence_proxy_async_smem();
+                    mbar_arrive(conv_bar(s));
+                }
             }
         }
+    }
     } else {
-        // ---------------------------------------------------------- drains (chunk sums -> int32 partial)
-        const uint32_t t_acc = tmem + ((uint32_t)((warp & 3) * 32) << 16);
-        const uint32_t t_part = t_acc + (uint32_t)a.part_col;
-        for (int ch = 0; ch + 1 < nchunks; ++ch) {
-            if (!mbar_wait(acc_full, ch & 1, abort_flag, a.err)) break;
-            tc_fence_after();
-            for (int col = 0; col < a.n_t; col += 32) {
-                uint32_t r[32];
-                tmem_ld32(t_acc + col, r);
-                if (ch > 0) {
-                    uint32_t p[32];
-                    tmem_ld32(t_part + col, p);
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) r[i] = (uint32_t)(__float2int_rn(__uint_as_float(r[i])) + (int)p[i]);
-                } else {
-                    tmem_wait_ld();
-#pragma unroll
-                    for (int i = 0; i < 32; ++i) r[i] = (uint32_t)__float2int_rn(__uint_as_float(r[i]));
-                }
-                tmem_st32(t_part + col, r);
-            }
-            tmem_wait_st();
-            tc_fence_before();
-            mbar_arrive(acc_empty);
-        }
-    }
-
-    // -------------------------------------------------------------- final epilogue, all eight warps
-    // Warps w and w+4 share TMEM lane quadrant w%4 and split the column groups.
-    // mma_done completes exactly once, after the last MMA (and hence after the
-    // last drain, which the MMA issuer waited for).
-    __syncwarp();
-    bool fin = mbar_wait(mma_done, 0, abort_flag, a.err);
-    fin = __all_sync(0xffffffffu, fin);
-    tc_fence_after();
-    const int esz = a.out_f32 ? 4 : 1;
-    const int row_bytes = a.n_t * esz, row_stride = row_bytes + 16;
-    if (fin) {
-        const int quad = warp & 3;
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 208;" ::: "memory");
+        // ---------------------------------------------------------- epilogue warpgroups (warps 4-7, 8-11)
+        const int wg = (warp - 4) >> 2;            // 0 or 1
+        const int quad = warp & 3;                 // TMEM lane quadrant this warp may access
         const int row = quad * 32 + lane;
-        EpiCtx e;
-        e.b_int = cb;
-        e.mult = cb + 256;
-        e.deq = reinterpret_cast<const float *>(cb + 512);
-        e.t_acc = tmem + ((uint32_t)(quad * 32) << 16);
-        e.t_part = e.t_acc + (uint32_t)a.part_col;
-        e.has_part = nchunks > 1;
-        // output tile staged in the (now idle) pipeline buffers, rows padded by
-        // 16 bytes so 8 consecutive rows fall in 8 different bank groups
-        e.row = smem + (size_t)row * row_stride;
+        const int et = threadIdx.x - 128 - 128 * wg;   // 0..127 within the warpgroup
+        const int esz = a.out_f32 ? 4 : 1;
+        const int row_bytes = a.n_t * esz;
+        uint8_t *stage_tile = staging + (size_t)(nbuf == 2 ? wg : 0) * kTileM * a.row_stride;
         const int G = max(32, max(a.hb_out, a.hb_next));
-        const int mine = warp >> 2;                // warps 4-7 take even groups, 0-3 odd
-        int gi = 0;
-        for (int col = 0; col < a.n_t; col += G, ++gi) {
-            if ((gi & 1) != (mine ^ 1)) continue;
-            if (G == 32) epi_group<32>(e, a, col);
-            else if (G == 64) epi_group<64>(e, a, col);
-            else epi_group128(e, a, col);
-        }
-    }
-    __syncthreads();
-    if (*abort_flag == 0) {
-        // coalesced copy-out: consecutive threads write consecutive 16-byte chunks
-        const int cpr = row_bytes >> 4;
-        for (int j = threadIdx.x; j < kTileM * cpr; j += kThreads) {
-            const int r = j / cpr, c = j - r * cpr;
-            const int oy = ho0 + r / a.tw, ox = wo0 + r % a.tw;
-            if (oy < a.ho && ox < a.wo) {
-                const long long pix = ((long long)img * a.ho + oy) * a.wo + ox;
-                const int4 v = *reinterpret_cast<const int4 *>(smem + (size_t)r * row_stride + c * 16);
-                *reinterpret_cast<int4 *>(static_cast<uint8_t *>(a.y) + (pix * a.co + n0) * esz + c * 16) = v;
+        int full_cnt[2] = {0, 0};
+        bool ok = true;
+        // Every epilogue thread runs the same loops (also after an abort, doing
+        // no work) so the warpgroup reaches each named barrier together.
+        for (int j = 0; j < my_tiles; ++j) {
+            const int b = j % nbuf;
+            if (nbuf == 2 && b != wg) continue;
+            int img, ho0, wo0, n0;
+            tile_coords(j, img, ho0, wo0, n0);
+            const uint32_t t_acc = tmem + (uint32_t)(b * a.buf_cols) + ((uint32_t)(quad * 32) << 16);
+            const uint32_t t_part = t_acc + (uint32_t)a.n_t;
+            for (int ch = 0; ch < nchunks; ++ch) {
+                if (ok) {
+                    ok = __all_sync(0xffffffffu, mbar_wait(acc_full(b), full_cnt[b] & 1, abort_flag, a.err));
+                    ++full_cnt[b];
+                    tc_fence_after();
+                }
+                if (ch + 1 < nchunks) {
+                    if (!ok) continue;
+                    // drain: chunk sum -> int32 partial (with one buffer the two warpgroups split the columns)
+                    for (int col = 0; col < a.n_t; col += 32) {
+                        if (nbuf == 1 && ((col >> 5) & 1) != wg) continue;
+                        uint32_t r[32];
+                        tmem_ld32(t_acc + col, r);
+                        if (ch > 0) {
+                            uint32_t p[32];
+                            tmem_ld32(t_part + col, p);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) r[i] = (uint32_t)(__float2int_rn(__uint_as_float(r[i])) + (int)p[i]);
+                        } else {
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) r[i] = (uint32_t)__float2int_rn(__uint_as_float(r[i]));
+                        }
+                        tmem_st32(t_part + col, r);
+                    }
+                    tmem_wait_st();
+                    tc_fence_before();
+                    mbar_arrive(acc_empty(b));
+                    continue;
+                }
+                // final chunk: epilogue into the shared-memory output tile
+                if (ok) {
+                EpiCtx e;
+                e.b_int = cb + n0;
+                e.mult = cb + a.co + n0;
+                e.deq = reinterpret_cast<const float *>(cb + 2 * a.co) + n0;
+                e.t_acc = t_acc;
+                e.t_part = t_part;
+                e.has_part = nchunks > 1;
+                e.row = stage_tile + (size_t)row * a.row_stride;
+                e.gout = nullptr;
+                if (a.out_f32) {
+                    const int oy = ho0 + row / a.tw, ox = wo0 + row % a.tw;
+                    if (oy < a.ho && ox < a.wo)
+                        e.gout = static_cast<float *>(a.y) + (((long long)img * a.ho + oy) * a.wo + ox) * a.co + n0;
+                }
+                int gi = 0;
+                for (int col = 0; col < a.n_t; col += G, ++gi) {
+                    if (nbuf == 1 && (gi & 1) != wg) continue;
+                    if (G == 32) epi_group<32>(e, a, col);
+                    else if (G == 64) epi_group<64>(e, a, col);
+                    else epi_group128(e, a, col);
+                }
+                tc_fence_before();
+                mbar_arrive(acc_free(b));              // TMEM reads of this buffer are complete
+                }
+                // coalesced copy-out: consecutive threads write consecutive 16-byte chunks
+                const int nthr = nbuf == 2 ? 128 : 256;
+                const int tid = nbuf == 2 ? et : et + 128 * wg;
+                if (nbuf == 2) asm volatile("bar.sync %0, 128;" ::"r"(2 + wg) : "memory");
+                else asm volatile("bar.sync 4, 256;" ::: "memory");
+                const int cpr = row_bytes >> 4;
+                for (int jj = tid; ok && !a.out_f32 && jj < kTileM * cpr; jj += nthr) {
+                    const int r = jj / cpr, c = jj - r * cpr;
+                    const int oy = ho0 + r / a.tw, ox = wo0 + r % a.tw;
+                    if (oy < a.ho && ox < a.wo) {
+                        const long long pix = ((long long)img * a.ho + oy) * a.wo + ox;
+                        const int4 v = *reinterpret_cast<const int4 *>(stage_tile + (size_t)r * a.row_stride + c * 16);
+                        *reinterpret_cast<int4 *>(static_cast<uint8_t *>(a.y) + (pix * a.co + n0) * esz + c * 16) = v;
+                    }
+                }
+                if (nbuf == 2) asm volatile("bar.sync %0, 128;" ::"r"(2 + wg) : "memory");
+                else asm volatile("bar.sync 4, 256;" ::: "memory");
             }
         }
     }
@@ -723,12 +800,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const ConvArgs &a, int smem_bytes, cudaStream_t s) {
     static int configured_smem = 0;
+    static int sms = 0;
     if (smem_bytes > configured_smem) {
         cudaError_t e = cudaFuncSetAttribute(conv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
         if (e != cudaSuccess) return e;
         configured_smem = smem_bytes;
     }
-    dim3 grid((unsigned)(a.n * a.tiles_w * a.tiles_h), (unsigned)(a.co / a.n_t));
+    if (!sms) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (sms <= 0) sms = 148;
+    }
+    const int grid = a.num_tiles < sms ? a.num_tiles : sms;
     conv_kernel<<<grid, kThreads, smem_bytes, s>>>(tmA, tmB, a);
     return cudaGetLastError();
 }

@@ -56,8 +56,11 @@ struct ConvArgs {
     int gather;                      // small-channel loader
     int chunk_kb;                    // reduction blocks per exact fp32 chunk
     int stages;
-    int tmem_cols, part_col;
+    int tmem_cols;                   // TMEM columns allocated (power of two)
+    int nbuf, buf_cols;              // accumulator buffers and columns per buffer (acc [+ int32 partial])
+    int num_tiles, n_tiles_n;        // output tiles in the launch, N tiles per M tile
     int stage_bytes, b_bytes, raw_bytes;
+    int staging_bytes, row_stride;   // shared-memory output tiles after the stages
     int const_off;                   // offsets from the barrier area: epilogue constants,
     int win_off, win_h, win_w;       // small-channel input window and its size
     const int8_t *x;
