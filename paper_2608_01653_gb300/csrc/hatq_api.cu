@@ -447,7 +447,6 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     a.chunk_kb = 16;
     a.b_bytes = a.n_t * 128;
     a.raw_bytes = g.gather ? 0 : 8192;
-    a.stage_bytes = 16384 + a.b_bytes + a.raw_bytes;
     a.n_tiles_n = d->c_out / a.n_t;
     {
         const long long nt = (long long)n * a.tiles_w * a.tiles_h * a.n_tiles_n;
@@ -472,6 +471,13 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     const int const_bytes = (3 * d->c_out * 4 + 127) & ~127;
     const int fixed = 1024 /* align */ + 8 * (3 * 8 + 7) + 16 + 128 + table_bytes + const_bytes + win_bytes;
     const int budget = 227 * 1024 - 1024 /* static */ - fixed - a.staging_bytes;
+    // a stage holds `sub` 64-wide reduction blocks: [fp16 A x sub | weights x sub | INT8 box x sub];
+    // two blocks per stage halve the barrier round trips per MMA where two such stages fit
+    const int one = 16384 + a.b_bytes + a.raw_bytes;
+    a.sub = (!g.gather && a.num_kb > 1 && budget / (2 * one) >= 2) ? 2 : 1;
+    a.stage_bytes = a.sub * one;
+    a.b_off = a.sub * 16384;
+    a.raw_off = a.b_off + a.sub * a.b_bytes;
     a.stages = budget / a.stage_bytes;
     if (a.stages > 8) a.stages = 8;
     if (g.gather && a.stages > 4) a.stages = 4;

@@ -423,6 +423,8 @@ __device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a,
 // warpgroup w then takes the tiles of buffer w while the MMA issuer already
 // fills the other buffer; with one buffer both epilogue warpgroups split the
 // columns of every tile.
+// SUB: 64-wide reduction blocks per pipeline stage (1 or 2)
+template <int SUB>
 __global__ void __launch_bounds__(kThreads, 1)
     conv_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const ConvArgs a) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -519,18 +521,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int j = 0; j < my_tiles && ok; ++j) {
                 int img, ho0, wo0, n0;
                 tile_coords(j, img, ho0, wo0, n0);
-                for (int kb = 0; kb < a.num_kb; ++kb, ++it) {
+                for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB, ++it) {
                     const int s = it % S, r = it / S;
+                    const int nsub = min(SUB, a.num_kb - kb0);
                     if (!mbar_wait(empty_bar(s), (r & 1) ^ 1, abort_flag, a.err)) { ok = false; break; }
                     const uint32_t st = smem_addr(smem + (size_t)s * a.stage_bytes);
-                    mbar_expect_tx(full_bar(s), tx_bytes);
-                    tma_load_2d(st + 16384, &tmB, full_bar(s), kb * kBlockK, n0);
-                    if (!a.gather) {
-                        const int tap = kb / a.cin_kb;
-                        const int c0 = (kb - tap * a.cin_kb) * kBlockK;
-                        const int ky = tap / a.kw, kx = tap - (tap / a.kw) * a.kw;
-                        tma_load_4d(st + 16384 + a.b_bytes, &tmA, full_bar(s), c0, wo0 * a.stride + kx - a.pad,
-                                    ho0 * a.stride + ky - a.pad, img);
+                    mbar_expect_tx(full_bar(s), tx_bytes * (uint32_t)nsub);
+#pragma unroll
+                    for (int u = 0; u < SUB; ++u) {
+                        if (u >= nsub) break;
+                        const int kb = kb0 + u;
+                        tma_load_2d(st + a.b_off + u * a.b_bytes, &tmB, full_bar(s), kb * kBlockK, n0);
+                        if (!a.gather) {
+                            const int tap = kb / a.cin_kb;
+                            const int c0 = (kb - tap * a.cin_kb) * kBlockK;
+                            const int ky = tap / a.kw, kx = tap - (tap / a.kw) * a.kw;
+                            tma_load_4d(st + a.raw_off + u * 8192, &tmA, full_bar(s), c0, wo0 * a.stride + kx - a.pad,
+                                        ho0 * a.stride + ky - a.pad, img);
+                        }
                     }
                     issued_round[s] = r;
                 }
@@ -559,10 +567,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!mbar_wait(acc_free(b), ((j / nbuf) - 1) & 1, abort_flag, a.err)) { ok = false; break; }
                     tc_fence_after();
                 }
-                for (int kb = 0; kb < a.num_kb; ++kb, ++it) {
+                // a stage holds SUB 64-wide reduction blocks; chunk boundaries
+                // (multiples of chunk_kb, itself a multiple of SUB) fall between stages
+                for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB, ++it) {
                     const int s = it % S, r = it / S;
-                    const int ck = kb % a.chunk_kb;
-                    if (ck == 0 && kb > 0) {   // wait until the previous chunk was drained
+                    const int nsub = min(SUB, a.num_kb - kb0);
+                    const int ck0 = kb0 % a.chunk_kb;
+                    if (ck0 == 0 && kb0 > 0) {   // wait until the previous chunk was drained
                         if (!mbar_wait(acc_empty(b), empty_cnt[b] & 1, abort_flag, a.err)) { ok = false; break; }
                         ++empty_cnt[b];
                         tc_fence_after();
@@ -571,14 +582,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!mbar_wait(conv_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t st = smem_addr(smem + (size_t)s * a.stage_bytes);
-                    const uint64_t da = sdesc_sw128(st);
-                    const uint64_t db = sdesc_sw128(st + 16384);
 #pragma unroll
-                    for (int kk = 0; kk < kBlockK / 16; ++kk)   // K = 16 per instruction, 32 bytes apart
-                        umma_f16(d_tmem, da + (uint64_t)(2 * kk), db + (uint64_t)(2 * kk), idesc,
-                                 (ck > 0 || kk > 0) ? 1u : 0u);
+                    for (int u = 0; u < SUB; ++u) {
+                        if (u >= nsub) break;
+                        const uint64_t da = sdesc_sw128(st + u * 16384);
+                        const uint64_t db = sdesc_sw128(st + a.b_off + u * a.b_bytes);
+#pragma unroll
+                        for (int kk = 0; kk < kBlockK / 16; ++kk)   // K = 16 per instruction, 32 bytes apart
+                            umma_f16(d_tmem, da + (uint64_t)(2 * kk), db + (uint64_t)(2 * kk), idesc,
+                                     (ck0 + u > 0 || kk > 0) ? 1u : 0u);
+                    }
                     umma_commit(empty_bar(s));
-                    if (ck == a.chunk_kb - 1 || kb == a.num_kb - 1) umma_commit(acc_full(b));
+                    const int kb_end = kb0 + nsub;
+                    if (kb_end % a.chunk_kb == 0 || kb_end == a.num_kb) umma_commit(acc_full(b));
                 }
             }
             umma_commit(mma_done);
@@ -594,12 +610,16 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = true;
         if (!a.gather) {
             for (int j = 0; j < my_tiles && ok; ++j) {
-                for (int kb = 0; kb < a.num_kb; ++kb, ++it) {
+                for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB, ++it) {
                     const int s = it % S, r = it / S;
+                    const int nsub = min(SUB, a.num_kb - kb0);
                     ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
                     if (!ok) break;
-                    uint8_t *st = smem + (size_t)s * a.stage_bytes;
-                    const uint8_t *raw = st + 16384 + a.b_bytes;
+#pragma unroll
+                    for (int u = 0; u < SUB; ++u) {
+                    if (u >= nsub) break;
+                    uint8_t *st = smem + (size_t)s * a.stage_bytes + u * 16384;
+                    const uint8_t *raw = smem + (size_t)s * a.stage_bytes + a.raw_off + u * 8192;
                     int4 v[kPasses];                       // all loads first, then convert and store
 #pragma unroll
                     for (int p = 0; p < kPasses; ++p) {
@@ -617,6 +637,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         i8x4_to_f16x4((uint32_t)v[p].w, h[6], h[7]);
                         *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
                         *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
+                    }
                     }
                     fence_proxy_async_smem();
                     mbar_arrive(conv_bar(s));
@@ -812,21 +833,33 @@ __global__ void __launch_bounds__(kThreads, 1)
 }  // namespace
 
 cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const ConvArgs &a, int smem_bytes, cudaStream_t s) {
-    static int configured_smem = 0;
-    static int sms = 0;
-    if (smem_bytes > configured_smem) {
-        cudaError_t e = cudaFuncSetAttribute(conv_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+    // the shared-memory opt-in and the SM count are per device
+    constexpr int kMaxDev = 64;
+    static int configured_smem[kMaxDev][2] = {};
+    static int sms_of[kMaxDev] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
+    if (a.sub != 1 && (a.sub != 2 || a.gather)) return cudaErrorInvalidValue;   // gathered tiles: one block per stage
+    const int v = a.sub == 2 ? 1 : 0;
+    if (smem_bytes > configured_smem[dev][v]) {
+        e = cudaFuncSetAttribute(v ? conv_kernel<2> : conv_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 smem_bytes);
         if (e != cudaSuccess) return e;
-        configured_smem = smem_bytes;
+        configured_smem[dev][v] = smem_bytes;
     }
-    if (!sms) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (sms <= 0) sms = 148;
+    if (!sms_of[dev]) {
+        int sms = 0;
+        e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return e;
+        sms_of[dev] = sms > 0 ? sms : 1;
     }
-    const int grid = a.num_tiles < sms ? a.num_tiles : sms;
-    conv_kernel<<<grid, kThreads, smem_bytes, s>>>(tmA, tmB, a);
+    const int grid = a.num_tiles < sms_of[dev] ? a.num_tiles : sms_of[dev];
+    if (v)
+        conv_kernel<2><<<grid, kThreads, smem_bytes, s>>>(tmA, tmB, a);
+    else
+        conv_kernel<1><<<grid, kThreads, smem_bytes, s>>>(tmA, tmB, a);
     return cudaGetLastError();
 }
 

@@ -60,6 +60,8 @@ struct ConvArgs {
     int nbuf, buf_cols;              // accumulator buffers and columns per buffer (acc [+ int32 partial])
     int num_tiles, n_tiles_n;        // output tiles in the launch, N tiles per M tile
     int stage_bytes, b_bytes, raw_bytes;
+    int sub;                         // 64-wide reduction blocks per pipeline stage (1 or 2)
+    int b_off, raw_off;              // offsets of the weight and INT8 boxes inside a stage
     int staging_bytes, row_stride;   // shared-memory output tiles after the stages
     int const_off;                   // offsets from the barrier area: epilogue constants,
     int win_off, win_h, win_w;       // small-channel input window and its size
