@@ -615,28 +615,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int nsub = min(SUB, a.num_kb - kb0);
                     ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
                     if (!ok) break;
-#pragma unroll
+#pragma unroll 1
                     for (int u = 0; u < SUB; ++u) {
                     if (u >= nsub) break;
                     uint8_t *st = smem + (size_t)s * a.stage_bytes + u * 16384;
                     const uint8_t *raw = smem + (size_t)s * a.stage_bytes + a.raw_off + u * 8192;
-                    int4 v[kPasses];                       // all loads first, then convert and store
+                    // thread -> (row m, 8-element chunk c): 8 consecutive lanes cover one
+                    // row, i.e. all 32 banks for both the 8-byte loads and the swizzled stores
+                    uint2 v[2 * kPasses];                  // all loads first, then convert and store
 #pragma unroll
-                    for (int p = 0; p < kPasses; ++p) {
+                    for (int p = 0; p < 2 * kPasses; ++p) {
                         const int idx = p * kConvThreads + ct;
-                        v[p] = *reinterpret_cast<const int4 *>(raw + (idx >> 2) * 64 + (idx & 3) * 16);
+                        v[p] = *reinterpret_cast<const uint2 *>(raw + idx * 8);
                     }
 #pragma unroll
-                    for (int p = 0; p < kPasses; ++p) {
+                    for (int p = 0; p < 2 * kPasses; ++p) {
                         const int idx = p * kConvThreads + ct;
-                        const int m = idx >> 2, q = idx & 3;    // row, 16-element quarter of the 64-wide block
-                        uint32_t h[8];
-                        i8x4_to_f16x4((uint32_t)v[p].x, h[0], h[1]);
-                        i8x4_to_f16x4((uint32_t)v[p].y, h[2], h[3]);
-                        i8x4_to_f16x4((uint32_t)v[p].z, h[4], h[5]);
-                        i8x4_to_f16x4((uint32_t)v[p].w, h[6], h[7]);
-                        *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
-                        *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
+                        uint32_t h[4];
+                        i8x4_to_f16x4(v[p].x, h[0], h[1]);
+                        i8x4_to_f16x4(v[p].y, h[2], h[3]);
+                        *reinterpret_cast<int4 *>(st + sw128_offset(idx >> 3, idx & 7)) =
+                            make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
                     }
                     }
                     fence_proxy_async_smem();
