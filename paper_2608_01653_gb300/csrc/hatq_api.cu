@@ -453,13 +453,15 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
         if (nt >= (1LL << 31)) return fail(HATQ_ERR_UNSUPPORTED, "too many output tiles");
         a.num_tiles = (int)nt;
     }
-    // TMEM: one or two accumulator buffers of n_t fp32 columns (+ n_t int32
-    // partial columns when the reduction spans several exact chunks)
+    // TMEM: two fp32 regions of n_t columns; exact chunk g of the reduction
+    // accumulates in region g & 1. Without drains the two epilogue warpgroups
+    // alternate tiles (nbuf = 2); with drains both take every chunk, each for
+    // half of the columns, keeping int32 partials in registers (nbuf = 1).
     const bool drains = a.num_kb > a.chunk_kb;
-    a.buf_cols = a.n_t * (drains ? 2 : 1);
-    a.nbuf = 2 * a.buf_cols <= 512 ? 2 : 1;
+    a.buf_cols = a.n_t;
+    a.nbuf = drains ? 1 : 2;
     a.tmem_cols = 32;
-    while (a.tmem_cols < a.nbuf * a.buf_cols) a.tmem_cols <<= 1;
+    while (a.tmem_cols < 2 * a.n_t) a.tmem_cols <<= 1;
     // shared memory: [stages][output tiles][barriers | gather table | constants | window]
     const int esz = L->out_f32 ? 4 : 1;
     a.row_stride = a.n_t * esz + 16;                 // padded rows: 8 consecutive rows hit 8 bank groups

@@ -241,8 +241,7 @@ struct EpiCtx {
     const int *mult;
     const float *deq;
     uint32_t t_acc;      // TMEM address of this warp's lanes, column 0 of the accumulator
-    uint32_t t_part;     // ... of the int32 partial region
-    bool has_part;
+    bool int_acc;        // the accumulator holds exact int32 totals (else exact fp32 integers)
     uint8_t *row;        // this thread's row of the shared-memory output tile (INT8 output)
     float *gout;         // float32 output: this thread's pixel row in global memory, or null
 };
@@ -251,14 +250,11 @@ struct EpiCtx {
 __device__ __forceinline__ void load_acc16(const EpiCtx &e, int col, int (&v)[16]) {
     uint32_t r[16];
     tmem_ld16(e.t_acc + col, r);
-    if (e.has_part) {
-        uint32_t p[16];
-        tmem_ld16(e.t_part + col, p);
-        tmem_wait_ld();
+    tmem_wait_ld();
+    if (e.int_acc) {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) v[i] = __float2int_rn(__uint_as_float(r[i])) + (int)p[i];
+        for (int i = 0; i < 16; ++i) v[i] = (int)r[i];
     } else {
-        tmem_wait_ld();
 #pragma unroll
         for (int i = 0; i < 16; ++i) v[i] = __float2int_rn(__uint_as_float(r[i]));
     }
@@ -418,11 +414,13 @@ __device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a,
 // ------------------------------------------------------------------ kernel
 
 // One CTA per SM, looping over output tiles (tile t -> M tile t / n_tiles_n,
-// N tile t % n_tiles_n). The stage ring runs continuously across tiles. The
-// accumulator is double-buffered in TMEM when two buffers fit: epilogue
-// warpgroup w then takes the tiles of buffer w while the MMA issuer already
-// fills the other buffer; with one buffer both epilogue warpgroups split the
-// columns of every tile.
+// N tile t % n_tiles_n). The stage ring runs continuously across tiles. TMEM
+// holds two fp32 accumulator regions and the reduction runs in exact chunks
+// of at most 1024 (sums below 2^24), chunk g accumulating in region g & 1, so
+// the MMA issuer fills one region while the epilogue empties the other. With
+// one chunk per tile epilogue warpgroup w takes the tiles of region w; with
+// several, both warpgroups drain every chunk into int32 register partials
+// (half of the 32-column groups each) and finish the tile together.
 // SUB: 64-wide reduction blocks per pipeline stage (1 or 2)
 template <int SUB>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -433,13 +431,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *staging = smem + (size_t)S * a.stage_bytes;
     uint8_t *bar_area = staging + (size_t)a.staging_bytes;
     const uint32_t bar0 = smem_addr(bar_area);
-    // barriers: full[S], conv[S], empty[S], acc_full[2], acc_empty[2], acc_free[2], mma_done
+    // barriers: full[S], conv[S], empty[S], acc_full[2], acc_empty[2], (unused)[2], mma_done
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
     auto conv_bar = [&](int s) { return bar0 + 8u * (S + s); };
     auto empty_bar = [&](int s) { return bar0 + 8u * (2 * S + s); };
     auto acc_full = [&](int b) { return bar0 + 8u * (3 * S + b); };
     auto acc_empty = [&](int b) { return bar0 + 8u * (3 * S + 2 + b); };
-    auto acc_free = [&](int b) { return bar0 + 8u * (3 * S + 4 + b); };
     const uint32_t mma_done = bar0 + 8u * (3 * S + 6);
     uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_area + 8 * (3 * S + 7));
     volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_area + 8 * (3 * S + 7) + 4);
@@ -455,8 +452,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int tiles_per_img = a.tiles_w * a.tiles_h;
+    // nbuf == 2: the epilogue warpgroups alternate tiles, each taking all columns;
+    // nbuf == 1 (reduction in several exact chunks): both warpgroups take every
+    // chunk, each for half of the 32-column groups, and keep the int32 partial
+    // sums of their columns in registers.
     const int nbuf = a.nbuf;
-    const int ep_count = nbuf == 2 ? 128 : 256;     // epilogue threads that arrive per buffer
+    const int ep_count = nbuf == 2 ? 128 : 256;     // epilogue threads that release a region
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -467,7 +468,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int b = 0; b < 2; ++b) {
             mbar_init(acc_full(b), 1);
             mbar_init(acc_empty(b), ep_count);
-            mbar_init(acc_free(b), ep_count);
         }
         mbar_init(mma_done, 1);
         *abort_flag = 0;
@@ -559,24 +559,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t idesc = idesc_f16(a.n_t);
             bool ok = true;
             int it = 0;
-            int empty_cnt[2] = {0, 0};
+            int g = 0;                       // exact chunks issued so far; chunk g accumulates in region g & 1
+            uint32_t d_tmem = tmem;
             for (int j = 0; j < my_tiles && ok; ++j) {
-                const int b = j % nbuf;
-                const uint32_t d_tmem = tmem + (uint32_t)(b * a.buf_cols);
-                if (j >= nbuf) {      // wait until the epilogue released this buffer
-                    if (!mbar_wait(acc_free(b), ((j / nbuf) - 1) & 1, abort_flag, a.err)) { ok = false; break; }
-                    tc_fence_after();
-                }
                 // a stage holds SUB 64-wide reduction blocks; chunk boundaries
                 // (multiples of chunk_kb, itself a multiple of SUB) fall between stages
                 for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB, ++it) {
                     const int s = it % S, r = it / S;
                     const int nsub = min(SUB, a.num_kb - kb0);
                     const int ck0 = kb0 % a.chunk_kb;
-                    if (ck0 == 0 && kb0 > 0) {   // wait until the previous chunk was drained
-                        if (!mbar_wait(acc_empty(b), empty_cnt[b] & 1, abort_flag, a.err)) { ok = false; break; }
-                        ++empty_cnt[b];
-                        tc_fence_after();
+                    if (ck0 == 0) {
+                        d_tmem = tmem + (uint32_t)((g & 1) * a.n_t);
+                        if (g >= 2) {        // wait until the epilogue released the region
+                            if (!mbar_wait(acc_empty(g & 1), ((g >> 1) - 1) & 1, abort_flag, a.err)) { ok = false; break; }
+                            tc_fence_after();
+                        }
                     }
                     if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
                     if (!mbar_wait(conv_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
@@ -594,7 +591,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     umma_commit(empty_bar(s));
                     const int kb_end = kb0 + nsub;
-                    if (kb_end % a.chunk_kb == 0 || kb_end == a.num_kb) umma_commit(acc_full(b));
+                    if (kb_end % a.chunk_kb == 0 || kb_end == a.num_kb) {
+                        umma_commit(acc_full(g & 1));
+                        ++g;
+                    }
                 }
             }
             umma_commit(mma_done);
@@ -732,57 +732,77 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int row_bytes = a.n_t * esz;
         uint8_t *stage_tile = staging + (size_t)(nbuf == 2 ? wg : 0) * kTileM * a.row_stride;
         const int G = max(32, max(a.hb_out, a.hb_next));
-        int full_cnt[2] = {0, 0};
+        uint32_t part[4][32];                      // nbuf == 1: int32 partial sums of column groups 2k + wg
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+#pragma unroll
+            for (int i = 0; i < 32; ++i) part[k][i] = 0u;
         bool ok = true;
         // Every epilogue thread runs the same loops (also after an abort, doing
-        // no work) so the warpgroup reaches each named barrier together.
+        // no work) so the warpgroups reach each named barrier together.
         for (int j = 0; j < my_tiles; ++j) {
-            const int b = j % nbuf;
-            if (nbuf == 2 && b != wg) continue;
+            if (nbuf == 2 && (j & 1) != wg) continue;
             int img, ho0, wo0, n0;
             tile_coords(j, img, ho0, wo0, n0);
-            const uint32_t t_acc = tmem + (uint32_t)(b * a.buf_cols) + ((uint32_t)(quad * 32) << 16);
-            const uint32_t t_part = t_acc + (uint32_t)a.n_t;
             for (int ch = 0; ch < nchunks; ++ch) {
+                const int g = j * nchunks + ch;    // chunk index, as counted by the MMA issuer
+                const int reg = g & 1;
+                const uint32_t t_acc = tmem + (uint32_t)(reg * a.n_t) + ((uint32_t)(quad * 32) << 16);
                 if (ok) {
-                    ok = __all_sync(0xffffffffu, mbar_wait(acc_full(b), full_cnt[b] & 1, abort_flag, a.err));
-                    ++full_cnt[b];
+                    ok = __all_sync(0xffffffffu, mbar_wait(acc_full(reg), (g >> 1) & 1, abort_flag, a.err));
                     tc_fence_after();
                 }
                 if (ch + 1 < nchunks) {
-                    if (!ok) continue;
-                    // drain: chunk sum -> int32 partial (with one buffer the two warpgroups split the columns)
-                    for (int col = 0; col < a.n_t; col += 32) {
-                        if (nbuf == 1 && ((col >> 5) & 1) != wg) continue;
-                        uint32_t r[32];
-                        tmem_ld32(t_acc + col, r);
-                        if (ch > 0) {
-                            uint32_t p[32];
-                            tmem_ld32(t_part + col, p);
+                    // drain: chunk sum -> register partials; the region goes straight back to the MMA issuer
+                    if (ok) {
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const int col = (2 * k + wg) * 32;
+                            if (col >= a.n_t) break;
+                            uint32_t r[32];
+                            tmem_ld32(t_acc + col, r);
                             tmem_wait_ld();
 #pragma unroll
-                            for (int i = 0; i < 32; ++i) r[i] = (uint32_t)(__float2int_rn(__uint_as_float(r[i])) + (int)p[i]);
-                        } else {
-                            tmem_wait_ld();
-#pragma unroll
-                            for (int i = 0; i < 32; ++i) r[i] = (uint32_t)__float2int_rn(__uint_as_float(r[i]));
+                            for (int i = 0; i < 32; ++i) part[k][i] += (uint32_t)__float2int_rn(__uint_as_float(r[i]));
                         }
-                        tmem_st32(t_part + col, r);
                     }
-                    tmem_wait_st();
                     tc_fence_before();
-                    mbar_arrive(acc_empty(b));
+                    mbar_arrive(acc_empty(reg));
                     continue;
                 }
-                // final chunk: epilogue into the shared-memory output tile
+                if (nbuf == 1) {
+                    // last chunk: chunk sum + partial -> exact int32 totals, written back in place so
+                    // that each 64/128-wide transform group can read all of its columns
+                    if (ok) {
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const int col = (2 * k + wg) * 32;
+                            if (col >= a.n_t) break;
+                            uint32_t r[32];
+                            tmem_ld32(t_acc + col, r);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) r[i] = part[k][i] + (uint32_t)__float2int_rn(__uint_as_float(r[i]));
+                            tmem_st32(t_acc + col, r);
+                        }
+                        tmem_wait_st();
+                    }
+                    tc_fence_before();
+                    asm volatile("bar.sync 4, 256;" ::: "memory");
+                    tc_fence_after();
+                }
+                // the partials restart at zero for the next tile (and are dead during the groups)
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) part[k][i] = 0u;
                 if (ok) {
                 EpiCtx e;
                 e.b_int = cb + n0;
                 e.mult = cb + a.co + n0;
                 e.deq = reinterpret_cast<const float *>(cb + 2 * a.co) + n0;
                 e.t_acc = t_acc;
-                e.t_part = t_part;
-                e.has_part = nchunks > 1;
+                e.int_acc = nbuf == 1;
                 e.row = stage_tile + (size_t)row * a.row_stride;
                 e.gout = nullptr;
                 if (a.out_f32) {
@@ -797,9 +817,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     else if (G == 64) epi_group<64>(e, a, col);
                     else epi_group128(e, a, col);
                 }
-                tc_fence_before();
-                mbar_arrive(acc_free(b));              // TMEM reads of this buffer are complete
                 }
+                tc_fence_before();
+                mbar_arrive(acc_empty(reg));           // TMEM reads of this region are complete
                 // coalesced copy-out: consecutive threads write consecutive 16-byte chunks
                 const int nthr = nbuf == 2 ? 128 : 256;
                 const int tid = nbuf == 2 ? et : et + 128 * wg;

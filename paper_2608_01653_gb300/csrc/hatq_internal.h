@@ -57,7 +57,7 @@ struct ConvArgs {
     int chunk_kb;                    // reduction blocks per exact fp32 chunk
     int stages;
     int tmem_cols;                   // TMEM columns allocated (power of two)
-    int nbuf, buf_cols;              // accumulator buffers and columns per buffer (acc [+ int32 partial])
+    int nbuf, buf_cols;              // 2: epilogue warpgroups alternate tiles; 1: they split columns (drains); n_t
     int num_tiles, n_tiles_n;        // output tiles in the launch, N tiles per M tile
     int stage_bytes, b_bytes, raw_bytes;
     int sub;                         // 64-wide reduction blocks per pipeline stage (1 or 2)
