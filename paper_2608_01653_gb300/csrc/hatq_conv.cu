@@ -208,6 +208,21 @@ __device__ __forceinline__ int requant8(long long v, int n) {
     return q < -127 ? -127 : (q > 127 ? 127 : q);
 }
 
+// The same rounding for 32 <= n <= 62 in 32-bit pieces: with k = 2^(n-1) - 1
+// and s = n - 32, v + k + bit_n(v) stays below 2^63 and its arithmetic shift
+// by n is the high word shifted by s.
+__device__ __forceinline__ int requant8_hi(long long v, int s, unsigned long long k) {
+    const uint32_t bit = ((uint32_t)((unsigned long long)v >> 32) >> s) & 1u;
+    const long long u = v + (long long)k + (long long)bit;
+    const int q = (int)(u >> 32) >> s;
+    return min(max(q, -127), 127);
+}
+// Low bytes of four codes in [-127, 127] packed into one word.
+__device__ __forceinline__ uint32_t pack4(int q0, int q1, int q2, int q3) {
+    return __byte_perm(__byte_perm((uint32_t)q0, (uint32_t)q1, 0x0040), __byte_perm((uint32_t)q2, (uint32_t)q3, 0x0040),
+                       0x5410);
+}
+
 template <int G, int HB, typename T>
 __device__ __forceinline__ void fwht_fixed(T (&t)[G]) {
 #pragma unroll
@@ -294,15 +309,30 @@ __device__ __forceinline__ void scale_f32(const EpiCtx &e, int col, const int (&
 // thread's row of the shared-memory output tile (copied out coalesced later).
 template <int G>
 __device__ __forceinline__ void store_codes(const ConvArgs &a, uint8_t *row, int col, const long long (&t)[G]) {
+    if (a.shift >= 32) {
+        const int sh = a.shift - 32;
+        const unsigned long long k = (1ull << (a.shift - 1)) - 1;
+#pragma unroll
+        for (int i = 0; i < G / 16; ++i) {
+            uint32_t w[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int b = 16 * i + 4 * j;
+                w[j] = pack4(requant8_hi(t[b], sh, k), requant8_hi(t[b + 1], sh, k), requant8_hi(t[b + 2], sh, k),
+                             requant8_hi(t[b + 3], sh, k));
+            }
+            reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
+        }
+        return;
+    }
 #pragma unroll
     for (int i = 0; i < G / 16; ++i) {
         uint32_t w[4];
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
             const int b = 16 * i + 4 * j;
-            w[j] = (uint32_t)(requant8(t[b], a.shift) & 0xff) | ((uint32_t)(requant8(t[b + 1], a.shift) & 0xff) << 8) |
-                   ((uint32_t)(requant8(t[b + 2], a.shift) & 0xff) << 16) |
-                   ((uint32_t)(requant8(t[b + 3], a.shift) & 0xff) << 24);
+            w[j] = pack4(requant8(t[b], a.shift), requant8(t[b + 1], a.shift), requant8(t[b + 2], a.shift),
+                         requant8(t[b + 3], a.shift));
         }
         reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
     }
