@@ -87,10 +87,12 @@ typedef struct {
     int out_f32;          /* 1: dequantized float32 output; 0: INT8 codes at s_y */
     int shift;            /* shared right shift n (Eq. integer_fixed_point_scale) */
     int k_pad;            /* packed reduction length = columns of w_i8 / w_f16 */
-    int gather;           /* 1: small-channel layer (c_in % 16 != 0), reduction packed densely */
+    int gather;           /* 1: small-channel layer (c_in % 16 != 0): kernel row ky holds the kw*c_in
+                             entries (kx, c_in) padded with zero weights to a multiple of 8 */
     float s_x;            /* scale of the INT8 operand this layer consumes */
     float s_y;            /* scale of the INT8 codes it emits */
-    int8_t *w_i8;         /* [c_out][k_pad] weight codes w_int, K order (kh, kw, c_in) */
+    int8_t *w_i8;         /* [c_out][k_pad] weight codes w_int, K order (kh, kw, c_in); c_in padded to a
+                             multiple of 64 per tap (gather == 0) or kw*c_in padded to 8 per row */
     uint16_t *w_f16;      /* [c_out][k_pad] the same codes as IEEE fp16 (exact), tensor-core operand */
     int32_t *b_int;       /* [c_out] bias codes, Eq. supp_bias_quantization */
     int32_t *mult;        /* [c_out] multipliers M_c, Eq. integer_fixed_point_scale */

@@ -79,7 +79,7 @@ EncodeTiledFn encode_fn() {
 // ------------------------------------------------------------ geometry
 
 struct Geometry {
-    int gather, cin_pad, k_pad, n_t, G;
+    int gather, cin_pad, seg, k_pad, n_t, G;
 };
 
 hatq_status check_desc(const hatq_conv_desc *d) {
@@ -111,16 +111,23 @@ bool fusable(int hb_out, int hb_next) {
 }
 
 hatq_status geometry(const hatq_conv_desc *d, int hb_next, Geometry *g) {
+    // Packed reduction order. c_in % 16 == 0: (ky, kx, ci) with ci padded to a
+    // multiple of 64 per tap. Otherwise (small c_in): kernel row ky holds the
+    // kw * c_in entries (kx, ci) of one contiguous input-row segment, padded
+    // with zero weights to seg (a multiple of 8), rows back to back.
     g->gather = d->c_in % 16 != 0;
     g->cin_pad = (d->c_in + 63) / 64 * 64;
-    g->k_pad = g->gather ? (d->kh * d->kw * d->c_in + 63) / 64 * 64 : d->kh * d->kw * g->cin_pad;
+    g->seg = (d->kw * d->c_in + 7) / 8 * 8;
+    g->k_pad = g->gather ? (d->kh * g->seg + 63) / 64 * 64 : d->kh * d->kw * g->cin_pad;
     const int hb_out = d->form == HATQ_WH ? d->hb_out : 0;
     int G = 32;
     if (hb_out > G) G = hb_out;
     if (hb_next > G) G = hb_next;
     g->G = G;
     g->n_t = 0;
-    for (int nt = 256; nt >= G; nt -= 16)
+    // at most 224 columns, so that two accumulator regions leave at least 64
+    // TMEM columns for the fp16 A operand
+    for (int nt = 224; nt >= G; nt -= 16)
         if (nt % G == 0 && d->c_out % nt == 0) { g->n_t = nt; break; }
     if (!g->n_t) return fail(HATQ_ERR_UNSUPPORTED, "no output-channel tile for c_out=%d with group %d", d->c_out, G);
     return HATQ_OK;
@@ -277,7 +284,8 @@ hatq_status hatq_prepare_weights_host(const hatq_conv_desc *d, const float *w_oh
                 q = q < -127.0 ? -127.0 : (q > 127.0 ? 127.0 : q);
                 const int qi = (int)q;
                 sum_abs += qi < 0 ? -qi : qi;
-                const long long k = g.gather ? (long long)tap * ci + c : (long long)tap * g.cin_pad + c;
+                const long long k = g.gather ? (long long)(tap / d->kw) * g.seg + (tap % d->kw) * ci + c
+                                             : (long long)tap * g.cin_pad + c;
                 w_i8_out[(size_t)o * g.k_pad + k] = (int8_t)qi;
                 w_f16_out[(size_t)o * g.k_pad + k] = f16_bits(qi);
             }
@@ -453,38 +461,47 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
         if (nt >= (1LL << 31)) return fail(HATQ_ERR_UNSUPPORTED, "too many output tiles");
         a.num_tiles = (int)nt;
     }
-    // TMEM: two fp32 regions of n_t columns; exact chunk g of the reduction
-    // accumulates in region g & 1. Without drains the two epilogue warpgroups
-    // alternate tiles (nbuf = 2); with drains both take every chunk, each for
-    // half of the columns, keeping int32 partials in registers (nbuf = 1).
+    // TMEM (all 512 columns): two fp32 regions of n_t columns, exact chunk g
+    // of the reduction accumulating in region g & 1, then the ring of fp16
+    // A-operand slots. Without drains the two epilogue warpgroups alternate
+    // tiles (nbuf = 2); with drains both take every chunk, each for half of
+    // the columns, keeping int32 partials in registers (nbuf = 1).
     const bool drains = a.num_kb > a.chunk_kb;
     a.buf_cols = a.n_t;
     a.nbuf = drains ? 1 : 2;
-    a.tmem_cols = 32;
-    while (a.tmem_cols < 2 * a.n_t) a.tmem_cols <<= 1;
+    a.tmem_cols = 512;
+    a.a_col = 2 * a.n_t;
+    a.seg = g.seg;
     // shared memory: [stages][output tiles][barriers | gather table | constants | window]
     const int esz = L->out_f32 ? 4 : 1;
     a.row_stride = a.n_t * esz + 16;                 // padded rows: 8 consecutive rows hit 8 bank groups
     a.staging_bytes = L->out_f32 ? 0 : a.nbuf * kTileRows * a.row_stride;   // float32 output is stored directly
     a.win_h = (a.th - 1) * d->stride + d->kh;
     a.win_w = (a.tw - 1) * d->stride + d->kw;
-    const int win_bytes = g.gather ? (a.win_h * a.win_w * d->c_in + 127) & ~127 : 0;
-    const int table_bytes = g.gather ? a.num_kb * 64 * 4 : 0;
+    a.win_pitch = (a.win_w * d->c_in + 15) & ~15;
+    // + 16 bytes: the gather reads up to 11 bytes past a row segment
+    const int win_bytes = g.gather ? (a.win_h * a.win_pitch + 16 + 127) & ~127 : 0;
+    const int table_bytes = g.gather ? a.num_kb * 8 * 4 : 0;
     const int const_bytes = (3 * d->c_out * 4 + 127) & ~127;
-    const int fixed = 1024 /* align */ + 8 * (3 * 8 + 7) + 16 + 128 + table_bytes + const_bytes + win_bytes;
+    const int fixed = 1024 /* align */ + 8 * (3 * 8 + 9) + 16 + 128 + table_bytes + const_bytes + win_bytes;
     const int budget = 227 * 1024 - 1024 /* static */ - fixed - a.staging_bytes;
-    // a stage holds `sub` 64-wide reduction blocks: [fp16 A x sub | weights x sub | INT8 box x sub];
-    // two blocks per stage halve the barrier round trips per MMA where two such stages fit
-    const int one = 16384 + a.b_bytes + a.raw_bytes;
-    a.sub = (!g.gather && a.num_kb > 1 && budget / (2 * one) >= 2) ? 2 : 1;
+    // a stage holds `sub` 64-wide reduction blocks: [weights x sub | INT8 box x sub];
+    // two blocks per stage halve the barrier round trips per MMA where three
+    // such stages and two A slots of 64 columns fit
+    const int one = a.b_bytes + a.raw_bytes;
+    const int free_cols = 512 - a.a_col;
+    a.sub = (!g.gather && a.num_kb > 1 && budget / (2 * one) >= 3 && free_cols >= 128) ? 2 : 1;
+    a.a_slots = free_cols / (32 * a.sub);
+    if (a.a_slots > 4) a.a_slots = 4;
+    if (a.a_slots < 2) return fail(HATQ_ERR_UNSUPPORTED, "no TMEM room for the A operand (n_t=%d)", a.n_t);
     a.stage_bytes = a.sub * one;
-    a.b_off = a.sub * 16384;
-    a.raw_off = a.b_off + a.sub * a.b_bytes;
+    a.b_off = 0;
+    a.raw_off = a.sub * a.b_bytes;
     a.stages = budget / a.stage_bytes;
     if (a.stages > 8) a.stages = 8;
     if (g.gather && a.stages > 4) a.stages = 4;
     if (a.stages < 2) return fail(HATQ_ERR_UNSUPPORTED, "tile does not fit in shared memory");
-    const int bar_bytes = 8 * (3 * a.stages + 7) + 16;
+    const int bar_bytes = 8 * (3 * a.stages + 9) + 16;
     a.const_off = (bar_bytes + table_bytes + 127) & ~127;
     a.win_off = a.const_off + const_bytes;
     const int smem_bytes = a.stages * a.stage_bytes + a.staging_bytes + 1024 + a.win_off + win_bytes;
@@ -512,7 +529,7 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
         const cuuint32_t box[4] = {64, (cuuint32_t)(a.tw * d->stride), (cuuint32_t)(a.th * d->stride), 1};
         const cuuint32_t estr[4] = {1, (cuuint32_t)d->stride, (cuuint32_t)d->stride, 1};
         CUresult r = enc(&tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<int8_t *>(x), dims, strides, box, estr,
-                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "activation tensor map encoding failed (%d)", (int)r);
     } else {

@@ -39,8 +39,8 @@
 namespace hatq {
 namespace {
 
-constexpr int kThreads = 384;
-constexpr int kConvThreads = 64;       // converter warps 2-3
+constexpr int kThreads = 512;
+constexpr int kConvThreads = 128;      // converter warps 12-15, one per TMEM lane quadrant
 constexpr int kBlockK = 64;            // fp16 elements per 128-byte swizzle row
 constexpr int kTileM = 128;
 constexpr long long kWaitLimitCycles = 4000000000LL;   // about 2 s at 2 GHz
@@ -91,9 +91,6 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
 __device__ __forceinline__ void fence_barrier_init() {
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
-__device__ __forceinline__ void fence_proxy_async_smem() {
-    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
 __device__ __forceinline__ void tc_fence_before() {
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
 }
@@ -130,11 +127,13 @@ __device__ __forceinline__ uint32_t idesc_f16(int n) {
     return (1u << 4) | ((uint32_t)(n >> 3) << 17) | ((uint32_t)(kTileM >> 4) << 24);
 }
 
-__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+// D (+)= A * B^T with the A operand in TMEM (lane = row, two fp16 per 32-bit
+// column, K ascending) and B described in shared memory.
+__device__ __forceinline__ void umma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b, uint32_t idesc, uint32_t acc) {
     asm volatile(
         "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
-        " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
-        "l"(a), "l"(b), "r"(idesc), "r"(acc)
+        " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(acc)
         : "memory");
 }
 __device__ __forceinline__ void umma_commit(uint32_t bar) {
@@ -181,12 +180,6 @@ __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t
     asm("prmt.b32 %0, %1, %2, %3;" : "=r"(b) : "r"(u), "r"(0x64646464u), "r"(0x4342u));
     asm("sub.f16x2 %0, %1, %2;" : "=r"(lo) : "r"(a), "r"(0x64806480u));
     asm("sub.f16x2 %0, %1, %2;" : "=r"(hi) : "r"(b), "r"(0x64806480u));
-}
-
-// Byte offset of 16-byte chunk `chunk` of row `row` in a 128B-swizzled
-// K-major tile (8-row groups of 1024 bytes).
-__device__ __forceinline__ uint32_t sw128_offset(int row, int chunk) {
-    return (uint32_t)((row >> 3) * 1024 + (row & 7) * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
 // ------------------------------------------------------------------ epilogue math
@@ -461,15 +454,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t *staging = smem + (size_t)S * a.stage_bytes;
     uint8_t *bar_area = staging + (size_t)a.staging_bytes;
     const uint32_t bar0 = smem_addr(bar_area);
-    // barriers: full[S], conv[S], empty[S], acc_full[2], acc_empty[2], (unused)[2], mma_done
+    // barriers: full[S], conv[S], empty[S], acc_full[2], acc_empty[2], a_free[4], mma_done
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
     auto conv_bar = [&](int s) { return bar0 + 8u * (S + s); };
     auto empty_bar = [&](int s) { return bar0 + 8u * (2 * S + s); };
     auto acc_full = [&](int b) { return bar0 + 8u * (3 * S + b); };
     auto acc_empty = [&](int b) { return bar0 + 8u * (3 * S + 2 + b); };
-    const uint32_t mma_done = bar0 + 8u * (3 * S + 6);
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_area + 8 * (3 * S + 7));
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_area + 8 * (3 * S + 7) + 4);
+    auto a_free = [&](int q) { return bar0 + 8u * (3 * S + 4 + q); };
+    const uint32_t mma_done = bar0 + 8u * (3 * S + 8);
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_area + 8 * (3 * S + 9));
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_area + 8 * (3 * S + 9) + 4);
 
     // A failure already recorded by this launch (or an earlier, unread one)
     // ends every CTA that has not started, so a fault cannot serialize waits.
@@ -499,6 +493,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(acc_full(b), 1);
             mbar_init(acc_empty(b), ep_count);
         }
+        for (int q = 0; q < 4; ++q) mbar_init(a_free(q), 1);
         mbar_init(mma_done, 1);
         *abort_flag = 0;
         fence_barrier_init();
@@ -535,11 +530,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         wo0 = (rem - ty * a.tiles_w) * a.tw;
     };
 
-    // Register split: warpgroup 0 (producer, MMA issuer, converters) gives
-    // registers up, the two epilogue warpgroups take them (launch: 384 x 168;
-    // after: 128 x 88 + 256 x 208 = 64512, and per scheduler 88 + 2 x 208 <= 512).
+    // Register split by warpgroup (launch: 512 x 128 = 65536): warpgroup 0
+    // (producer, MMA issuer, two idle warps) 40, warpgroup 3 (converters) 72,
+    // warpgroups 1-2 (epilogue) 200: 128 x (40 + 72) + 256 x 200 = 65536, and
+    // per scheduler (one warp of each warpgroup) 32 x (40 + 72 + 2 x 200) = 16384.
+    const int SA = a.a_slots;
     if (warp < 4) {
-    asm volatile("setmaxnreg.dec.sync.aligned.u32 88;" ::: "memory");
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 40;" ::: "memory");
     if (warp == 0) {
         // ---------------------------------------------------------- TMA producer
         if (lane == 0) {
@@ -608,18 +605,20 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
                     if (!mbar_wait(conv_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
                     tc_fence_after();
+                    const int slot = it % SA;
                     const uint32_t st = smem_addr(smem + (size_t)s * a.stage_bytes);
+                    const uint32_t a_t = tmem + (uint32_t)(a.a_col + slot * SUB * 32);
 #pragma unroll
                     for (int u = 0; u < SUB; ++u) {
                         if (u >= nsub) break;
-                        const uint64_t da = sdesc_sw128(st + u * 16384);
                         const uint64_t db = sdesc_sw128(st + a.b_off + u * a.b_bytes);
 #pragma unroll
-                        for (int kk = 0; kk < kBlockK / 16; ++kk)   // K = 16 per instruction, 32 bytes apart
-                            umma_f16(d_tmem, da + (uint64_t)(2 * kk), db + (uint64_t)(2 * kk), idesc,
-                                     (ck0 + u > 0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < kBlockK / 16; ++kk)   // K = 16 per instruction: 8 TMEM columns, 32 bytes of B
+                            umma_f16_ts(d_tmem, a_t + (uint32_t)(u * 32 + kk * 8), db + (uint64_t)(2 * kk), idesc,
+                                        (ck0 + u > 0 || kk > 0) ? 1u : 0u);
                     }
                     umma_commit(empty_bar(s));
+                    umma_commit(a_free(slot));
                     const int kb_end = kb0 + nsub;
                     if (kb_end % a.chunk_kb == 0 || kb_end == a.num_kb) {
                         umma_commit(acc_full(g & 1));
@@ -632,67 +631,72 @@ __global__ void __launch_bounds__(kThreads, 1)
             while (!mbar_try_wait(mma_done, 0) && clock64() - t0 < kWaitLimitCycles) {
             }
         }
-    } else if (warp < 4) {
-        // ---------------------------------------------------------- converters
-        constexpr int kPasses = 512 / kConvThreads;   // 128 rows x 4 quarters per 64-wide block
-        const int ct = threadIdx.x - 64;              // 0..kConvThreads-1
+    }
+    } else if (warp >= 12) {
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 72;" ::: "memory");
+        // ---------------------------------------------------------- converters (warps 12-15)
+        // Thread m converts row m of the A operand (output pixel m of the tile)
+        // into TMEM lane m: 64 INT8 codes -> 32 columns of fp16 pairs.
+        const int quad = warp & 3;
+        const int m = quad * 32 + lane;               // 0..127
+        const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)a.a_col;
         int it = 0;
         bool ok = true;
+        // wait for stage s and A slot it % SA (released by the MMAs that read it)
+        auto acquire = [&](int s, int r) {
+            bool w = mbar_wait(full_bar(s), r & 1, abort_flag, a.err);
+            if (w && it >= SA) w = mbar_wait(a_free(it % SA), ((it / SA) - 1) & 1, abort_flag, a.err);
+            w = __all_sync(0xffffffffu, w);
+            tc_fence_after();
+            return w;
+        };
         if (!a.gather) {
             for (int j = 0; j < my_tiles && ok; ++j) {
                 for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB, ++it) {
                     const int s = it % S, r = it / S;
                     const int nsub = min(SUB, a.num_kb - kb0);
-                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
+                    ok = acquire(s, r);
                     if (!ok) break;
+                    // row m of the INT8 box: 64 bytes, 16-byte chunks permuted by the 64-byte swizzle
+                    const uint8_t *raw = smem + (size_t)s * a.stage_bytes + a.raw_off + m * 64;
+                    const int sw = (m >> 1) & 3;
+                    const uint32_t t_slot = t_lane + (uint32_t)((it % SA) * SUB * 32);
 #pragma unroll 1
                     for (int u = 0; u < SUB; ++u) {
-                    if (u >= nsub) break;
-                    uint8_t *st = smem + (size_t)s * a.stage_bytes + u * 16384;
-                    const uint8_t *raw = smem + (size_t)s * a.stage_bytes + a.raw_off + u * 8192;
-                    // thread -> (row m, 8-element chunk c): 8 consecutive lanes cover one
-                    // row, i.e. all 32 banks for both the 8-byte loads and the swizzled stores
-                    uint2 v[2 * kPasses];                  // all loads first, then convert and store
+                        if (u >= nsub) break;
+                        uint4 v[4];
 #pragma unroll
-                    for (int p = 0; p < 2 * kPasses; ++p) {
-                        const int idx = p * kConvThreads + ct;
-                        v[p] = *reinterpret_cast<const uint2 *>(raw + idx * 8);
-                    }
+                        for (int q = 0; q < 4; ++q) v[q] = *reinterpret_cast<const uint4 *>(raw + u * 8192 + ((q ^ sw) << 4));
+                        uint32_t h[32];
 #pragma unroll
-                    for (int p = 0; p < 2 * kPasses; ++p) {
-                        const int idx = p * kConvThreads + ct;
-                        uint32_t h[4];
-                        i8x4_to_f16x4(v[p].x, h[0], h[1]);
-                        i8x4_to_f16x4(v[p].y, h[2], h[3]);
-                        *reinterpret_cast<int4 *>(st + sw128_offset(idx >> 3, idx & 7)) =
-                            make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
+                        for (int q = 0; q < 4; ++q) {
+                            i8x4_to_f16x4(v[q].x, h[8 * q + 0], h[8 * q + 1]);
+                            i8x4_to_f16x4(v[q].y, h[8 * q + 2], h[8 * q + 3]);
+                            i8x4_to_f16x4(v[q].z, h[8 * q + 4], h[8 * q + 5]);
+                            i8x4_to_f16x4(v[q].w, h[8 * q + 6], h[8 * q + 7]);
+                        }
+                        tmem_st32(t_slot + (uint32_t)(u * 32), h);
                     }
-                    }
-                    fence_proxy_async_smem();
+                    tmem_wait_st();
+                    tc_fence_before();
                     mbar_arrive(conv_bar(s));
                 }
             }
         } else {
-            // Small-channel layer: each tile's input window ((th-1)s+kh rows of
+            // Small-channel layer. Each tile's input window ((th-1)s+kh rows of
             // (tw-1)s+kw pixels, zero outside the image) is copied to shared
-            // memory with coalesced byte loads, then the packed reduction index
-            // k = (ky, kx, ci) is gathered from it through a per-CTA offset table.
-            int *tab = reinterpret_cast<int *>(bar_area + 8 * (3 * S + 7) + 16);
+            // memory; kernel row ky of output pixel m is then one contiguous
+            // kw*c-byte segment of window row py*s+ky, read as 8-entry pieces
+            // through a per-CTA table (window offset of each piece, -1 = zero).
+            int *tab = reinterpret_cast<int *>(bar_area + 8 * (3 * S + 9) + 16);
             uint8_t *win = bar_area + a.win_off;
-            const int taps = a.kh * a.kw;
-            for (int k = ct; k < a.num_kb * kBlockK; k += kConvThreads) {
-                const int tap = k / a.c, ci = k - tap * a.c;
-                const int ky = tap / a.kw, kx = tap - ky * a.kw;
-                tab[k] = tap < taps ? (ky * a.win_w + kx) * a.c + ci : -1;
+            for (int q = m; q < a.num_kb * 8; q += kConvThreads) {
+                const int k0 = q * 8, ky = k0 / a.seg;
+                tab[q] = ky < a.kh ? ky * a.win_pitch + (k0 - ky * a.seg) : -1;
             }
-            int rb[kPasses];
-#pragma unroll
-            for (int p = 0; p < kPasses; ++p) {
-                const int m = (p * kConvThreads + ct) >> 2;
-                rb[p] = ((m / a.tw) * a.stride * a.win_w + (m % a.tw) * a.stride) * a.c;
-            }
+            const int rbase = (m / a.tw) * a.stride * a.win_pitch + (m % a.tw) * a.stride * a.c;
             // Every converter thread runs the same tile loop (also after an
-            // abort, doing no work) so both warps reach each named barrier.
+            // abort, doing no work) so all four warps reach each named barrier.
             for (int j = 0; j < my_tiles; ++j) {
                 int img, ho0, wo0, n0;
                 tile_coords(j, img, ho0, wo0, n0);
@@ -702,22 +706,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int row_b = a.win_w * a.c;
                     const int b_lo = max(0, -ix_lo) * a.c, b_hi = min(a.win_w, a.w - ix_lo) * a.c;
                     // per row, all of a thread's loads are issued before its stores
-                    // (one memory round trip per 16 x 64 bytes instead of per byte)
                     for (int r = 0; r < a.win_h; ++r) {
                         const int iy = ho0 * a.stride - a.pad + r;
                         const bool row_in = iy >= 0 && iy < a.h;
                         const int8_t *src = a.x + (((long long)img * a.h + (row_in ? iy : 0)) * a.w + ix_lo) * a.c;
-                        for (int b0 = ct; b0 < row_b; b0 += 16 * kConvThreads) {
-                            uint8_t v[16];
+                        for (int b0 = m; b0 < row_b; b0 += 8 * kConvThreads) {
+                            uint8_t v[8];
 #pragma unroll
-                            for (int u = 0; u < 16; ++u) {
+                            for (int u = 0; u < 8; ++u) {
                                 const int b = b0 + u * kConvThreads;
                                 v[u] = (row_in && b >= b_lo && b < b_hi) ? (uint8_t)__ldg(src + b) : (uint8_t)0;
                             }
 #pragma unroll
-                            for (int u = 0; u < 16; ++u) {
+                            for (int u = 0; u < 8; ++u) {
                                 const int b = b0 + u * kConvThreads;
-                                if (b < row_b) win[r * row_b + b] = v[u];
+                                if (b < row_b) win[r * a.win_pitch + b] = v[u];
                             }
                         }
                     }
@@ -725,34 +728,32 @@ __global__ void __launch_bounds__(kThreads, 1)
                 asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // window complete
                 for (int kb = 0; kb < a.num_kb && ok; ++kb, ++it) {
                     const int s = it % S, r = it / S;
-                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
+                    ok = acquire(s, r);
                     if (!ok) break;
-                    uint8_t *st = smem + (size_t)s * a.stage_bytes;
+                    uint32_t h[32];
 #pragma unroll
-                    for (int p = 0; p < kPasses; ++p) {
-                        const int idx = p * kConvThreads + ct;
-                        const int m = idx >> 2, q = idx & 3;
-                        uint32_t w4[4] = {0u, 0u, 0u, 0u};
-#pragma unroll
-                        for (int jj = 0; jj < 16; ++jj) {
-                            const int off = tab[kb * kBlockK + q * 16 + jj];
-                            const uint32_t bb = off >= 0 ? (uint32_t)win[rb[p] + off] : 0u;
-                            w4[jj >> 2] |= bb << (8 * (jj & 3));
+                    for (int q = 0; q < 8; ++q) {
+                        const int off = tab[kb * 8 + q];
+                        uint32_t w0 = 0u, w1 = 0u;
+                        if (off >= 0) {
+                            const int o = rbase + off;
+                            const uint32_t *p = reinterpret_cast<const uint32_t *>(win + (o & ~3));
+                            const uint32_t x0 = p[0], x1 = p[1], x2 = p[2];
+                            w0 = __funnelshift_r(x0, x1, (uint32_t)(o & 3) * 8u);
+                            w1 = __funnelshift_r(x1, x2, (uint32_t)(o & 3) * 8u);
                         }
-                        uint32_t h[8];
-#pragma unroll
-                        for (int jj = 0; jj < 4; ++jj) i8x4_to_f16x4(w4[jj], h[2 * jj], h[2 * jj + 1]);
-                        *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q)) = make_int4((int)h[0], (int)h[1], (int)h[2], (int)h[3]);
-                        *reinterpret_cast<int4 *>(st + sw128_offset(m, 2 * q + 1)) = make_int4((int)h[4], (int)h[5], (int)h[6], (int)h[7]);
+                        i8x4_to_f16x4(w0, h[4 * q + 0], h[4 * q + 1]);
+                        i8x4_to_f16x4(w1, h[4 * q + 2], h[4 * q + 3]);
                     }
-                    fence_proxy_async_smem();
+                    tmem_st32(t_lane + (uint32_t)((it % SA) * 32), h);
+                    tmem_wait_st();
+                    tc_fence_before();
                     mbar_arrive(conv_bar(s));
                 }
             }
         }
-    }
     } else {
-        asm volatile("setmaxnreg.inc.sync.aligned.u32 208;" ::: "memory");
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 200;" ::: "memory");
         // ---------------------------------------------------------- epilogue warpgroups (warps 4-7, 8-11)
         const int wg = (warp - 4) >> 2;            // 0 or 1
         const int quad = warp & 3;                 // TMEM lane quadrant this warp may access

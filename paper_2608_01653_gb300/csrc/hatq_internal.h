@@ -54,17 +54,20 @@ struct ConvArgs {
     int num_kb;                      // 64-wide reduction blocks
     int cin_kb;                      // reduction blocks per kernel tap (tiled loader)
     int gather;                      // small-channel loader
+    int seg;                         // small-channel loader: reduction entries per kernel row (kw * c, padded to 8)
     int chunk_kb;                    // reduction blocks per exact fp32 chunk
     int stages;
     int tmem_cols;                   // TMEM columns allocated (power of two)
+    int a_col, a_slots;              // TMEM column of the fp16 A-operand ring and its slots (sub x 32 columns each)
     int nbuf, buf_cols;              // 2: epilogue warpgroups alternate tiles; 1: they split columns (drains); n_t
     int num_tiles, n_tiles_n;        // output tiles in the launch, N tiles per M tile
     int stage_bytes, b_bytes, raw_bytes;
     int sub;                         // 64-wide reduction blocks per pipeline stage (1 or 2)
-    int b_off, raw_off;              // offsets of the weight and INT8 boxes inside a stage
+    int b_off, raw_off;              // offsets of the weight and INT8 (64-byte swizzled) boxes inside a stage
     int staging_bytes, row_stride;   // shared-memory output tiles after the stages
     int const_off;                   // offsets from the barrier area: epilogue constants,
     int win_off, win_h, win_w;       // small-channel input window and its size
+    int win_pitch;                   // bytes per window row
     const int8_t *x;
     const int32_t *b_int;
     const int32_t *mult;

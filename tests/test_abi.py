@@ -39,7 +39,9 @@ def test_version_and_last_error(lib):
 
 @pytest.mark.parametrize("desc,k_pad", [
     (H.make_desc(192, 192, 5, 2, 2, "DH", hb_in=64), 25 * 192),
-    (H.make_desc(3, 192, 5, 2, 2, "WH", hb_out=64), 128),       # small-channel packing 75 -> 128
+    (H.make_desc(3, 192, 5, 2, 2, "WH", hb_out=64), 128),       # small-channel packing 5 x 16 -> 128
+    (H.make_desc(3, 64, 3, 1, 1, "WH", hb_out=64), 64),         # 3 x 16 -> 64
+    (H.make_desc(5, 64, 5, 1, 2, "WH", hb_out=64), 192),        # 5 x 32 -> 192
     (H.make_desc(32, 224, 3, 1, 1, "DH", hb_in=32), 9 * 64),    # c_in padded to 64 per tap
     (H.make_desc(224, 128, 3, 1, 1, "WH", hb_out=128), 9 * 256),
     (H.make_desc(128, 128, 1, 1, 0, "DH", hb_in=128), 128),
@@ -83,7 +85,10 @@ def _oracle_packed(p, desc, k_pad):
     co, kh, kw, ci = p.w_int.shape
     out = np.zeros((co, k_pad), np.int8)
     if ci % 16:
-        out[:, :kh * kw * ci] = p.w_int.reshape(co, -1)
+        seg = (kw * ci + 7) // 8 * 8            # one kernel row (kx, ci), zero-padded to a multiple of 8
+        tmp = np.zeros((co, kh, seg), np.int8)
+        tmp[:, :, :kw * ci] = p.w_int.reshape(co, kh, kw * ci)
+        out[:, :kh * seg] = tmp.reshape(co, -1)
     else:
         cin_pad = (ci + 63) // 64 * 64
         tmp = np.zeros((co, kh * kw, cin_pad), np.int8)
