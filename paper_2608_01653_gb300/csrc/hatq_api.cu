@@ -485,12 +485,16 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     const int const_bytes = (3 * d->c_out * 4 + 127) & ~127;
     const int fixed = 1024 /* align */ + 8 * (3 * 8 + 9) + 16 + 128 + table_bytes + const_bytes + win_bytes;
     const int budget = 227 * 1024 - 1024 /* static */ - fixed - a.staging_bytes;
-    // a stage holds `sub` 64-wide reduction blocks: [weights x sub | INT8 box x sub];
-    // two blocks per stage halve the barrier round trips per MMA where three
-    // such stages and two A slots of 64 columns fit
+    // a stage holds `sub` 64-wide reduction blocks: [weights x sub | INT8 box x sub].
+    // The cost of a stage is dominated by its barrier hand-offs, not its bytes,
+    // so take the widest stage that still leaves two stages and two A slots:
+    // four blocks (two 4-block stages, 2 x 128 TMEM columns), else two (three
+    // stages, 2 x 64 columns), else one.
     const int one = a.b_bytes + a.raw_bytes;
     const int free_cols = 512 - a.a_col;
-    a.sub = (!g.gather && a.num_kb > 1 && budget / (2 * one) >= 3 && free_cols >= 128) ? 2 : 1;
+    a.sub = 1;
+    if (!g.gather && a.num_kb >= 4 && budget / (4 * one) >= 2 && free_cols >= 256) a.sub = 4;
+    else if (!g.gather && a.num_kb > 1 && budget / (2 * one) >= 3 && free_cols >= 128) a.sub = 2;
     a.a_slots = free_cols / (32 * a.sub);
     if (a.a_slots > 4) a.a_slots = 4;
     if (a.a_slots < 2) return fail(HATQ_ERR_UNSUPPORTED, "no TMEM room for the A operand (n_t=%d)", a.n_t);

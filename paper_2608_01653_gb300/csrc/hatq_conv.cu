@@ -444,7 +444,7 @@ __device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a,
 // one chunk per tile epilogue warpgroup w takes the tiles of region w; with
 // several, both warpgroups drain every chunk into int32 register partials
 // (half of the 32-column groups each) and finish the tile together.
-// SUB: 64-wide reduction blocks per pipeline stage (1 or 2)
+// SUB: 64-wide reduction blocks per pipeline stage (1, 2 or 4)
 template <int SUB>
 __global__ void __launch_bounds__(kThreads, 1)
     conv_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const ConvArgs a) {
@@ -642,39 +642,46 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)a.a_col;
         int it = 0;
         bool ok = true;
-        // wait for stage s and A slot it % SA (released by the MMAs that read it)
-        auto acquire = [&](int s, int r) {
-            bool w = mbar_wait(full_bar(s), r & 1, abort_flag, a.err);
-            if (w && it >= SA) w = mbar_wait(a_free(it % SA), ((it / SA) - 1) & 1, abort_flag, a.err);
+        // wait until A slot it % SA was released by the MMAs that last read it
+        auto slot_free = [&]() {
+            bool w = it < SA || mbar_wait(a_free(it % SA), ((it / SA) - 1) & 1, abort_flag, a.err);
             w = __all_sync(0xffffffffu, w);
             tc_fence_after();
             return w;
         };
         if (!a.gather) {
+            // row m of a 64-wide INT8 box (64 bytes, 16-byte chunks permuted by the
+            // 64-byte swizzle) -> 32 columns of fp16 pairs
+            auto convert_row = [&](const uint8_t *raw, uint32_t (&h)[32]) {
+                const int sw = (m >> 1) & 3;
+                uint4 v[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) v[q] = *reinterpret_cast<const uint4 *>(raw + ((q ^ sw) << 4));
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    i8x4_to_f16x4(v[q].x, h[8 * q + 0], h[8 * q + 1]);
+                    i8x4_to_f16x4(v[q].y, h[8 * q + 2], h[8 * q + 3]);
+                    i8x4_to_f16x4(v[q].z, h[8 * q + 4], h[8 * q + 5]);
+                    i8x4_to_f16x4(v[q].w, h[8 * q + 6], h[8 * q + 7]);
+                }
+            };
             for (int j = 0; j < my_tiles && ok; ++j) {
                 for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB, ++it) {
                     const int s = it % S, r = it / S;
                     const int nsub = min(SUB, a.num_kb - kb0);
-                    ok = acquire(s, r);
+                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
                     if (!ok) break;
-                    // row m of the INT8 box: 64 bytes, 16-byte chunks permuted by the 64-byte swizzle
                     const uint8_t *raw = smem + (size_t)s * a.stage_bytes + a.raw_off + m * 64;
-                    const int sw = (m >> 1) & 3;
                     const uint32_t t_slot = t_lane + (uint32_t)((it % SA) * SUB * 32);
+                    uint32_t h[32];
+                    convert_row(raw, h);              // the first block is converted before the slot frees up
+                    ok = slot_free();
+                    if (!ok) break;
+                    tmem_st32(t_slot, h);
 #pragma unroll 1
-                    for (int u = 0; u < SUB; ++u) {
+                    for (int u = 1; u < SUB; ++u) {
                         if (u >= nsub) break;
-                        uint4 v[4];
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) v[q] = *reinterpret_cast<const uint4 *>(raw + u * 8192 + ((q ^ sw) << 4));
-                        uint32_t h[32];
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            i8x4_to_f16x4(v[q].x, h[8 * q + 0], h[8 * q + 1]);
-                            i8x4_to_f16x4(v[q].y, h[8 * q + 2], h[8 * q + 3]);
-                            i8x4_to_f16x4(v[q].z, h[8 * q + 4], h[8 * q + 5]);
-                            i8x4_to_f16x4(v[q].w, h[8 * q + 6], h[8 * q + 7]);
-                        }
+                        convert_row(raw + u * 8192, h);
                         tmem_st32(t_slot + (uint32_t)(u * 32), h);
                     }
                     tmem_wait_st();
@@ -727,9 +734,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // window complete
                 for (int kb = 0; kb < a.num_kb && ok; ++kb, ++it) {
+                    // the operand comes from the window: it is built first, then the
+                    // stage (which keeps conv[s] in step with the MMA issuer) and the
+                    // A slot are waited for
                     const int s = it % S, r = it / S;
-                    ok = acquire(s, r);
-                    if (!ok) break;
                     uint32_t h[32];
 #pragma unroll
                     for (int q = 0; q < 8; ++q) {
@@ -745,6 +753,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                         i8x4_to_f16x4(w0, h[4 * q + 0], h[4 * q + 1]);
                         i8x4_to_f16x4(w1, h[4 * q + 2], h[4 * q + 3]);
                     }
+                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
+                    if (!ok) break;
+                    ok = slot_free();
+                    if (!ok) break;
                     tmem_st32(t_lane + (uint32_t)((it % SA) * 32), h);
                     tmem_wait_st();
                     tc_fence_before();
@@ -885,17 +897,19 @@ __global__ void __launch_bounds__(kThreads, 1)
 cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const ConvArgs &a, int smem_bytes, cudaStream_t s) {
     // the shared-memory opt-in and the SM count are per device
     constexpr int kMaxDev = 64;
-    static int configured_smem[kMaxDev][2] = {};
+    static int configured_smem[kMaxDev][3] = {};
     static int sms_of[kMaxDev] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
-    if (a.sub != 1 && (a.sub != 2 || a.gather)) return cudaErrorInvalidValue;   // gathered tiles: one block per stage
-    const int v = a.sub == 2 ? 1 : 0;
+    if ((a.sub != 1 && a.sub != 2 && a.sub != 4) || (a.gather && a.sub != 1) || a.chunk_kb % a.sub)
+        return cudaErrorInvalidValue;   // gathered tiles: one block per stage
+    const int v = a.sub == 4 ? 2 : (a.sub == 2 ? 1 : 0);
+    void (*const kern)(const CUtensorMap, const CUtensorMap, const ConvArgs) =
+        v == 2 ? conv_kernel<4> : (v == 1 ? conv_kernel<2> : conv_kernel<1>);
     if (smem_bytes > configured_smem[dev][v]) {
-        e = cudaFuncSetAttribute(v ? conv_kernel<2> : conv_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 smem_bytes);
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
         if (e != cudaSuccess) return e;
         configured_smem[dev][v] = smem_bytes;
     }
@@ -906,10 +920,7 @@ cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const Co
         sms_of[dev] = sms > 0 ? sms : 1;
     }
     const int grid = a.num_tiles < sms_of[dev] ? a.num_tiles : sms_of[dev];
-    if (v)
-        conv_kernel<2><<<grid, kThreads, smem_bytes, s>>>(tmA, tmB, a);
-    else
-        conv_kernel<1><<<grid, kThreads, smem_bytes, s>>>(tmA, tmB, a);
+    kern<<<grid, kThreads, smem_bytes, s>>>(tmA, tmB, a);
     return cudaGetLastError();
 }
 
