@@ -540,42 +540,46 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
         // ---------------------------------------------------------- TMA producer
         if (lane == 0) {
+            // stage s with phase parity ph, advanced incrementally (the issuing
+            // threads of the pipeline avoid integer division)
             const uint32_t tx_bytes = (uint32_t)(a.b_bytes + (a.gather ? 0 : a.raw_bytes));
-            int issued_round[8];
-            for (int s = 0; s < 8; ++s) issued_round[s] = -1;
+            int issued_ph[8];
+            for (int q = 0; q < 8; ++q) issued_ph[q] = -1;
             bool ok = true;
-            int it = 0;
+            int s = 0;
+            uint32_t ph = 0;
             for (int j = 0; j < my_tiles && ok; ++j) {
                 int img, ho0, wo0, n0;
                 tile_coords(j, img, ho0, wo0, n0);
-                for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB, ++it) {
-                    const int s = it % S, r = it / S;
+                int cb = 0, kx = 0, ky = 0;          // 64-channel block, kernel column and row of block kb
+                for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB) {
                     const int nsub = min(SUB, a.num_kb - kb0);
-                    if (!mbar_wait(empty_bar(s), (r & 1) ^ 1, abort_flag, a.err)) { ok = false; break; }
+                    if (!mbar_wait(empty_bar(s), ph ^ 1, abort_flag, a.err)) { ok = false; break; }
                     const uint32_t st = smem_addr(smem + (size_t)s * a.stage_bytes);
                     mbar_expect_tx(full_bar(s), tx_bytes * (uint32_t)nsub);
 #pragma unroll
                     for (int u = 0; u < SUB; ++u) {
                         if (u >= nsub) break;
-                        const int kb = kb0 + u;
-                        tma_load_2d(st + a.b_off + u * a.b_bytes, &tmB, full_bar(s), kb * kBlockK, n0);
+                        tma_load_2d(st + a.b_off + u * a.b_bytes, &tmB, full_bar(s), (kb0 + u) * kBlockK, n0);
                         if (!a.gather) {
-                            const int tap = kb / a.cin_kb;
-                            const int c0 = (kb - tap * a.cin_kb) * kBlockK;
-                            const int ky = tap / a.kw, kx = tap - (tap / a.kw) * a.kw;
-                            tma_load_4d(st + a.raw_off + u * 8192, &tmA, full_bar(s), c0, wo0 * a.stride + kx - a.pad,
-                                        ho0 * a.stride + ky - a.pad, img);
+                            tma_load_4d(st + a.raw_off + u * 8192, &tmA, full_bar(s), cb * kBlockK,
+                                        wo0 * a.stride + kx - a.pad, ho0 * a.stride + ky - a.pad, img);
+                            if (++cb == a.cin_kb) {
+                                cb = 0;
+                                if (++kx == a.kw) { kx = 0; ++ky; }
+                            }
                         }
                     }
-                    issued_round[s] = r;
+                    issued_ph[s] = (int)ph;
+                    if (++s == S) { s = 0; ph ^= 1u; }
                 }
             }
             if (!ok) {
                 // let our own copies land before the CTA unwinds
-                for (int s = 0; s < S && s < 8; ++s)
-                    if (issued_round[s] >= 0) {
+                for (int q = 0; q < S && q < 8; ++q)
+                    if (issued_ph[q] >= 0) {
                         const long long t0 = clock64();
-                        while (!mbar_try_wait(full_bar(s), issued_round[s] & 1) && clock64() - t0 < kWaitLimitCycles) {
+                        while (!mbar_try_wait(full_bar(q), (uint32_t)issued_ph[q]) && clock64() - t0 < kWaitLimitCycles) {
                         }
                     }
             }
@@ -584,46 +588,51 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------------------------------------------------- MMA issuer
         if (lane == 0) {
             const uint32_t idesc = idesc_f16(a.n_t);
+            // weight descriptor of stage 0, block 0; a stage / block moves its start address field
+            const uint64_t desc0 = sdesc_sw128(smem_addr(smem) + (uint32_t)a.b_off);
+            const uint32_t stage_step = (uint32_t)a.stage_bytes >> 4, blk_step = (uint32_t)a.b_bytes >> 4;
             bool ok = true;
-            int it = 0;
+            int s = 0, slot = 0;
+            uint32_t ph = 0;
             int g = 0;                       // exact chunks issued so far; chunk g accumulates in region g & 1
             uint32_t d_tmem = tmem;
             for (int j = 0; j < my_tiles && ok; ++j) {
                 // a stage holds SUB 64-wide reduction blocks; chunk boundaries
                 // (multiples of chunk_kb, itself a multiple of SUB) fall between stages
-                for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB, ++it) {
-                    const int s = it % S, r = it / S;
+                int ck = 0;                  // blocks of the current exact chunk already issued
+                for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB) {
                     const int nsub = min(SUB, a.num_kb - kb0);
-                    const int ck0 = kb0 % a.chunk_kb;
-                    if (ck0 == 0) {
+                    if (ck == 0) {
                         d_tmem = tmem + (uint32_t)((g & 1) * a.n_t);
                         if (g >= 2) {        // wait until the epilogue released the region
                             if (!mbar_wait(acc_empty(g & 1), ((g >> 1) - 1) & 1, abort_flag, a.err)) { ok = false; break; }
                             tc_fence_after();
                         }
                     }
-                    if (!mbar_wait(full_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
-                    if (!mbar_wait(conv_bar(s), r & 1, abort_flag, a.err)) { ok = false; break; }
+                    if (!mbar_wait(full_bar(s), ph, abort_flag, a.err)) { ok = false; break; }
+                    if (!mbar_wait(conv_bar(s), ph, abort_flag, a.err)) { ok = false; break; }
                     tc_fence_after();
-                    const int slot = it % SA;
-                    const uint32_t st = smem_addr(smem + (size_t)s * a.stage_bytes);
+                    const uint64_t db0 = desc0 + (uint64_t)((uint32_t)s * stage_step);
                     const uint32_t a_t = tmem + (uint32_t)(a.a_col + slot * SUB * 32);
 #pragma unroll
                     for (int u = 0; u < SUB; ++u) {
                         if (u >= nsub) break;
-                        const uint64_t db = sdesc_sw128(st + a.b_off + u * a.b_bytes);
+                        const uint64_t db = db0 + (uint64_t)((uint32_t)u * blk_step);
 #pragma unroll
                         for (int kk = 0; kk < kBlockK / 16; ++kk)   // K = 16 per instruction: 8 TMEM columns, 32 bytes of B
                             umma_f16_ts(d_tmem, a_t + (uint32_t)(u * 32 + kk * 8), db + (uint64_t)(2 * kk), idesc,
-                                        (ck0 + u > 0 || kk > 0) ? 1u : 0u);
+                                        (ck + u > 0 || kk > 0) ? 1u : 0u);
                     }
                     umma_commit(empty_bar(s));
                     umma_commit(a_free(slot));
-                    const int kb_end = kb0 + nsub;
-                    if (kb_end % a.chunk_kb == 0 || kb_end == a.num_kb) {
+                    ck += nsub;
+                    if (ck == a.chunk_kb || kb0 + nsub == a.num_kb) {
                         umma_commit(acc_full(g & 1));
                         ++g;
+                        ck = 0;
                     }
+                    if (++s == S) { s = 0; ph ^= 1u; }
+                    if (++slot == SA) slot = 0;
                 }
             }
             umma_commit(mma_done);
@@ -640,11 +649,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int quad = warp & 3;
         const int m = quad * 32 + lane;               // 0..127
         const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16) + (uint32_t)a.a_col;
-        int it = 0;
         bool ok = true;
-        // wait until A slot it % SA was released by the MMAs that last read it
+        // stage s (phase parity ph) and A slot (use parity sph), advanced incrementally
+        int s = 0, slot = 0;
+        uint32_t ph = 0, sph = 0;
+        bool reuse = false;                           // the slot was used before (some slot wrapped)
+        auto advance = [&]() {
+            if (++s == S) { s = 0; ph ^= 1u; }
+            if (++slot == SA) { slot = 0; sph ^= 1u; reuse = true; }
+        };
+        // wait until the A slot was released by the MMAs that last read it
         auto slot_free = [&]() {
-            bool w = it < SA || mbar_wait(a_free(it % SA), ((it / SA) - 1) & 1, abort_flag, a.err);
+            bool w = !reuse || mbar_wait(a_free(slot), sph ^ 1u, abort_flag, a.err);
             w = __all_sync(0xffffffffu, w);
             tc_fence_after();
             return w;
@@ -666,13 +682,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             };
             for (int j = 0; j < my_tiles && ok; ++j) {
-                for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB, ++it) {
-                    const int s = it % S, r = it / S;
+                for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB) {
                     const int nsub = min(SUB, a.num_kb - kb0);
-                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
+                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), ph, abort_flag, a.err));
                     if (!ok) break;
                     const uint8_t *raw = smem + (size_t)s * a.stage_bytes + a.raw_off + m * 64;
-                    const uint32_t t_slot = t_lane + (uint32_t)((it % SA) * SUB * 32);
+                    const uint32_t t_slot = t_lane + (uint32_t)(slot * SUB * 32);
                     uint32_t h[32];
                     convert_row(raw, h);              // the first block is converted before the slot frees up
                     ok = slot_free();
@@ -687,6 +702,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tmem_wait_st();
                     tc_fence_before();
                     mbar_arrive(conv_bar(s));
+                    advance();
                 }
             }
         } else {
@@ -733,11 +749,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                 }
                 asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // window complete
-                for (int kb = 0; kb < a.num_kb && ok; ++kb, ++it) {
+                for (int kb = 0; kb < a.num_kb && ok; ++kb) {
                     // the operand comes from the window: it is built first, then the
                     // stage (which keeps conv[s] in step with the MMA issuer) and the
                     // A slot are waited for
-                    const int s = it % S, r = it / S;
                     uint32_t h[32];
 #pragma unroll
                     for (int q = 0; q < 8; ++q) {
@@ -753,14 +768,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                         i8x4_to_f16x4(w0, h[4 * q + 0], h[4 * q + 1]);
                         i8x4_to_f16x4(w1, h[4 * q + 2], h[4 * q + 3]);
                     }
-                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), r & 1, abort_flag, a.err));
+                    ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), ph, abort_flag, a.err));
                     if (!ok) break;
                     ok = slot_free();
                     if (!ok) break;
-                    tmem_st32(t_lane + (uint32_t)((it % SA) * 32), h);
+                    tmem_st32(t_lane + (uint32_t)(slot * 32), h);
                     tmem_wait_st();
                     tc_fence_before();
                     mbar_arrive(conv_bar(s));
+                    advance();
                 }
             }
         }
