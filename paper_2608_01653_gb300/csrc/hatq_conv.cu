@@ -11,24 +11,25 @@
 // fp32 accumulators in tensor memory (TMEM). Every product is an integer of
 // magnitude <= 127^2 and every partial sum of a 1024-long reduction chunk is
 // an integer of magnitude <= 1024 * 127^2 < 2^24, so all fp32 values involved
-// are exactly representable integers and the chunk sum is exact. After each
-// chunk the epilogue warps convert the chunk sum to int32 and add it to an
-// int32 partial held in a second TMEM region, so the full accumulator is the
-// exact int32 sum.
+// are exactly representable integers and the chunk sum is exact. Chunk g
+// accumulates in TMEM region g & 1; the epilogue warps convert finished chunks
+// to int32 and add them into int32 partials in their registers, so the full
+// accumulator is the exact int32 sum.
 //
-// Warp roles (one 128 x N_t output tile per CTA, 256 threads; two warps per
-// SM sub-partition, so each thread may hold up to 255 registers):
-//   warp 0     TMA producer: weight tile (fp16, 128B-swizzled) and, for
-//              c_in % 16 == 0, the INT8 activation box of one kernel tap and
-//              64 input channels (zero fill outside the image = zero padding).
-//   warp 1     TMEM allocation; lane 0 issues the MMAs and commits.
-//   warps 2-3  converters: INT8 box -> fp16 operand tile in the 128B-swizzled
-//              K-major layout the MMA descriptor expects (or, for small c_in,
-//              a gather from the tile's input window staged in shared memory).
-//   warps 4-7  drain fp32 chunk sums into the int32 partial.
-//   all warps  final epilogue once the last MMA completed: warps w and w+4
-//              share TMEM lane quadrant w%4 and split the column groups; the
-//              output tile is staged in shared memory and copied out coalesced.
+// Persistent kernel, one CTA per SM, 512 threads in four warpgroups:
+//   warp 0      TMA producer: weight tile (fp16, 128B-swizzled) and, for
+//               c_in % 16 == 0, the INT8 activation box of one kernel tap and
+//               64 input channels (64B-swizzled; zero fill outside the image =
+//               zero padding), SUB 64-wide blocks per pipeline stage.
+//   warp 1      TMEM allocation; lane 0 issues the MMAs (A operand in TMEM,
+//               B in shared memory) and commits.
+//   warps 2-3   idle (they complete warpgroup 0 for the register split).
+//   warps 4-11  epilogue warpgroups: drains and the fused requantize /
+//               Hadamard epilogue into a shared-memory output tile, copied out
+//               coalesced.
+//   warps 12-15 converters, one per TMEM lane quadrant: INT8 row -> fp16 pairs
+//               in a TMEM slot ring (for small c_in, gathered from the tile's
+//               input window staged in shared memory).
 // Every mbarrier wait is bounded: on expiry the kernel records an error word,
 // raises a CTA-wide abort flag and unwinds (waiting, again bounded, for its own
 // MMAs and copies) before freeing TMEM.
