@@ -10,9 +10,9 @@
 // (hb <= 256, hb | C, 16 | C) lies inside one warp: the first log2(min(hb,16))
 // butterfly stages run inside a lane, the rest across lanes with __shfl_xor.
 //
-// INT8 entry: the integer butterfly runs on packed int16 pairs (|partial| <=
-// 127 * 2^s < 2^15 for hb <= 256, so 16-bit lanes are exact), then
-// y = clamp(round_half_even(M_q v / 2^n_q)).
+// INT8 entry: the integer butterfly runs on sign-extended int32 elements
+// (cross-lane stages as one shuffle and one multiply-add by +-1), then
+// y = clamp(round_half_even(M_q v / 2^n_q)), for n_q >= 32 in 32-bit pieces.
 // FP16 entry: fp32 butterfly, y = clamp(rint(v * inv)), inv = 1/(sqrt(hb) s).
 #include <cuda_fp16.h>
 
@@ -29,60 +29,41 @@ __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
     return d;
 }
 
-// 16 int8 codes -> 8 registers, register k = (element 2k | element 2k+1 << 16),
-// sign-extended to int16 (prmt selector bit 3 replicates the byte's sign).
-__device__ __forceinline__ void unpack_i8x16(const int4 raw, uint32_t (&r)[8]) {
+// 16 int8 codes -> 16 sign-extended int32 (prmt selector bit 3 replicates the sign).
+__device__ __forceinline__ void unpack_i8x16_i32(const int4 raw, int (&v)[16]) {
     const uint32_t w[4] = {(uint32_t)raw.x, (uint32_t)raw.y, (uint32_t)raw.z, (uint32_t)raw.w};
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        r[2 * i] = prmt(w[i], 0u, 0x9180u);
-        r[2 * i + 1] = prmt(w[i], 0u, 0xB3A2u);
+        v[4 * i + 0] = (int)prmt(w[i], 0u, 0x8880u);
+        v[4 * i + 1] = (int)prmt(w[i], 0u, 0x9991u);
+        v[4 * i + 2] = (int)prmt(w[i], 0u, 0xAAA2u);
+        v[4 * i + 3] = (int)prmt(w[i], 0u, 0xBBB3u);
     }
 }
 
-// Sylvester butterfly over 16 packed elements of one lane plus the
-// cross-lane stages; afterwards each element holds (H~_hb x)_j.
-__device__ __forceinline__ void butterfly_i16(uint32_t (&r)[8], int hb, int lane) {
-    if (hb >= 2) {
+// Sylvester butterfly over the 16 elements of one lane plus the cross-lane
+// stages; afterwards each element holds (H~_hb x)_j. In a cross-lane stage
+// the upper lane of a pair keeps partner - own, the lower own + partner.
+__device__ __forceinline__ void butterfly_i32(int (&v)[16], int hb, int lane) {
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const uint32_t sw = prmt(r[k], 0u, 0x1032u);
-            r[k] = prmt(__vadd2(r[k], sw), __vsub2(r[k], sw), 0x5410u);
-        }
-    }
-    if (hb >= 4) {
+    for (int h = 1; h < 16; h <<= 1) {
+        if (h >= hb) break;
 #pragma unroll
-        for (int k = 0; k < 8; k += 2) {
-            const uint32_t a = r[k], b = r[k + 1];
-            r[k] = __vadd2(a, b);
-            r[k + 1] = __vsub2(a, b);
-        }
-    }
-    if (hb >= 8) {
-#pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            if (k & 2) continue;
-            const uint32_t a = r[k], b = r[k + 2];
-            r[k] = __vadd2(a, b);
-            r[k + 2] = __vsub2(a, b);
-        }
-    }
-    if (hb >= 16) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const uint32_t a = r[k], b = r[k + 4];
-            r[k] = __vadd2(a, b);
-            r[k + 4] = __vsub2(a, b);
+        for (int i = 0; i < 16; ++i) {
+            if (i & h) continue;
+            const int a = v[i], b = v[i + h];
+            v[i] = a + b;
+            v[i + h] = a - b;
         }
     }
 #pragma unroll
     for (int m = 1; m < 16; m <<= 1) {
         if (16 * m >= hb) break;
-        const bool upper = (lane & m) != 0;
+        const int sgn = (lane & m) ? -1 : 1;
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const uint32_t p = __shfl_xor_sync(0xffffffffu, r[k], m);
-            r[k] = upper ? __vsub2(p, r[k]) : __vadd2(r[k], p);
+        for (int i = 0; i < 16; ++i) {
+            const int p = __shfl_xor_sync(0xffffffffu, v[i], m);
+            v[i] = p + sgn * v[i];
         }
     }
 }
@@ -121,13 +102,18 @@ __device__ __forceinline__ int requant(long long P, int n) {
 
 __device__ __forceinline__ int clamp127(int v) { return v < -127 ? -127 : (v > 127 ? 127 : v); }
 
-__device__ __forceinline__ uint32_t pack4(int a, int b, int c, int d) {
-    return (uint32_t)(a & 0xff) | ((uint32_t)(b & 0xff) << 8) | ((uint32_t)(c & 0xff) << 16) |
-           ((uint32_t)(d & 0xff) << 24);
+// requant for 32 <= n <= 62 with k = 2^(n-1) - 1 and s = n - 32: P + k + bit_n(P)
+// stays below 2^63 (|P| < 2^62) and its arithmetic shift by n is the high word
+// shifted by s.
+__device__ __forceinline__ int requant_hi(long long P, int s, long long k) {
+    const uint32_t bit = ((uint32_t)((unsigned long long)P >> 32) >> s) & 1u;
+    const long long u = P + k + (long long)bit;
+    return clamp127((int)(u >> 32) >> s);
+}
+__device__ __forceinline__ uint32_t pack4p(int a, int b, int c, int d) {
+    return __byte_perm(__byte_perm((uint32_t)a, (uint32_t)b, 0x0040), __byte_perm((uint32_t)c, (uint32_t)d, 0x0040), 0x5410);
 }
 
-__device__ __forceinline__ int lo16(uint32_t r) { return (int)(short)(r & 0xffffu); }
-__device__ __forceinline__ int hi16(uint32_t r) { return ((int)r) >> 16; }
 
 // MODE 0: static scale. MODE 1: scale from the dynamic parameter block.
 // MODE 2: max-abs pass of the dynamic mode (no store).
@@ -171,22 +157,27 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
         const long long e0 = (t << 9) + lane * 16;
         const bool valid = e0 < a.total;
         if (!F16) {
-            uint32_t r[8];
-            unpack_i8x16(cur0, r);
-            butterfly_i16(r, a.hb, lane);
+            int v[16];
+            unpack_i8x16_i32(cur0, v);
+            butterfly_i32(v, a.hb, lane);
             if (MODE == 2) {
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    const uint32_t m0 = (uint32_t)abs(lo16(r[k])), m1 = (uint32_t)abs(hi16(r[k]));
-                    local_max = max(local_max, max(m0, m1));
-                }
+                for (int k = 0; k < 16; ++k) local_max = max(local_max, (uint32_t)abs(v[k]));
             } else if (valid) {
                 uint32_t o[4];
+                const int m32 = (int)mult;            // M_q < 2^31
+                if (shift >= 32) {
+                    const int sh = shift - 32;
+                    const long long k = (1LL << (shift - 1)) - 1;
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const uint32_t r0 = r[2 * i], r1 = r[2 * i + 1];
-                    o[i] = pack4(requant(mult * lo16(r0), shift), requant(mult * hi16(r0), shift),
-                                 requant(mult * lo16(r1), shift), requant(mult * hi16(r1), shift));
+                    for (int i = 0; i < 4; ++i)
+                        o[i] = pack4p(requant_hi((long long)m32 * v[4 * i], sh, k), requant_hi((long long)m32 * v[4 * i + 1], sh, k),
+                                      requant_hi((long long)m32 * v[4 * i + 2], sh, k), requant_hi((long long)m32 * v[4 * i + 3], sh, k));
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        o[i] = pack4p(requant((long long)m32 * v[4 * i], shift), requant((long long)m32 * v[4 * i + 1], shift),
+                                      requant((long long)m32 * v[4 * i + 2], shift), requant((long long)m32 * v[4 * i + 3], shift));
                 }
                 *reinterpret_cast<int4 *>(a.y + e0) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
             }
@@ -205,11 +196,16 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
 #pragma unroll
                 for (int i = 0; i < 16; ++i) local_maxf = fmaxf(local_maxf, fabsf(f[i]));
             } else if (valid) {
+                // clamp(rint(f * inv)): clamping to [-127, 127] first and adding
+                // 1.5 * 2^23 rounds half to even into the low mantissa bits, whose
+                // low byte is the two's-complement code
+                uint32_t q[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    q[i] = __float_as_uint(fminf(fmaxf(f[i] * inv, -127.f), 127.f) + 12582912.f);
                 uint32_t o[4];
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    o[i] = pack4(clamp127(__float2int_rn(f[4 * i] * inv)), clamp127(__float2int_rn(f[4 * i + 1] * inv)),
-                                 clamp127(__float2int_rn(f[4 * i + 2] * inv)), clamp127(__float2int_rn(f[4 * i + 3] * inv)));
+                for (int i = 0; i < 4; ++i) o[i] = pack4p((int)q[4 * i], (int)q[4 * i + 1], (int)q[4 * i + 2], (int)q[4 * i + 3]);
                 *reinterpret_cast<int4 *>(a.y + e0) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
             }
         }
