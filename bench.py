@@ -41,8 +41,8 @@ CALIB = os.path.join(ROOT, "tests", "golden", "calibration.json")
 PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_BF16_TFLOPS = 1900.0
 FALLBACK_HBM_GBS = 6800.0
-CPU_SAMPLE_HW = (512, 768)        # bounded oracle sample: one 768x512 crop of image 0
-CPU_SAMPLE_LATENT = (32, 48)
+CPU_SAMPLE_HW = (1024, 1536)      # bounded oracle sample: one 1536x1024 crop of image 0 (~10-15 s)
+CPU_SAMPLE_LATENT = (64, 96)
 
 
 def parse():
@@ -184,6 +184,26 @@ def run_reference(args, cfg, scales):
     print(json.dumps(line), flush=True)
 
 
+def replica_seed(base_seed: int, rank: int) -> int:
+    """Input seed of one replica: every rank draws its own batch of images."""
+    return base_seed + 7919 * rank
+
+
+def job_step_time(local_ms: float, dist=None, device=None) -> float:
+    """Step time of the whole job: the maximum over ranks (all-reduce MAX)."""
+    if dist is None:
+        return local_ms
+    import torch
+    t = torch.tensor([float(local_ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(images_per_rank: int, world: int, step_ms: float) -> float:
+    """Whole-job images/s: the images all ranks processed over the slowest rank's step."""
+    return world * images_per_rank / (step_ms / 1000.0)
+
+
 def workload_name(cfg):
     if cfg.name == "cfg4":
         return ("cfg4: LIC analysis chain 3->192->192->192->320 (5x5 s2, WH,DH,DH,DH) + hyperprior "
@@ -294,7 +314,7 @@ def main():
         plan = C.plan_chain(ch)
         chain = Chain(ch.layers, params, scales[ch.name], plan, ch.out_f32, device=dev)
         kind = H.IN_F16 if ch.input_kind == "f16" else H.IN_I8
-        x_host = C.chain_input(ch.with_batch(ch.n, ch.h, ch.w, ch.input_seed + 7919 * rank))
+        x_host = C.chain_input(ch.with_batch(ch.n, ch.h, ch.w, replica_seed(ch.input_seed, rank)))
         x_pin = torch.from_numpy(x_host).pin_memory()
         x_dev = x_pin.to(dev)
         outs, scratch = chain.alloc(ch.n, ch.h, ch.w, dev)
@@ -349,11 +369,8 @@ def main():
         step(records)
     t1.record(stream)
     torch.cuda.synchronize()
-    ms = t0.elapsed_time(t1) / args.steps
+    ms = job_step_time(t0.elapsed_time(t1) / args.steps, dist, dev)
     if dist:
-        tt = torch.tensor([ms], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms = float(tt.item())
         dist.barrier()
     clocks = sampler.stop()
     H.sync_status()
@@ -381,15 +398,11 @@ def main():
             e2e_step()
         s1.record(stream)
         torch.cuda.synchronize()
-        e2e_ms = s0.elapsed_time(s1) / args.steps
-        if dist:
-            tt = torch.tensor([e2e_ms], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e2e_ms = float(tt.item())
+        e2e_ms = job_step_time(s0.elapsed_time(s1) / args.steps, dist, dev)
         H.sync_status()
         h2d = sum(c["x_pin"].numel() * c["x_pin"].element_size() for c in chains)
         d2h = sum(c["out_pin"].numel() * c["out_pin"].element_size() for c in chains)
-        e2e = {"value": world * images_step / (e2e_ms / 1000.0), "unit": "images/s", "h2d_bytes_per_step": h2d,
+        e2e = {"value": job_throughput(images_step, world, e2e_ms), "unit": "images/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
 
     if rank != 0:
@@ -423,7 +436,7 @@ def main():
         except Exception as ex:  # the oracle is a reported baseline only
             cpu = {"value": None, "unit": "images/s", "cores": None, "kind": "oracle", "sample": f"failed: {ex}"}
 
-    value = world * images_step / (ms / 1000.0)
+    value = job_throughput(images_step, world, ms)
     line = {
         "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
         "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",

@@ -229,6 +229,16 @@ const char *hatq_last_error(void);
  * so work enqueued after a failure produces no output until it is read. */
 hatq_status hatq_sync_status(hatq_stream stream);
 
+/* Failure-detection self test (the paper has no counterpart): launches one
+ * thread that waits, through the same bounded mbarrier wait the convolution
+ * pipeline uses, on a barrier nothing arrives at. The wait expires after
+ * limit_cycles SM clock cycles (1 .. 4e9) and records the timeout in the
+ * device error word, so the next hatq_sync_status() returns HATQ_ERR_TIMEOUT
+ * (and clears it); convolutions enqueued before that read are skipped, as after
+ * a real expiry. Stream-ordered; HATQ_ERR_INVALID_ARG for a limit out of range.
+ * Nothing faults or hangs: the device stays usable. */
+hatq_status hatq_selftest_wait(unsigned long long limit_cycles, hatq_stream stream);
+
 /* Library version, (major << 16) | minor. */
 int hatq_version(void);
 

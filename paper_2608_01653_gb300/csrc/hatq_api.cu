@@ -571,6 +571,15 @@ hatq_status hatq_layer(const void *x, int x_kind, float s_in, int n, int h, int 
     return hatq_conv2d_i8(static_cast<const int8_t *>(scratch), n, h, w, L, y, stream);
 }
 
+hatq_status hatq_selftest_wait(unsigned long long limit_cycles, hatq_stream stream) {
+    if (limit_cycles == 0 || limit_cycles > 4000000000ull) return fail(HATQ_ERR_INVALID_ARG, "limit must be in 1..4e9 cycles");
+    int *p = err_word();
+    if (!p) return fail(HATQ_ERR_CUDA, "no CUDA device");
+    cudaError_t e = hatq::launch_wait_selftest(p, (long long)limit_cycles, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "self-test launch");
+    return HATQ_OK;
+}
+
 hatq_status hatq_sync_status(hatq_stream stream) {
     cudaError_t e = cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "stream synchronization");

@@ -71,8 +71,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 }
 
 // Bounded wait. Returns false when the CTA aborts (this wait expired, or
-// another role raised the abort flag).
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag, int *err) {
+// another role raised the abort flag, or the device error word is set).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag, int *err,
+                                          long long limit = kWaitLimitCycles) {
     if (mbar_try_wait(bar, parity)) return true;
     const long long t0 = clock64();
     for (uint32_t spin = 1;; ++spin) {
@@ -80,7 +81,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
         if ((spin & 63) == 0) {
             if (*abort_flag) return false;
             if (*reinterpret_cast<volatile int *>(err) != 0) { *abort_flag = 1; return false; }
-            if (clock64() - t0 > kWaitLimitCycles) {
+            if (clock64() - t0 > limit) {
                 *abort_flag = 1;
                 atomicExch(err, kErrWaitTimeout);
                 return false;
@@ -88,6 +89,7 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
         }
     }
 }
+
 
 __device__ __forceinline__ void fence_barrier_init() {
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -909,7 +911,25 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+// Failure-detection self test: one thread waits, through the pipeline's
+// bounded wait, on an mbarrier nothing arrives at; the wait expires after
+// `limit` cycles and records kErrWaitTimeout in the error word.
+__global__ void wait_selftest_kernel(int *err, long long limit) {
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ int abort_flag;
+    if (threadIdx.x != 0) return;
+    abort_flag = 0;
+    mbar_init(smem_addr(&bar), 1);
+    fence_barrier_init();
+    (void)mbar_wait(smem_addr(&bar), 0, &abort_flag, err, limit);
+}
+
 }  // namespace
+
+cudaError_t launch_wait_selftest(int *err, long long limit_cycles, cudaStream_t s) {
+    wait_selftest_kernel<<<1, 32, 0, s>>>(err, limit_cycles);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const ConvArgs &a, int smem_bytes, cudaStream_t s) {
     // the shared-memory opt-in and the SM count are per device

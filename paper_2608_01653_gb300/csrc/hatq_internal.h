@@ -42,6 +42,7 @@ struct DynParams {
 };
 
 cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s);
+cudaError_t launch_wait_selftest(int *err, long long limit_cycles, cudaStream_t s);
 cudaError_t launch_act_dynamic(const ActQuantArgs &a, float s_in, float *s_used, cudaStream_t s);
 
 // ---------------------------------------------------------------- conv

@@ -71,6 +71,7 @@ def load(build: bool = True) -> ctypes.CDLL:
             "hatq_layer_launches": (_I, [_I, _F, ctypes.POINTER(PreparedStruct)]),
             "hatq_last_error": (ctypes.c_char_p, []),
             "hatq_sync_status": (_I, [_P]),
+            "hatq_selftest_wait": (_I, [ctypes.c_ulonglong, _P]),
             "hatq_version": (_I, []),
         }
         for name, (res, args) in sig.items():
@@ -272,6 +273,12 @@ def layer_launches(x_kind, s_in, L: PreparedLayer) -> int:
 
 def sync_status(stream=None):
     _check(load().hatq_sync_status(_stream(stream)))
+
+
+def selftest_wait(limit_cycles: int, stream=None):
+    """hatq_selftest_wait: make one bounded device wait expire on purpose
+    (failure-detection test; the next sync_status() raises ERR_TIMEOUT)."""
+    _check(load().hatq_selftest_wait(int(limit_cycles), _stream(stream)))
 
 
 def version() -> int:

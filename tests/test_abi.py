@@ -29,6 +29,13 @@ def test_exports_every_declared_function(lib):
         assert hasattr(lib, name), f"libhatq.so does not export {name}"
 
 
+def test_selftest_wait_checks_its_limit_on_the_host(lib):
+    # argument errors are returned before any launch, so this needs no GPU
+    assert lib.hatq_selftest_wait(0, None) == H.ERR_INVALID_ARG
+    assert lib.hatq_selftest_wait(4_000_000_001, None) == H.ERR_INVALID_ARG
+    assert "limit" in H.last_error()
+
+
 def test_version_and_last_error(lib):
     assert H.version() == 1
     d = H.make_desc(64, 48, 3, 1, 1, "DH", hb_in=64)          # c_out not a multiple of 32
