@@ -43,6 +43,8 @@ FALLBACK_BF16_TFLOPS = 1900.0
 FALLBACK_HBM_GBS = 6800.0
 CPU_SAMPLE_HW = (1024, 1536)      # bounded oracle sample: one 1536x1024 crop of image 0 (~10-15 s)
 CPU_SAMPLE_LATENT = (64, 96)
+REF_SAMPLE_HW = (512, 768)        # per step of --impl reference (~3 s), so K steps end within minutes
+REF_SAMPLE_LATENT = (32, 48)
 
 
 def parse():
@@ -130,7 +132,7 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ oracle (CPU baseline / reference arm)
 
-def oracle_sample(cfg, scales, threads=None):
+def oracle_sample(cfg, scales, threads=None, hw=CPU_SAMPLE_HW, latent=CPU_SAMPLE_LATENT):
     """Runs the oracle as it stands on a bounded crop of the same workload and
     returns (seconds, images-equivalent, algorithmic ops, threads)."""
     from oracle import hatq_oracle as O
@@ -140,9 +142,9 @@ def oracle_sample(cfg, scales, threads=None):
     t_total, frac_img, ops = 0.0, 0.0, 0
     for ch in cfg.chains:
         if ch.name == "analysis":
-            h, w = CPU_SAMPLE_HW if cfg.name == "cfg4" else (ch.h, ch.w)
+            h, w = hw if cfg.name == "cfg4" else (ch.h, ch.w)
         else:
-            h, w = CPU_SAMPLE_LATENT if cfg.name == "cfg4" else (ch.h, ch.w)
+            h, w = latent if cfg.name == "cfg4" else (ch.h, ch.w)
         sub = ch.with_batch(1, h, w, ch.input_seed)
         x = C.chain_input(sub)
         params = C.chain_params(ch)
@@ -162,17 +164,17 @@ def run_reference(args, cfg, scales):
     if rank != 0:
         return
     for _ in range(args.warmup if args.warmup < 1 else 1):
-        oracle_sample(cfg, scales)
+        oracle_sample(cfg, scales, hw=REF_SAMPLE_HW, latent=REF_SAMPLE_LATENT)
     times = []
     frac = ops = threads = None
     for _ in range(args.steps):
-        t, frac, ops, threads = oracle_sample(cfg, scales)
+        t, frac, ops, threads = oracle_sample(cfg, scales, hw=REF_SAMPLE_HW, latent=REF_SAMPLE_LATENT)
         times.append(t)
     t = sum(times) / len(times)
     value = frac / t
     sample = (f"oracle (numpy fp64/int64 + C direct conv, OpenMP {threads} threads) on one "
-              f"{CPU_SAMPLE_HW[1]}x{CPU_SAMPLE_HW[0]} crop of image 0 and the matching "
-              f"{CPU_SAMPLE_LATENT[1]}x{CPU_SAMPLE_LATENT[0]} latent crop for every chain, "
+              f"{REF_SAMPLE_HW[1]}x{REF_SAMPLE_HW[0]} crop of image 0 and the matching "
+              f"{REF_SAMPLE_LATENT[1]}x{REF_SAMPLE_LATENT[0]} latent crop for every chain, "
               f"scaled to full 3840x2160 images")
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * t, "higher_is_better": True,
