@@ -530,3 +530,40 @@ def sqnr_db(x, xhat) -> float:
 def range_expands(x, hb: int) -> bool:
     """Indicator of Eq. (hadamard_sensitivity) for one tensor."""
     return float(np.max(np.abs(transform_real(x, hb)))) > float(np.max(np.abs(x)))
+
+
+# --------------------------------------------------------------------------
+# Profiling-based strategy selection: Eqs. (hadamard_sensitivity,
+# layerwise_hadamard_selection), on the INT8 codes a layer receives
+# --------------------------------------------------------------------------
+
+
+def range_expansion_codes(x_i8, hb: int):
+    """Per image k of an NHWC code tensor, the indicator of Eq.
+    (hadamard_sensitivity), ||T x_k||_inf > ||x_k||_inf with the normalized
+    block transform T = I (x) H~_hb / sqrt(hb). With integer codes it is decided
+    exactly as max|H~_hb x_k|^2 > hb * max|x_k|^2 (Python integers).
+    Returns (max|x_k|, max|H~ x_k|, indicator) as int64, int64, uint8 arrays."""
+    x = np.asarray(x_i8, dtype=np.int64)
+    n = x.shape[0]
+    flat = x.reshape(n, -1, x.shape[-1])
+    y = transform_int(flat, hb)
+    mx = np.abs(flat).reshape(n, -1).max(axis=1) if flat.size else np.zeros(n, np.int64)
+    mh = np.abs(y).reshape(n, -1).max(axis=1) if y.size else np.zeros(n, np.int64)
+    ind = np.array([int(h) ** 2 > hb * int(m) ** 2 for h, m in zip(mh, mx)], dtype=np.uint8)
+    return mx.astype(np.int64), mh.astype(np.int64), ind
+
+
+def expansion_probability(indicators) -> Fraction:
+    """p_l of Eq. (hadamard_sensitivity): the fraction of the M profiled images
+    whose range expands, as an exact rational."""
+    ind = [int(v) for v in np.asarray(indicators).ravel()]
+    if not ind:
+        raise ValueError("no profiled images")
+    return Fraction(sum(ind), len(ind))
+
+
+def select_form(p, tau=Fraction(4, 5)) -> str:
+    """pi_l of Eq. (layerwise_hadamard_selection): WH when p_l > tau_sel, else
+    DH (the paper uses tau_sel = 0.8)."""
+    return "WH" if Fraction(p) > Fraction(tau) else "DH"

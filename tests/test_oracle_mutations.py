@@ -13,7 +13,7 @@ from oracle import hatq_oracle as O
 _orig = {k: getattr(O, k) for k in ("sylvester", "transform_real", "transform_int", "rshift_rne",
                                     "fixed_point", "prepare_layer", "epilogue_int", "conv_codes",
                                     "quantize_act_i8", "transform_weights", "quantize_sym",
-                                    "act_multiplier")}
+                                    "act_multiplier", "range_expansion_codes", "select_form")}
 
 
 def _sylvester_bad(m):
@@ -91,7 +91,26 @@ def _quantize_floor(x, s):
     return np.clip(np.floor(np.asarray(x, dtype=np.float64) / s), -127, 127).astype(np.int64)
 
 
+def _profile_non_strict(x_i8, hb):
+    mx, mh, _ = _orig["range_expansion_codes"](x_i8, hb)
+    return mx, mh, np.array([int(h) ** 2 >= hb * int(m) ** 2 for h, m in zip(mh, mx)], np.uint8)
+
+
+def _profile_unnormalized(x_i8, hb):
+    mx, mh, _ = _orig["range_expansion_codes"](x_i8, hb)
+    return mx, mh, np.array([int(h) > int(m) for h, m in zip(mh, mx)], np.uint8)
+
+
+def _select_non_strict(p, tau=None):
+    from fractions import Fraction
+    tau = Fraction(4, 5) if tau is None else Fraction(tau)
+    return "WH" if Fraction(p) >= tau else "DH"
+
+
 MUTATIONS = {
+    "profile_non_strict": ("range_expansion_codes", _profile_non_strict),
+    "profile_unnormalized": ("range_expansion_codes", _profile_unnormalized),
+    "select_non_strict": ("select_form", _select_non_strict),
     "sylvester_sign": ("sylvester", _sylvester_bad),
     "normalize_by_m": ("transform_real", _transform_real_bad),
     "int_transform_sign": ("transform_int", _transform_int_bad),

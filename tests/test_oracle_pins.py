@@ -396,3 +396,69 @@ def test_range_expansion_indicator():
     spiky = rng.standard_normal((64, 64)) * 0.1
     spiky[:, 3] = 50.0 * np.sign(rng.standard_normal(64))
     assert not O.range_expands(spiky, 64)
+
+
+# ------------------------------------------------------- profiling (Eqs. hadamard_sensitivity, layerwise selection)
+
+@pytest.mark.parametrize("hb", [2, 4, 16, 32, 64, 128])
+def test_profile_constant_image_expands_by_sqrt_hb(hb):
+    """Closed form: a constant code c (a nonzero channel mean) accumulates
+    coherently into the constant basis, |T x|_inf = sqrt(hb) |c| > |c|."""
+    x = np.full((1, 2, 3, 2 * hb), -5, np.int8)
+    mx, mh, ind = O.range_expansion_codes(x, hb)
+    assert mx[0] == 5 and mh[0] == 5 * hb and ind[0] == 1
+
+
+@pytest.mark.parametrize("hb", [2, 8, 64, 256])
+def test_profile_spike_shrinks_by_sqrt_hb(hb):
+    """Closed form: one nonzero code per block spreads evenly, |T x|_inf =
+    |c| / sqrt(hb) < |c|: no expansion."""
+    x = np.zeros((1, 1, 2, hb), np.int8)
+    x[0, 0, 0, 3 % hb] = 100
+    x[0, 0, 1, 0] = -100
+    mx, mh, ind = O.range_expansion_codes(x, hb)
+    assert mx[0] == 100 and mh[0] == 100 and ind[0] == 0
+
+
+def test_profile_ties_and_odd_orders_are_exact():
+    """Strict '>' of Eq. hadamard_sensitivity on exact ties, and an odd power
+    of two (sqrt(hb) irrational) decided without rounding."""
+    tie = np.array([1, 1, 0, 0], np.int8).reshape(1, 1, 1, 4)      # T x = (1, 0, 1, 0): equal range
+    assert O.range_expansion_codes(tie, 4)[2][0] == 0
+    assert not O.range_expands(tie.astype(np.float64), 4)
+    assert O.range_expansion_codes(np.array([1, 1], np.int8).reshape(1, 1, 1, 2), 2)[2][0] == 1   # sqrt2 > 1
+    assert O.range_expansion_codes(np.array([3, -1], np.int8).reshape(1, 1, 1, 2), 2)[2][0] == 0  # 4/sqrt2 < 3
+    assert O.range_expansion_codes(np.zeros((2, 1, 1, 16), np.int8), 16)[2].tolist() == [0, 0]
+
+
+def test_profile_matches_dense_transform_per_image():
+    """Brute force: the dense normalized transform in fp64 per image gives the
+    same indicator wherever the two ranges are not within rounding of a tie."""
+    rng = np.random.default_rng(7)
+    x = rng.integers(-127, 128, size=(12, 3, 4, 64)).astype(np.int8)
+    x[::3] = np.abs(x[::3])                      # nonnegative images: nonzero channel means
+    x[1::3] = rng.integers(-2, 3, size=x[1::3].shape)              # small codes with one outlier channel:
+    x[1::3, ..., 5] = 120                                          # the transform spreads the outlier
+    mx, mh, ind = O.range_expansion_codes(x, 32)
+    T = O.blockdiag_transform(64, 32)
+    for k in range(x.shape[0]):
+        xf = x[k].reshape(-1, 64).astype(np.float64)
+        ref_h = np.abs(xf @ T.T).max()
+        assert mx[k] == np.abs(xf).max()
+        assert abs(mh[k] / math.sqrt(32) - ref_h) < 1e-9
+        if abs(ref_h - mx[k]) > 1e-9:
+            assert ind[k] == int(ref_h > mx[k])
+    assert 0 < ind.sum() < len(ind)
+
+
+def test_expansion_probability_and_selection():
+    """p_l is the expanding fraction of the M images; pi_l = WH only when
+    p_l > tau_sel (strict), with the paper's tau_sel = 0.8."""
+    from fractions import Fraction
+    assert O.expansion_probability([1, 1, 1, 1, 0]) == Fraction(4, 5)
+    assert O.select_form(Fraction(4, 5)) == "DH"
+    assert O.select_form(O.expansion_probability([1] * 5)) == "WH"
+    assert O.select_form(Fraction(81, 100)) == "WH"
+    assert O.select_form(Fraction(1, 2), tau=Fraction(1, 4)) == "WH"
+    with pytest.raises(ValueError):
+        O.expansion_probability([])
