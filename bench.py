@@ -53,8 +53,9 @@ def parse():
     p.add_argument("--steps", type=int, default=10)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--workload", default="cfg4", choices=["cfg4", "cfg2", "cfg1", "fwht"],
-                   help="fwht: the INT8 transform+requantize pass alone on the config-4 ga2 input")
+    p.add_argument("--workload", default="cfg4", choices=["cfg4", "cfg2", "cfg1", "fwht", "profile"],
+                   help="fwht: the INT8 transform+requantize pass alone on the config-4 ga2 input; "
+                        "profile: the range-expansion profiling pass on the same tensor")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--layer", default="", help="time one layer of the config-4 chains (e.g. ga2, h1, s0a)")
@@ -280,6 +281,24 @@ def run_fwht_mode(args):
                       "frac": gbs / peak}), flush=True)
 
 
+def run_profile_mode(args):
+    """The range-expansion profiling pass (Eq. hadamard_sensitivity, hb 64) over
+    a batch shaped like the config-4 ga2 input: 1 byte read per element."""
+    import torch
+    from paper_2608_01653_gb300 import hatq as H
+    H.load()
+    shape = (args.batch, 1080, 1920, 192)
+    x = torch.from_numpy(I.uniform_codes(shape, seed=9)).cuda()
+    ms = time_events(lambda: H.profile_range(x, 64), args.steps, args.warmup)
+    H.sync_status()
+    nbytes = x.numel()
+    peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
+    peak = peaks.get("hbm_gbs", FALLBACK_HBM_GBS)
+    gbs = nbytes / (ms / 1000) / 1e9
+    print(json.dumps({"mode": "profile", "shape": list(shape), "hb": 64, "ms": ms, "GB/s": gbs,
+                      "peak_hbm_gbs": peak, "frac": gbs / peak}), flush=True)
+
+
 # ------------------------------------------------------------------ GPU arm
 
 def main():
@@ -287,7 +306,7 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht") else args.workload)
+    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile") else args.workload)
     if args.impl == "reference":
         run_reference(args, cfg, scales)
         return
@@ -296,6 +315,9 @@ def main():
         return
     if args.workload == "fwht":
         run_fwht_mode(args)
+        return
+    if args.workload == "profile":
+        run_profile_mode(args)
         return
 
     import torch

@@ -229,6 +229,21 @@ const char *hatq_last_error(void);
  * so work enqueued after a failure produces no output until it is read. */
 hatq_status hatq_sync_status(hatq_stream stream);
 
+/* Range-expansion profiling for the layer-wise DH/WH selection
+ * (Eq. hadamard_sensitivity, Sec. profiling-based strategy selection).
+ * x: device NHWC int8 codes [n][h][w][c], 16-byte aligned, c % 16 == 0;
+ *    hb: the layer's input block (power of two in 2..256 dividing c).
+ * maxima: device int32 [n][2], caller-owned, overwritten with max|x_k| and
+ *    max|H~_hb x_k| of every image k (H~ the unnormalized block transform).
+ * expands: device uint8 [n] or NULL: 1 where max|H~ x_k|^2 > hb max|x_k|^2,
+ *    i.e. ||T x_k||_inf > ||x_k||_inf for the normalized transform T (exact).
+ * p_l of Eq. hadamard_sensitivity is the mean of `expands` over the profiled
+ * images and Eq. layerwise_hadamard_selection assigns WH iff p_l > tau_sel.
+ * Stream-ordered; shape/alignment errors are returned before any launch;
+ * n == 0 is a no-op. */
+hatq_status hatq_profile_range(const int8_t *x, int n, int h, int w, int c, int hb, int32_t *maxima,
+                               uint8_t *expands, hatq_stream stream);
+
 /* Failure-detection self test (the paper has no counterpart): launches one
  * thread that waits, through the same bounded mbarrier wait the convolution
  * pipeline uses, on a barrier nothing arrives at. The wait expires after

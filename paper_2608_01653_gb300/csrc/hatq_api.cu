@@ -571,6 +571,28 @@ hatq_status hatq_layer(const void *x, int x_kind, float s_in, int n, int h, int 
     return hatq_conv2d_i8(static_cast<const int8_t *>(scratch), n, h, w, L, y, stream);
 }
 
+hatq_status hatq_profile_range(const int8_t *x, int n, int h, int w, int c, int hb, int32_t *maxima, uint8_t *expands,
+                               hatq_stream stream) {
+    if (n < 0 || h < 1 || w < 1 || c < 1) return fail(HATQ_ERR_INVALID_ARG, "bad shape");
+    if (!pow2(hb) || hb < 2 || hb > 256 || c % hb)
+        return fail(HATQ_ERR_INVALID_ARG, "hb must be a power of two in 2..256 dividing c");
+    if (c % 16) return fail(HATQ_ERR_UNSUPPORTED, "profiling needs c % 16 == 0");
+    if (n == 0) return HATQ_OK;
+    if (!x || !maxima) return fail(HATQ_ERR_INVALID_ARG, "null argument");
+    if (reinterpret_cast<uintptr_t>(x) % 16) return fail(HATQ_ERR_INVALID_ARG, "x must be 16-byte aligned");
+    const long long per = (long long)h * w * c;
+    if (per >= (1LL << 40)) return fail(HATQ_ERR_UNSUPPORTED, "image too large");
+    hatq::ProfileArgs a{};
+    a.x = x;
+    a.per_image = per;
+    a.n = n;
+    a.hb = hb;
+    a.maxima = maxima;
+    cudaError_t e = hatq::launch_profile(a, expands, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "profiling launch");
+    return HATQ_OK;
+}
+
 hatq_status hatq_selftest_wait(unsigned long long limit_cycles, hatq_stream stream) {
     if (limit_cycles == 0 || limit_cycles > 4000000000ull) return fail(HATQ_ERR_INVALID_ARG, "limit must be in 1..4e9 cycles");
     int *p = err_word();

@@ -41,6 +41,15 @@ struct DynParams {
     unsigned long long reserved;
 };
 
+// ---------------------------------------------------------------- profiling
+struct ProfileArgs {
+    const int8_t *x;       // NHWC codes, n images of per_image elements
+    long long per_image;   // h * w * c, a multiple of 16
+    int n, hb;
+    int *maxima;           // [n][2]: max|x|, max|H~_hb x|
+};
+cudaError_t launch_profile(const ProfileArgs &a, uint8_t *expands, cudaStream_t s);
+
 cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s);
 cudaError_t launch_wait_selftest(int *err, long long limit_cycles, cudaStream_t s);
 cudaError_t launch_act_dynamic(const ActQuantArgs &a, float s_in, float *s_used, cudaStream_t s);

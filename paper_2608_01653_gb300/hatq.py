@@ -72,6 +72,7 @@ def load(build: bool = True) -> ctypes.CDLL:
             "hatq_last_error": (ctypes.c_char_p, []),
             "hatq_sync_status": (_I, [_P]),
             "hatq_selftest_wait": (_I, [ctypes.c_ulonglong, _P]),
+            "hatq_profile_range": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P]),
             "hatq_version": (_I, []),
         }
         for name, (res, args) in sig.items():
@@ -273,6 +274,35 @@ def layer_launches(x_kind, s_in, L: PreparedLayer) -> int:
 
 def sync_status(stream=None):
     _check(load().hatq_sync_status(_stream(stream)))
+
+
+def profile_range(x, hb: int, stream=None):
+    """hatq_profile_range on an NHWC int8 code tensor: returns (maxima [n, 2]
+    int32: max|x_k|, max|H~ x_k| per image; expands [n] uint8)."""
+    import torch
+    if x.dtype != torch.int8 or x.dim() != 4 or not x.is_cuda:
+        raise ValueError("x must be a CUDA int8 NHWC tensor")
+    x = x.contiguous()
+    n, h, w, c = x.shape
+    maxima = torch.empty((n, 2), dtype=torch.int32, device=x.device)
+    expands = torch.empty((n,), dtype=torch.uint8, device=x.device)
+    _check(load().hatq_profile_range(_ptr(x), n, h, w, c, hb, _ptr(maxima), _ptr(expands), _stream(stream)))
+    return maxima, expands
+
+
+def expansion_probability(expands):
+    """p_l: the fraction of profiled images whose range expands (exact)."""
+    from fractions import Fraction
+    vals = [int(v) for v in (expands.tolist() if hasattr(expands, "tolist") else expands)]
+    if not vals:
+        raise ValueError("no profiled images")
+    return Fraction(sum(vals), len(vals))
+
+
+def select_form(p, tau=0.8) -> str:
+    """pi_l: WH when p_l > tau_sel, else DH."""
+    from fractions import Fraction
+    return "WH" if Fraction(p) > Fraction(str(tau)) else "DH"
 
 
 def selftest_wait(limit_cycles: int, stream=None):

@@ -36,6 +36,14 @@ def test_selftest_wait_checks_its_limit_on_the_host(lib):
     assert "limit" in H.last_error()
 
 
+def test_profile_range_checks_arguments_on_the_host(lib):
+    assert lib.hatq_profile_range(None, 0, 4, 4, 64, 64, None, None, None) == H.OK       # empty batch
+    assert lib.hatq_profile_range(None, 1, 4, 4, 64, 48, None, None, None) == H.ERR_INVALID_ARG
+    assert lib.hatq_profile_range(None, 1, 4, 4, 40, 8, None, None, None) == H.ERR_UNSUPPORTED
+    assert lib.hatq_profile_range(None, 1, 4, 4, 64, 64, None, None, None) == H.ERR_INVALID_ARG
+    assert "null" in H.last_error()
+
+
 def test_version_and_last_error(lib):
     assert H.version() == 1
     d = H.make_desc(64, 48, 3, 1, 1, "DH", hb_in=64)          # c_out not a multiple of 32
