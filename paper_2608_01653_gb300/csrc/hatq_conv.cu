@@ -612,7 +612,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                             tc_fence_after();
                         }
                     }
-                    if (!mbar_wait(full_bar(s), ph, abort_flag, a.err)) { ok = false; break; }
+                    // conv[s] completes only after every converter observed full[s] (the TMA
+                    // bytes of this stage), so waiting for it orders the weight reads as well
                     if (!mbar_wait(conv_bar(s), ph, abort_flag, a.err)) { ok = false; break; }
                     tc_fence_after();
                     const uint64_t db0 = desc0 + (uint64_t)((uint32_t)s * stage_step);
