@@ -208,12 +208,40 @@ class Prepared:
         self.__dict__.update(kw)
 
 
+GENERAL_ACTS = ("silu", "gelu")
+
+
+def phi(kind: str, v: float) -> float:
+    """The non-homogeneous activations of Sec. general nonlinearities, fp64
+    (math-library exp / erf): SiLU v / (1 + e^-v), GELU v (1 + erf(v / sqrt 2)) / 2."""
+    if kind == "silu":
+        return v / (1.0 + math.exp(-v))
+    if kind == "gelu":
+        return 0.5 * v * (1.0 + math.erf(v / math.sqrt(2.0)))
+    raise ValueError(kind)
+
+
+def activation_lut(kind: str, s_z: float, s_u: float) -> np.ndarray:
+    """phi_int of Eq. (supp_general_activation) as an integer lookup table over
+    the preactivation codes z = -127..127 (index z + 127):
+    u = clamp(round(phi(s_z z) / s_u), -127, 127), rounded half to even (R2)."""
+    s_z = float(np.float32(s_z))
+    s_u = float(np.float32(s_u))
+    out = np.zeros(255, dtype=np.int64)
+    for i, z in enumerate(range(-QMAX, QMAX + 1)):
+        out[i] = min(max(int(round(phi(kind, s_z * z) / s_u)), -QMAX), QMAX)
+    return out
+
+
 def prepare_layer(w_ohwi, b, form: str, hb_in: int, hb_out: int, s_x: float,
                   s_y: float, act: str, hb_next: int, out_f32: bool,
-                  stride: int, pad: int) -> Prepared:
+                  stride: int, pad: int, s_z: float = None, s_u: float = None) -> Prepared:
     """Offline preparation of one layer (Sec. deployment realization).
     s_x: scale of the INT8 operand this layer consumes; s_y: scale of the
-    INT8 operand the next layer consumes (or of this layer's output)."""
+    INT8 operand the next layer consumes (or of this layer's output).
+    A non-homogeneous act ('silu', 'gelu') takes the two-step transition of
+    Sec. general nonlinearities with preactivation scale s_z and activation
+    scale s_u."""
     s_x = float(np.float32(s_x))
     s_y = float(np.float32(s_y))
     wprime, bbar = transform_weights(w_ohwi, b, form, hb_in, hb_out)
@@ -234,6 +262,19 @@ def prepare_layer(w_ohwi, b, form: str, hb_in: int, hb_out: int, s_x: float,
                     s_x=s_x, s_y=s_y, s_w=s_w, b_int=b_int,
                     w_int=w_int.reshape(wprime.shape).astype(np.int8),
                     a_bound=a_bound, wprime=wprime, bbar=bbar)
+    if act in GENERAL_ACTS:
+        if out_f32:
+            raise ValueError("the general transition emits INT8 codes")
+        s_z = float(np.float32(s_z))
+        s_u = float(np.float32(s_u))
+        # Eq. supp_general_output_scale: s_A,c / (gamma_out s_z) ~ M_out / 2^n_out, M before H_out
+        prep.M, prep.n = fixed_point(s_a / (g_out * s_z), a_bound, hb_out if form == "WH" else 1)
+        prep.lut = activation_lut(act, s_z, s_u)
+        # Eq. supp_general_input_scale: s_u / (gamma_in,next s_x,next) ~ M_in / 2^n_in
+        M_in, n_in = fixed_point([s_u / (g_in * s_y)], [QMAX], hb_next if hb_next else 1)
+        prep.M_in, prep.n_in = int(M_in[0]), n_in
+        prep.s_z, prep.s_u = s_z, s_u
+        return prep
     if out_f32:
         prep.deq = s_a / g_out
         prep.M, prep.n = None, 0
@@ -392,6 +433,22 @@ def epilogue_int(acc, p: Prepared) -> np.ndarray:
     return np.clip(rshift_rne(w, p.n), -QMAX, QMAX).astype(np.int8)
 
 
+def epilogue_general(acc, p: Prepared) -> np.ndarray:
+    """Transition through a non-homogeneous activation (Sec. general
+    nonlinearities), in the order of Eqs. (supp_general_preactivation,
+    supp_general_activation, supp_general_input_transition):
+        z = clamp(round(H~_out (M_out (.) a) / 2^n_out)),  u = phi_int(z),
+        x_next = clamp(round(H~_in,next(M_in u) / 2^n_in))."""
+    a = np.asarray(acc, dtype=np.int64) + p.b_int
+    t = p.M * a
+    v = transform_int(t, p.hb_out) if p.hb_out else t
+    z = np.clip(rshift_rne(v, p.n), -QMAX, QMAX)
+    u = p.lut[z + QMAX]
+    w = p.M_in * u
+    w = transform_int(w, p.hb_next) if p.hb_next else w
+    return np.clip(rshift_rne(w, p.n_in), -QMAX, QMAX).astype(np.int8)
+
+
 def epilogue_f32(acc, p: Prepared) -> np.ndarray:
     """Dequantized output: y = H_out (s_A (.) a) (WH) or s_A (.) a (DH), then phi;
     with deq_c = s_x s_w,c / gamma_out the WH form is H~_out (deq (.) a)."""
@@ -404,6 +461,8 @@ def epilogue_f32(acc, p: Prepared) -> np.ndarray:
 def conv_layer(x_op, p: Prepared, window=None):
     """One prepared layer on its INT8 operand: conv + epilogue."""
     acc = conv_codes(x_op, p.w_int, p.stride, p.pad, window)
+    if p.act in GENERAL_ACTS:
+        return epilogue_general(acc, p)
     return epilogue_f32(acc, p) if p.out_f32 else epilogue_int(acc, p)
 
 

@@ -13,7 +13,8 @@ from oracle import hatq_oracle as O
 _orig = {k: getattr(O, k) for k in ("sylvester", "transform_real", "transform_int", "rshift_rne",
                                     "fixed_point", "prepare_layer", "epilogue_int", "conv_codes",
                                     "quantize_act_i8", "transform_weights", "quantize_sym",
-                                    "act_multiplier", "range_expansion_codes", "select_form")}
+                                    "act_multiplier", "range_expansion_codes", "select_form",
+                                    "epilogue_general", "phi")}
 
 
 def _sylvester_bad(m):
@@ -107,7 +108,30 @@ def _select_non_strict(p, tau=None):
     return "WH" if Fraction(p) >= tau else "DH"
 
 
+def _general_h_before_m(acc, p):
+    a = np.asarray(acc, dtype=np.int64) + p.b_int
+    v = O.transform_int(a, p.hb_out) if p.hb_out else a
+    t = p.M * v
+    z = np.clip(O.rshift_rne(t, p.n), -127, 127)
+    w = p.M_in * p.lut[z + 127]
+    w = O.transform_int(w, p.hb_next) if p.hb_next else w
+    return np.clip(O.rshift_rne(w, p.n_in), -127, 127).astype(np.int8)
+
+
+def _general_lut_shifted(acc, p):
+    q = O.Prepared(**p.__dict__)
+    q.lut = np.concatenate([p.lut[1:], p.lut[-1:]])
+    return _orig["epilogue_general"](acc, q)
+
+
+def _phi_sign(kind, v):
+    return v / (1.0 + math.exp(v)) if kind == "silu" else _orig["phi"](kind, -v)
+
+
 MUTATIONS = {
+    "general_M_after_H_out": ("epilogue_general", _general_h_before_m),
+    "general_lut_index_shift": ("epilogue_general", _general_lut_shifted),
+    "phi_sign": ("phi", _phi_sign),
     "profile_non_strict": ("range_expansion_codes", _profile_non_strict),
     "profile_unnormalized": ("range_expansion_codes", _profile_unnormalized),
     "select_non_strict": ("select_form", _select_non_strict),

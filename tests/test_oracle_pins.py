@@ -462,3 +462,76 @@ def test_expansion_probability_and_selection():
     assert O.select_form(Fraction(1, 2), tau=Fraction(1, 4)) == "WH"
     with pytest.raises(ValueError):
         O.expansion_probability([])
+
+
+# ------------------------------------------------------- general nonlinearities (Sec. general nonlinearities)
+
+@pytest.mark.parametrize("kind", ["silu", "gelu"])
+def test_activation_lut_closed_forms(kind):
+    """phi_int of Eq. supp_general_activation: phi(0) = 0, the printed values
+    SiLU(1) = 0.7310585786300049 and GELU(1) = 0.8413447460685429, and the
+    identity phi(v) - phi(-v) = v shared by SiLU and GELU (two roundings:
+    within one code wherever the table does not clamp)."""
+    s_z, s_u = 1.0 / 64, 1.0 / 100
+    lut = O.activation_lut(kind, s_z, s_u)
+    assert lut[127] == 0
+    assert lut[127 + 64] == {"silu": 73, "gelu": 84}[kind]
+    for z in range(1, 128):
+        up, dn = int(lut[127 + z]), int(lut[127 - z])
+        if abs(up) < 127 and abs(dn) < 127:
+            assert abs((up - dn) - s_z * z / s_u) <= 1.0
+    assert all(lut[127 + z] <= lut[127 + z + 1] for z in range(0, 126))   # increasing for v >= 0
+
+
+def _general_case(form, hb_next, kind, seed=0):
+    c_in, c_out = 64, 64
+    x_real = np.maximum(I.activations((1, 8, 9, c_in), seed=seed + 80).astype(np.float64), 0)
+    w = I.weights(c_out, 3, 3, c_in, seed=seed + 81)
+    b = I.bias(c_out, seed=seed + 82)
+    hb_in, hb_out = (64, 0) if form == "DH" else (0, 64)
+    y_lin = O.conv_real(x_real, w, b, 1, 1)
+    phi = np.vectorize(lambda v: O.phi(kind, v))
+    u_real = phi(y_lin)
+    s_x = O.symmetric_scale(O.transform_real(x_real, 64)) if form == "DH" else O.symmetric_scale(x_real)
+    s_z = O.symmetric_scale(y_lin)
+    s_u = O.symmetric_scale(u_real)
+    target = O.transform_real(u_real, hb_next) if hb_next else u_real
+    s_y = O.symmetric_scale(target)
+    p = O.prepare_layer(w, b, form, hb_in, hb_out, s_x, s_y, kind, hb_next, False, 1, 1, s_z=s_z, s_u=s_u)
+    op = O.quantize_act_f16(x_real.astype(np.float16), hb_in if form == "DH" else 1, s_x)
+    return p, op, target, y_lin
+
+
+@pytest.mark.parametrize("kind", ["silu", "gelu"])
+def test_general_transition_matches_its_equations_step_by_step(kind):
+    """With s_u = s_y and no next transform the input-side rescale is exactly
+    2^n_in / 2^n_in, so the output codes are phi_int(z); z is recomputed here
+    from exact rationals of H~_out (M_out (.) a) / 2^n_out and phi_int from
+    the activation formula itself (not the table)."""
+    p, op, _, _ = _general_case("WH", 0, kind)
+    p.M_in, p.n_in = O.fixed_point([1.0], [127], 1)
+    p.M_in = int(p.M_in[0])
+    assert p.M_in == 2 ** p.n_in
+    got = O.conv_layer(op, p).astype(np.int64)
+    acc = O.conv_codes(op, p.w_int, 1, 1) + p.b_int
+    H = O.sylvester(64)
+    for (i, j) in [(0, 0), (3, 5), (7, 8)]:
+        a = [int(v) for v in acc[0, i, j]]
+        t = [int(m) * v for m, v in zip(p.M, a)]
+        for c in (0, 17, 63):
+            v = sum(int(H[c, k]) * t[k] for k in range(64))
+            z = min(max(O.round_half_even_fraction(Fraction(v, 2 ** p.n)), -127), 127)
+            u = min(max(int(round(O.phi(kind, p.s_z * z) / p.s_u)), -127), 127)
+            assert got[0, i, j, c] == u
+
+
+@pytest.mark.parametrize("form,hb_next,kind", [("DH", 0, "silu"), ("WH", 0, "gelu"), ("DH", 64, "gelu"),
+                                               ("WH", 32, "silu")])
+def test_general_transition_tracks_real_model(form, hb_next, kind):
+    """End to end: the two-step integer transition (preactivation codes, table,
+    fixed-point rescale with the fused next transform) stays close to the
+    fp64 model phi(conv) (and its next-layer transform)."""
+    p, op, target, _ = _general_case(form, hb_next, kind, seed=3)
+    y = O.conv_layer(op, p).astype(np.float64) * p.s_y
+    assert O.sqnr_db(target, y) > (24.0 if form == "DH" else 18.0)
+    assert np.mean(np.abs(O.conv_layer(op, p)) == 127) < 0.1
