@@ -53,7 +53,12 @@ typedef enum {
 } hatq_status;
 
 typedef enum { HATQ_DH = 0, HATQ_WH = 1 } hatq_form;
-typedef enum { HATQ_ACT_NONE = 0, HATQ_ACT_RELU = 1 } hatq_act;
+/* Activation between layers. NONE and RELU are positively homogeneous and
+ * fold into the single requantization of Eq. integer_hadamard_transition;
+ * SILU and GELU are not and take the two-step transition of Sec. general
+ * nonlinearities (preactivation codes, integer table, input-side rescale),
+ * prepared with hatq_prepare_weights_general. */
+typedef enum { HATQ_ACT_NONE = 0, HATQ_ACT_RELU = 1, HATQ_ACT_SILU = 2, HATQ_ACT_GELU = 3 } hatq_act;
 
 /* What a layer input holds (hatq_layer, hatq_quantize_act). */
 typedef enum {
@@ -99,7 +104,39 @@ typedef struct {
     float *deq;           /* [c_out] s_x s_w,c / gamma_out (float32 output mode) */
     float *s_w;           /* [c_out] per-output-channel weight scales */
     uint64_t opaque[16];
+    /* general transition (act SILU / GELU), written by hatq_prepare_weights_general;
+     * then `mult` / `shift` hold M_out / n_out of Eq. supp_general_output_scale */
+    float s_z;            /* preactivation scale */
+    float s_u;            /* activation-output scale */
+    int shift_in;         /* n_in of Eq. supp_general_input_scale */
+    int reserved;
+    long long mult_in;    /* M_in of Eq. supp_general_input_scale */
+    int8_t lut[256];      /* phi_int of Eq. supp_general_activation at z = -127..127 (index z + 127) */
 } hatq_prepared;
+
+/*
+ * Offline preparation of a layer followed by a non-homogeneous activation
+ * (Sec. general nonlinearities). The same weights, bias codes and caller-set
+ * device buffers as hatq_prepare_weights, and:
+ *   z = clamp(round(H~_out (M_out (.) a) / 2^n_out))      (Eq. supp_general_preactivation)
+ *   u = lut[z + 127] = clamp(round(phi(s_z z) / s_u))       (Eq. supp_general_activation)
+ *   x = clamp(round(H~_in,next (M_in u) / 2^n_in))         (Eq. supp_general_input_transition)
+ * with s_A,c / (gamma_out s_z) ~ M_out / 2^n_out and s_u / (gamma_in,next s_y)
+ * ~ M_in / 2^n_in, both pairs by the (M, n) rule of hatq_prepare_weights.
+ * act: HATQ_ACT_SILU or HATQ_ACT_GELU (phi evaluated in fp64); s_z, s_u > 0;
+ * the output and next-layer blocks are at most 64; INT8 output only.
+ */
+hatq_status hatq_prepare_weights_general(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                         float s_z, float s_u, float s_y, int act, int hb_next, hatq_prepared *out,
+                                         hatq_stream stream);
+
+/* The host half of hatq_prepare_weights_general into host arrays (sizes as for
+ * hatq_prepare_weights_host; mult_in, shift_in and the 256-entry table out). */
+hatq_status hatq_prepare_weights_general_host(const hatq_conv_desc *d, const float *w_ohwi, const float *bias,
+                                              float s_x, float s_z, float s_u, float s_y, int act, int hb_next,
+                                              int8_t *w_i8_out, uint16_t *w_f16_out, int32_t *b_int_out,
+                                              int32_t *mult_out, float *s_w_out, int *shift_out,
+                                              long long *mult_in_out, int *shift_in_out, int8_t *lut_out);
 
 /*
  * Device buffer sizes of a prepared layer: w_elems = c_out * k_pad (elements

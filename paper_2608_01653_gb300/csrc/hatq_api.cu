@@ -200,7 +200,8 @@ hatq_status validate_prepare(const hatq_conv_desc *d, const float *w_ohwi, float
     if (!w_ohwi) return fail(HATQ_ERR_INVALID_ARG, "null weights");
     if (!(s_x > 0.f) || !std::isfinite(s_x)) return fail(HATQ_ERR_INVALID_ARG, "s_x must be positive");
     if (!out_f32 && (!(s_y > 0.f) || !std::isfinite(s_y))) return fail(HATQ_ERR_INVALID_ARG, "s_y must be positive");
-    if (act != HATQ_ACT_NONE && act != HATQ_ACT_RELU) return fail(HATQ_ERR_INVALID_ARG, "unknown activation");
+    if (act != HATQ_ACT_NONE && act != HATQ_ACT_RELU && act != HATQ_ACT_SILU && act != HATQ_ACT_GELU)
+        return fail(HATQ_ERR_INVALID_ARG, "unknown activation");
     if (hb_next != 0 && (!pow2(hb_next) || hb_next < 2 || hb_next > 128 || d->c_out % hb_next))
         return fail(HATQ_ERR_INVALID_ARG, "hb_next must be 0 or a power of two in 2..128 dividing c_out");
     if (out_f32 && hb_next) return fail(HATQ_ERR_INVALID_ARG, "a float32 output has no next-layer transform");
@@ -211,33 +212,45 @@ hatq_status validate_prepare(const hatq_conv_desc *d, const float *w_ohwi, float
     return geometry(d, hb_next, g);
 }
 
-}  // namespace
+bool general_act(int act) { return act == HATQ_ACT_SILU || act == HATQ_ACT_GELU; }
 
-hatq_status hatq::report(hatq_status st, const char *msg) { return fail(st, "%s", msg); }
+// phi of Sec. general nonlinearities in fp64: SiLU v / (1 + e^-v), GELU v (1 + erf(v / sqrt 2)) / 2.
+double phi(int act, double v) {
+    if (act == HATQ_ACT_SILU) return v / (1.0 + std::exp(-v));
+    return 0.5 * v * (1.0 + std::erf(v / std::sqrt(2.0)));
+}
 
-extern "C" {
+// The second half of a general transition: preactivation / activation scales
+// in, table and input-side fixed point out (Eqs. supp_general_activation,
+// supp_general_input_scale).
+struct GeneralParams {
+    float s_z = 0.f, s_u = 0.f;
+    long long mult_in = 0;
+    int shift_in = 0;
+    int8_t lut[256] = {};
+};
 
-int hatq_version(void) { return (0 << 16) | 1; }
-
-const char *hatq_last_error(void) { return g_msg.c_str(); }
-
-hatq_status hatq_prepared_sizes(const hatq_conv_desc *d, size_t *w_elems, size_t *ch_elems) {
-    hatq_status st = check_desc(d);
-    if (st != HATQ_OK) return st;
-    Geometry g;
-    if ((st = geometry(d, 0, &g)) != HATQ_OK) return st;
-    if (w_elems) *w_elems = (size_t)d->c_out * g.k_pad;
-    if (ch_elems) *ch_elems = (size_t)d->c_out;
+hatq_status validate_general(const hatq_conv_desc *d, int act, int hb_next, int out_f32, float s_z, float s_u) {
+    if (!general_act(act)) return fail(HATQ_ERR_INVALID_ARG, "the general transition takes HATQ_ACT_SILU or HATQ_ACT_GELU");
+    if (out_f32) return fail(HATQ_ERR_INVALID_ARG, "the general transition emits INT8 codes");
+    if (!(s_z > 0.f) || !std::isfinite(s_z) || !(s_u > 0.f) || !std::isfinite(s_u))
+        return fail(HATQ_ERR_INVALID_ARG, "s_z and s_u must be positive");
+    const int hb_out = d->form == HATQ_WH ? d->hb_out : 0;
+    if (hb_out > 64 || hb_next > 64)
+        return fail(HATQ_ERR_UNSUPPORTED, "the general transition supports output and next-layer blocks up to 64");
     return HATQ_OK;
 }
 
-hatq_status hatq_prepare_weights_host(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
-                                      float s_y, int act, int hb_next, int out_f32, int8_t *w_i8_out,
-                                      uint16_t *w_f16_out, int32_t *b_int_out, int32_t *mult_out, float *deq_out,
-                                      float *s_w_out, int *shift_out) {
+hatq_status prepare_core(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x, float s_y,
+                         int act, int hb_next, int out_f32, GeneralParams *gen, int8_t *w_i8_out,
+                         uint16_t *w_f16_out, int32_t *b_int_out, int32_t *mult_out, float *deq_out, float *s_w_out,
+                         int *shift_out) {
     Geometry g;
     hatq_status st = validate_prepare(d, w_ohwi, s_x, s_y, act, hb_next, out_f32, &g);
     if (st != HATQ_OK) return st;
+    if (general_act(act) != (gen != nullptr))
+        return fail(HATQ_ERR_INVALID_ARG, "SiLU / GELU layers are prepared with hatq_prepare_weights_general");
+    if (gen && (st = validate_general(d, act, hb_next, out_f32, gen->s_z, gen->s_u)) != HATQ_OK) return st;
     if (!w_i8_out || !w_f16_out || !b_int_out || !mult_out || !deq_out || !s_w_out || !shift_out)
         return fail(HATQ_ERR_INVALID_ARG, "null output buffer");
     const int co = d->c_out, ci = d->c_in, taps = d->kh * d->kw;
@@ -306,20 +319,92 @@ hatq_status hatq_prepare_weights_host(const hatq_conv_desc *d, const float *w_oh
         for (int o = 0; o < co; ++o) mult_out[o] = 0;
         return HATQ_OK;
     }
-    const double alpha = g_out * g_in;
-    for (int o = 0; o < co; ++o) rho[o] = s_a[o] / (alpha * sy);
-    const long long gain = (long long)(d->form == HATQ_WH ? d->hb_out : 1) * (hb_next ? hb_next : 1);
     std::vector<int32_t> mult;
     int shift = 0;
-    if ((st = fixed_point(rho, abound, gain, mult, shift)) != HATQ_OK) return st;
+    if (gen) {
+        // Eq. supp_general_output_scale: s_A,c / (gamma_out s_z), M_out applied before H_out
+        const double sz = (double)gen->s_z, su = (double)gen->s_u;
+        for (int o = 0; o < co; ++o) rho[o] = s_a[o] / (g_out * sz);
+        if ((st = fixed_point(rho, abound, d->form == HATQ_WH ? d->hb_out : 1, mult, shift)) != HATQ_OK) return st;
+        // Eq. supp_general_activation as a table over z = -127..127
+        for (int z = -127; z <= 127; ++z) {
+            double u = std::nearbyint(phi(act, sz * (double)z) / su);
+            u = u < -127.0 ? -127.0 : (u > 127.0 ? 127.0 : u);
+            gen->lut[z + 127] = (int8_t)u;
+        }
+        gen->lut[255] = 0;
+        // Eq. supp_general_input_scale: s_u / (gamma_in,next s_x,next)
+        std::vector<int32_t> m_in;
+        int n_in = 0;
+        if ((st = fixed_point({su / (g_in * sy)}, {127LL}, hb_next ? hb_next : 1, m_in, n_in)) != HATQ_OK) return st;
+        gen->mult_in = m_in[0];
+        gen->shift_in = n_in;
+    } else {
+        const double alpha = g_out * g_in;
+        for (int o = 0; o < co; ++o) rho[o] = s_a[o] / (alpha * sy);
+        const long long gain = (long long)(d->form == HATQ_WH ? d->hb_out : 1) * (hb_next ? hb_next : 1);
+        if ((st = fixed_point(rho, abound, gain, mult, shift)) != HATQ_OK) return st;
+    }
     for (int o = 0; o < co; ++o) mult_out[o] = mult[o];
     *shift_out = shift;
     return HATQ_OK;
 }
 
-hatq_status hatq_prepare_weights(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
-                                 float s_y, int act, int hb_next, int out_f32, hatq_prepared *out,
-                                 hatq_stream stream) {
+}  // namespace
+
+hatq_status hatq::report(hatq_status st, const char *msg) { return fail(st, "%s", msg); }
+
+extern "C" {
+
+int hatq_version(void) { return (0 << 16) | 1; }
+
+const char *hatq_last_error(void) { return g_msg.c_str(); }
+
+hatq_status hatq_prepared_sizes(const hatq_conv_desc *d, size_t *w_elems, size_t *ch_elems) {
+    hatq_status st = check_desc(d);
+    if (st != HATQ_OK) return st;
+    Geometry g;
+    if ((st = geometry(d, 0, &g)) != HATQ_OK) return st;
+    if (w_elems) *w_elems = (size_t)d->c_out * g.k_pad;
+    if (ch_elems) *ch_elems = (size_t)d->c_out;
+    return HATQ_OK;
+}
+
+hatq_status hatq_prepare_weights_host(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                      float s_y, int act, int hb_next, int out_f32, int8_t *w_i8_out,
+                                      uint16_t *w_f16_out, int32_t *b_int_out, int32_t *mult_out, float *deq_out,
+                                      float *s_w_out, int *shift_out) {
+    return prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, nullptr, w_i8_out, w_f16_out, b_int_out,
+                        mult_out, deq_out, s_w_out, shift_out);
+}
+
+hatq_status hatq_prepare_weights_general_host(const hatq_conv_desc *d, const float *w_ohwi, const float *bias,
+                                              float s_x, float s_z, float s_u, float s_y, int act, int hb_next,
+                                              int8_t *w_i8_out, uint16_t *w_f16_out, int32_t *b_int_out,
+                                              int32_t *mult_out, float *s_w_out, int *shift_out,
+                                              long long *mult_in_out, int *shift_in_out, int8_t *lut_out) {
+    if (!mult_in_out || !shift_in_out || !lut_out) return fail(HATQ_ERR_INVALID_ARG, "null output buffer");
+    const int co = d ? d->c_out : 0;
+    std::vector<float> deq(co > 0 ? co : 1);
+    GeneralParams gen;
+    gen.s_z = s_z;
+    gen.s_u = s_u;
+    hatq_status st = prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, 0, &gen, w_i8_out, w_f16_out, b_int_out,
+                                  mult_out, deq.data(), s_w_out, shift_out);
+    if (st != HATQ_OK) return st;
+    *mult_in_out = gen.mult_in;
+    *shift_in_out = gen.shift_in;
+    std::memcpy(lut_out, gen.lut, 256);
+    return HATQ_OK;
+}
+
+}  // extern "C"
+
+namespace {
+
+hatq_status prepare_device(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x, float s_y,
+                           int act, int hb_next, int out_f32, GeneralParams *gen, hatq_prepared *out,
+                           hatq_stream stream) {
     Geometry g;
     hatq_status st = validate_prepare(d, w_ohwi, s_x, s_y, act, hb_next, out_f32, &g);
     if (st != HATQ_OK) return st;
@@ -335,8 +420,8 @@ hatq_status hatq_prepare_weights(const hatq_conv_desc *d, const float *w_ohwi, c
     std::vector<int32_t> b_int(co), mult(co);
     std::vector<float> deq(co), s_w(co);
     int shift = 0;
-    st = hatq_prepare_weights_host(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, w_i8.data(), w_f16.data(),
-                                   b_int.data(), mult.data(), deq.data(), s_w.data(), &shift);
+    st = prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, gen, w_i8.data(), w_f16.data(), b_int.data(),
+                      mult.data(), deq.data(), s_w.data(), &shift);
     if (st != HATQ_OK) return st;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     cudaError_t e;
@@ -372,7 +457,33 @@ hatq_status hatq_prepare_weights(const hatq_conv_desc *d, const float *w_ohwi, c
     out->gather = g.gather;
     out->s_x = s_x;
     out->s_y = out_f32 ? 0.f : s_y;
+    out->s_z = gen ? gen->s_z : 0.f;
+    out->s_u = gen ? gen->s_u : 0.f;
+    out->shift_in = gen ? gen->shift_in : 0;
+    out->reserved = 0;
+    out->mult_in = gen ? gen->mult_in : 0;
+    if (gen) std::memcpy(out->lut, gen->lut, sizeof out->lut);
+    else std::memset(out->lut, 0, sizeof out->lut);
     return HATQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+hatq_status hatq_prepare_weights(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                 float s_y, int act, int hb_next, int out_f32, hatq_prepared *out,
+                                 hatq_stream stream) {
+    return prepare_device(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, nullptr, out, stream);
+}
+
+hatq_status hatq_prepare_weights_general(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                         float s_z, float s_u, float s_y, int act, int hb_next, hatq_prepared *out,
+                                         hatq_stream stream) {
+    GeneralParams gen;
+    gen.s_z = s_z;
+    gen.s_u = s_u;
+    return prepare_device(d, w_ohwi, bias, s_x, s_y, act, hb_next, 0, &gen, out, stream);
 }
 
 hatq_status hatq_quantize_act(const void *x, int x_kind, float s_in, int n, int h, int w, int c, int hb, float s_out,
@@ -482,7 +593,8 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     // + 16 bytes: the gather reads up to 11 bytes past a row segment
     const int win_bytes = g.gather ? (a.win_h * a.win_pitch + 16 + 127) & ~127 : 0;
     const int table_bytes = g.gather ? a.num_kb * 8 * 4 : 0;
-    const int const_bytes = (3 * d->c_out * 4 + 127) & ~127;
+    const bool general = L->act == HATQ_ACT_SILU || L->act == HATQ_ACT_GELU;
+    const int const_bytes = ((3 * d->c_out * 4 + 127) & ~127) + (general ? 256 : 0);
     const int fixed = 1024 /* align */ + 8 * (3 * 8 + 9) + 16 + 128 + table_bytes + const_bytes + win_bytes;
     const int budget = 227 * 1024 - 1024 /* static */ - fixed - a.staging_bytes;
     // a stage holds `sub` 64-wide reduction blocks: [weights x sub | INT8 box x sub].
@@ -517,7 +629,12 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     a.shift = L->shift;
     a.hb_out = d->form == HATQ_WH ? d->hb_out : 0;
     a.hb_next = L->hb_next;
-    a.act = L->act;
+    a.act = L->act == HATQ_ACT_RELU ? 1 : 0;
+    a.general = general ? 1 : 0;
+    a.shift_in = L->shift_in;
+    a.mult_in = L->mult_in;
+    a.lut_off = a.const_off + ((3 * d->c_out * 4 + 127) & ~127);
+    std::memcpy(a.lut, L->lut, sizeof a.lut);
     a.out_f32 = L->out_f32;
     a.y = y;
     a.err = err_word();

@@ -213,6 +213,11 @@ __device__ __forceinline__ int requant8_hi(long long v, int s, unsigned long lon
     const int q = (int)(u >> 32) >> s;
     return min(max(q, -127), 127);
 }
+// requant8 with the 32-bit-piece path for shifts >= 32 (n is uniform).
+__device__ __forceinline__ int requant8_any(long long v, int n) {
+    return n >= 32 ? requant8_hi(v, n - 32, (1ull << (n - 1)) - 1) : requant8(v, n);
+}
+
 // Low bytes of four codes in [-127, 127] packed into one word.
 __device__ __forceinline__ uint32_t pack4(int q0, int q1, int q2, int q3) {
     return __byte_perm(__byte_perm((uint32_t)q0, (uint32_t)q1, 0x0040), __byte_perm((uint32_t)q2, (uint32_t)q3, 0x0040),
@@ -255,6 +260,7 @@ struct EpiCtx {
     bool int_acc;        // the accumulator holds exact int32 totals (else exact fp32 integers)
     uint8_t *row;        // this thread's row of the shared-memory output tile (INT8 output)
     float *gout;         // float32 output: this thread's pixel row in global memory, or null
+    const int8_t *lut;   // general transition: phi_int table (shared memory), index z + 127
 };
 
 // Exact int32 accumulator of 16 columns starting at tile column `col`, bias included.
@@ -333,6 +339,21 @@ __device__ __forceinline__ void store_codes(const ConvArgs &a, uint8_t *row, int
         reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
     }
 }
+// Codes already in [-127, 127], written to this thread's row of the output tile.
+template <int G>
+__device__ __forceinline__ void store_codes_i32(uint8_t *row, int col, const int (&x)[G]) {
+#pragma unroll
+    for (int i = 0; i < G / 16; ++i) {
+        uint32_t w[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int b = 16 * i + 4 * j;
+            w[j] = pack4(x[b], x[b + 1], x[b + 2], x[b + 3]);
+        }
+        reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
+    }
+}
+
 // Float32 output goes straight to global memory (no shared-memory staging).
 template <int G>
 __device__ __forceinline__ void store_f32(float *gout, int col, const float (&t)[G]) {
@@ -348,6 +369,28 @@ __device__ __forceinline__ float relu(float v) { return fmaxf(v, 0.f); }
 // One group of G <= 64 columns held entirely in registers.
 template <int G>
 __device__ __forceinline__ void epi_group(const EpiCtx &e, const ConvArgs &a, int col) {
+    if (a.general) {
+        // Sec. general nonlinearities: z = clamp(round(H~_out (M_out (.) a) / 2^n_out)),
+        // u = phi_int(z), x = clamp(round(H~_next (M_in u) / 2^n_in)); |H~_next u| <= 127 * 64
+        // fits int32 and M_in is one scalar, so the next transform runs on u itself
+        long long t[G];
+#pragma unroll
+        for (int q = 0; q < G / 16; ++q) {
+            int v[16];
+            load_acc16(e, col + 16 * q, v);
+            scale_i64(e, col + 16 * q, v, t + 16 * q);
+        }
+        if (a.hb_out) fwht<G>(t, a.hb_out);
+        int u[G];
+#pragma unroll
+        for (int i = 0; i < G; ++i) u[i] = (int)e.lut[requant8_any(t[i], a.shift) + 127];
+        if (a.hb_next) fwht<G>(u, a.hb_next);
+        int x[G];
+#pragma unroll
+        for (int i = 0; i < G; ++i) x[i] = requant8_any(a.mult_in * (long long)u[i], a.shift_in);
+        store_codes_i32<G>(e.row, col, x);
+        return;
+    }
     if (!a.out_f32) {
         long long t[G];
 #pragma unroll
@@ -450,7 +493,8 @@ __device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a,
 // SUB: 64-wide reduction blocks per pipeline stage (1, 2 or 4)
 template <int SUB>
 __global__ void __launch_bounds__(kThreads, 1)
-    conv_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB, const ConvArgs a) {
+    conv_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                const __grid_constant__ ConvArgs a) {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int S = a.stages;
@@ -515,6 +559,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         cb[a.co + c] = a.mult[c];
         reinterpret_cast<float *>(cb)[2 * a.co + c] = a.deq[c];
     }
+    int8_t *lut_s = reinterpret_cast<int8_t *>(bar_area + a.lut_off);
+    if (a.general)
+        for (int i = threadIdx.x; i < 256; i += kThreads) lut_s[i] = a.lut[i];
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -866,6 +913,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 e.deq = reinterpret_cast<const float *>(cb + 2 * a.co) + n0;
                 e.t_acc = t_acc;
                 e.int_acc = nbuf == 1;
+                e.lut = lut_s;
                 e.row = stage_tile + (size_t)row * a.row_stride;
                 e.gout = nullptr;
                 if (a.out_f32) {

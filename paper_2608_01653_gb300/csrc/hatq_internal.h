@@ -82,9 +82,15 @@ struct ConvArgs {
     const int32_t *b_int;
     const int32_t *mult;
     const float *deq;
-    int shift, hb_out, hb_next, act, out_f32;
+    int shift, hb_out, hb_next, act, out_f32;   // act: 1 = ReLU folded into the single requantization
     void *y;
     int *err;
+    // general transition (Sec. general nonlinearities): shift = n_out, mult = M_out,
+    // then the table and the input-side pair (mult_in, shift_in)
+    int general, shift_in;
+    int lut_off;                     // offset of the table copy from the barrier area
+    long long mult_in;
+    int8_t lut[256];
 };
 
 cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const ConvArgs &a,

@@ -17,10 +17,11 @@ from . import build as _build
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_OVERFLOW, ERR_CUDA, ERR_TIMEOUT = range(6)
 DH, WH = 0, 1
-ACT_NONE, ACT_RELU = 0, 1
+ACT_NONE, ACT_RELU, ACT_SILU, ACT_GELU = 0, 1, 2, 3
 IN_OPERAND, IN_I8, IN_F16 = 0, 1, 2
 
-_ACTS = {"none": ACT_NONE, "relu": ACT_RELU}
+_ACTS = {"none": ACT_NONE, "relu": ACT_RELU, "silu": ACT_SILU, "gelu": ACT_GELU}
+GENERAL_ACTS = ("silu", "gelu")
 _FORMS = {"DH": DH, "WH": WH}
 
 
@@ -42,7 +43,9 @@ class PreparedStruct(ctypes.Structure):
                 ("s_x", ctypes.c_float), ("s_y", ctypes.c_float),
                 ("w_i8", ctypes.c_void_p), ("w_f16", ctypes.c_void_p), ("b_int", ctypes.c_void_p),
                 ("mult", ctypes.c_void_p), ("deq", ctypes.c_void_p), ("s_w", ctypes.c_void_p),
-                ("opaque", ctypes.c_uint64 * 16)]
+                ("opaque", ctypes.c_uint64 * 16),
+                ("s_z", ctypes.c_float), ("s_u", ctypes.c_float), ("shift_in", ctypes.c_int),
+                ("reserved", ctypes.c_int), ("mult_in", ctypes.c_longlong), ("lut", ctypes.c_int8 * 256)]
 
 
 _LIB = None
@@ -62,6 +65,11 @@ def load(build: bool = True) -> ctypes.CDLL:
                                          ctypes.POINTER(ctypes.c_size_t)]),
             "hatq_prepare_weights": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _I, _I, _I,
                                           ctypes.POINTER(PreparedStruct), _P]),
+            "hatq_prepare_weights_general": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _F, _F, _I, _I,
+                                                  ctypes.POINTER(PreparedStruct), _P]),
+            "hatq_prepare_weights_general_host": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _F, _F, _I, _I,
+                                                       _P, _P, _P, _P, _P, ctypes.POINTER(_I),
+                                                       ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(_I), _P]),
             "hatq_prepare_weights_host": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _I, _I, _I,
                                                _P, _P, _P, _P, _P, _P, ctypes.POINTER(_I)]),
             "hatq_quantize_act": (_I, [_P, _I, _F, _I, _I, _I, _I, _I, _F, _P, _P, _P, _P]),
@@ -212,15 +220,54 @@ class PreparedLayer:
 
 
 def prepare_weights(desc: ConvDesc, w_ohwi, bias, s_x, s_y, act="none", hb_next=0, out_f32=False,
-                    stream=None, device="cuda") -> PreparedLayer:
-    """hatq_prepare_weights: offline transform, quantize and pack into device buffers."""
+                    stream=None, device="cuda", s_z=None, s_u=None) -> PreparedLayer:
+    """hatq_prepare_weights (or, for act 'silu' / 'gelu', hatq_prepare_weights_general
+    with preactivation scale s_z and activation scale s_u): offline transform,
+    quantize and pack into device buffers."""
     L = PreparedLayer(desc, device)
     w = np.ascontiguousarray(w_ohwi, dtype=np.float32)
     b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
-    _check(load().hatq_prepare_weights(ctypes.byref(desc), w.ctypes.data, None if b is None else b.ctypes.data,
-                                       float(s_x), float(s_y), _ACTS.get(act, act), int(hb_next),
-                                       int(bool(out_f32)), ctypes.byref(L.struct), _stream(stream)))
+    bp = None if b is None else b.ctypes.data
+    if act in GENERAL_ACTS:
+        if out_f32 or s_z is None or s_u is None:
+            raise ValueError("a SiLU / GELU layer emits INT8 codes and needs s_z and s_u")
+        _check(load().hatq_prepare_weights_general(ctypes.byref(desc), w.ctypes.data, bp, float(s_x), float(s_z),
+                                                   float(s_u), float(s_y), _ACTS[act], int(hb_next),
+                                                   ctypes.byref(L.struct), _stream(stream)))
+        return L
+    _check(load().hatq_prepare_weights(ctypes.byref(desc), w.ctypes.data, bp, float(s_x), float(s_y),
+                                       _ACTS.get(act, act), int(hb_next), int(bool(out_f32)),
+                                       ctypes.byref(L.struct), _stream(stream)))
     return L
+
+
+@dataclass
+class HostGeneral:
+    w_i8: np.ndarray
+    b_int: np.ndarray
+    mult: np.ndarray
+    s_w: np.ndarray
+    shift: int
+    mult_in: int
+    shift_in: int
+    lut: np.ndarray
+
+
+def prepare_weights_general_host(desc: ConvDesc, w_ohwi, bias, s_x, s_z, s_u, s_y, act, hb_next=0) -> HostGeneral:
+    """hatq_prepare_weights_general_host: the host half of a SiLU / GELU layer's preparation."""
+    w_elems, ch = prepared_sizes(desc)
+    w = np.ascontiguousarray(w_ohwi, dtype=np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    w_i8, w_f16 = np.zeros(w_elems, np.int8), np.zeros(w_elems, np.uint16)
+    b_int, mult, s_w = np.zeros(ch, np.int32), np.zeros(ch, np.int32), np.zeros(ch, np.float32)
+    lut = np.zeros(256, np.int8)
+    shift, shift_in, mult_in = ctypes.c_int(), ctypes.c_int(), ctypes.c_longlong()
+    _check(load().hatq_prepare_weights_general_host(
+        ctypes.byref(desc), w.ctypes.data, None if b is None else b.ctypes.data, float(s_x), float(s_z), float(s_u),
+        float(s_y), _ACTS[act], int(hb_next), w_i8.ctypes.data, w_f16.ctypes.data, b_int.ctypes.data,
+        mult.ctypes.data, s_w.ctypes.data, ctypes.byref(shift), ctypes.byref(mult_in), ctypes.byref(shift_in),
+        lut.ctypes.data))
+    return HostGeneral(w_i8.reshape(desc.c_out, -1), b_int, mult, s_w, shift.value, mult_in.value, shift_in.value, lut)
 
 
 def quantize_act(x, x_kind, s_in, hb, s_out, y=None, s_used=None, workspace=None, stream=None):

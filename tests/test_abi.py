@@ -12,6 +12,7 @@ import pytest
 from oracle import hatq_oracle as O
 from paper_2608_01653_gb300 import hatq as H
 from synth import configs as C
+from synth import inputs as I
 
 GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
 
@@ -148,3 +149,53 @@ def test_host_prepare_zero_weights_and_no_bias():
     w = np.zeros((64, 1, 1, 64), np.float32)
     got = H.prepare_weights_host(d, w, None, 0.1, 0.1)
     assert not got.w_i8.any() and np.all(got.s_w == 1.0) and not got.b_int.any()
+
+
+def _general_scales(L, w, b, kind, hb_next, seed):
+    x_real = np.maximum(I.activations((1, 6, 7, L.c_in), seed=seed).astype(np.float64), 0)
+    y = O.conv_real(x_real, w, b, L.stride, L.pad)
+    u = np.vectorize(lambda v: O.phi(kind, v))(y)
+    s_x = O.symmetric_scale(O.transform_real(x_real, L.hb_in)) if L.form == "DH" else O.symmetric_scale(x_real)
+    tgt = O.transform_real(u, hb_next) if hb_next else u
+    return (float(np.float32(s_x)), float(np.float32(O.symmetric_scale(y))), float(np.float32(O.symmetric_scale(u))),
+            float(np.float32(O.symmetric_scale(tgt))))
+
+
+GENERAL_CASES = [
+    ("dh3x3_silu", C.layer("a", 64, 64, 3, 1, 1, "DH", "silu", hb_in=64), 0),
+    ("wh3x3_gelu_next64", C.layer("a", 64, 128, 3, 1, 1, "WH", "gelu", hb_out=64), 64),
+    ("dh5x5s2_gelu_next32", C.layer("a", 192, 192, 5, 2, 2, "DH", "gelu", hb_in=64), 32),
+    ("wh5x5s2_c3_silu", C.layer("a", 3, 64, 5, 2, 2, "WH", "silu", hb_out=32), 64),
+]
+
+
+@pytest.mark.parametrize("case", GENERAL_CASES, ids=lambda c: c[0])
+def test_general_host_prepare_matches_oracle_bit_exact(case):
+    name, L, hb_next = case
+    w = I.weights(L.c_out, L.k, L.k, L.c_in, seed=31)
+    b = I.bias(L.c_out, seed=32)
+    s_x, s_z, s_u, s_y = _general_scales(L, w, b, L.act, hb_next, 33)
+    got = H.prepare_weights_general_host(H.desc_from_spec(L), w, b, s_x, s_z, s_u, s_y, L.act, hb_next)
+    ref = O.prepare_layer(w, b, L.form, L.hb_in, L.hb_out, s_x, s_y, L.act, hb_next, False, L.stride, L.pad,
+                          s_z=s_z, s_u=s_u)
+    assert np.array_equal(got.w_i8, _oracle_packed(ref, H.desc_from_spec(L), got.w_i8.shape[1]))
+    assert np.array_equal(got.b_int, ref.b_int)
+    assert np.array_equal(got.mult.astype(np.int64), ref.M) and got.shift == ref.n
+    assert got.mult_in == ref.M_in and got.shift_in == ref.n_in
+    assert np.array_equal(got.lut[:255].astype(np.int64), ref.lut)
+
+
+def test_general_prepare_rejects_what_it_does_not_cover(lib):
+    d = H.make_desc(64, 128, 3, 1, 1, "WH", hb_out=128)
+    w = np.zeros((128, 3, 3, 64), np.float32)
+    with pytest.raises(H.HatqError) as e:                       # 128-wide output block
+        H.prepare_weights_general_host(d, w, None, 0.1, 0.1, 0.1, 0.1, "silu", 0)
+    assert e.value.status == H.ERR_UNSUPPORTED
+    d = H.make_desc(64, 64, 3, 1, 1, "DH", hb_in=64)
+    w = np.zeros((64, 3, 3, 64), np.float32)
+    with pytest.raises(H.HatqError) as e:                       # nonpositive activation scale
+        H.prepare_weights_general_host(d, w, None, 0.1, 0.0, 0.1, 0.1, "gelu", 0)
+    assert e.value.status == H.ERR_INVALID_ARG
+    with pytest.raises(H.HatqError) as e:                       # SiLU through the homogeneous entry point
+        H.prepare_weights_host(d, w, None, 0.1, 0.1, "silu", 0)
+    assert e.value.status == H.ERR_INVALID_ARG
