@@ -60,6 +60,8 @@ def parse():
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--layer", default="", help="time one layer of the config-4 chains (e.g. ga2, h1, s0a)")
     p.add_argument("--batch", type=int, default=8, help="batch for --layer / the FWHT pass")
+    p.add_argument("--act", default=None, choices=["none", "relu", "silu", "gelu"],
+                   help="--layer: time the layer with this activation instead of its own")
     return p.parse_args()
 
 
@@ -244,8 +246,18 @@ def run_layer_mode(args, cfg, scales):
                 params = C.chain_params(ch)[i]
                 hb_next = C.plan_chain(ch)[i]
                 sc = scales[ch.name][i]
-                P = H.prepare_weights(H.desc_from_spec(L), params[0], params[1], sc["s_x"], sc["s_out"], L.act,
-                                      hb_next, False)
+                act = args.act or L.act
+                if act in H.GENERAL_ACTS:
+                    # same layer through the general transition; the calibrated output scale
+                    # stands in for s_z and s_u (timing only: the table's values do not
+                    # change the work)
+                    if max(L.hb_out if L.form == "WH" else 0, hb_next) > 64:
+                        raise SystemExit(f"layer {L.name}: the general transition covers blocks up to 64")
+                    P = H.prepare_weights(H.desc_from_spec(L), params[0], params[1], sc["s_x"], sc["s_out"], act,
+                                          hb_next, s_z=sc["s_out"], s_u=sc["s_out"])
+                else:
+                    P = H.prepare_weights(H.desc_from_spec(L), params[0], params[1], sc["s_x"], sc["s_out"], act,
+                                          hb_next, False)
                 x = torch.from_numpy(I.activations_i8((n, h, w, L.c_in), seed=5, s_in=0.05)).cuda()
                 y = torch.empty(P.out_shape(n, h, w), dtype=torch.int8, device="cuda")
                 ms = time_events(lambda: H.conv2d_i8(x, P, y=y), args.steps, args.warmup)
@@ -254,7 +266,8 @@ def run_layer_mode(args, cfg, scales):
                 peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
                 peak = peaks.get("bf16_tflops", FALLBACK_BF16_TFLOPS)
                 tf = flops / (ms / 1000) / 1e12
-                print(json.dumps({"mode": "layer", "layer": L.name, "chain": ch.name, "batch": n, "in_hw": [h, w],
+                print(json.dumps({"mode": "layer", "layer": L.name, "act": act, "chain": ch.name, "batch": n,
+                                  "in_hw": [h, w],
                                   "c_in": L.c_in, "c_out": L.c_out, "k": L.k, "stride": L.stride, "form": L.form,
                                   "hb_next": hb_next, "ms": ms, "tflops": tf, "peak_bf16_burst": peak,
                                   "frac": tf / peak}), flush=True)
