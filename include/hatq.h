@@ -209,13 +209,17 @@ hatq_status hatq_quantize_act(const void *x, int x_kind, float s_in, int n, int 
  *   a = sum_k x_int w_int + b_int                    (exact integer)
  *   INT8 output:  y = clamp(round(H~_next phi(H~_out (M (.) a)) / 2^n))
  *   float output: y = phi(H~_out (deq (.) a))        (float32, no rounding)
- * where H~_out is applied for WH layers and H~_next when hb_next > 0.
+ * where H~_out is applied for WH layers and H~_next when hb_next > 0; a layer
+ * prepared by hatq_prepare_weights_general (SiLU / GELU) takes that entry
+ * point's two-step transition instead.
  *   x   device NHWC int8 [n][h][w][c_in], the layer's operand (basis and scale s_x).
  *   y   device NHWC [n][ho][wo][c_out], int8 or float32 (L->out_f32),
  *       ho = (h + 2 pad - kh) / stride + 1 (floor), likewise wo.
  * The reduction runs on the tensor cores with the codes held exactly as fp16
  * operands and fp32 partial sums that stay below 2^24 in magnitude, moved to
  * int32 every 1024 reduction elements, so the accumulator is exact.
+ * Work is enqueued only: results are complete once `stream` is synchronized
+ * (check them with hatq_sync_status()).
  */
 hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prepared *L,
                            void *y, hatq_stream stream);
