@@ -58,6 +58,132 @@ def sylvester(m: int) -> np.ndarray:
     return H
 
 
+# --------------------------------------------------------------------------
+# Paper-exact orders (Supp. Hadamard construction): Paley-I / Paley-II and
+# Kronecker products, Eq. (hadamard_order), padded transforms of Eq.
+# (supp_padded_transforms). Reading: q is restricted to primes (the paper
+# allows prime powers, whose finite-field arithmetic is not built here).
+# --------------------------------------------------------------------------
+
+
+def _is_prime(q: int) -> bool:
+    if q < 2:
+        return False
+    f = 2
+    while f * f <= q:
+        if q % f == 0:
+            return False
+        f += 1
+    return True
+
+
+def _jacobsthal(q: int) -> np.ndarray:
+    """Q[i, j] = chi(j - i) with chi the quadratic character modulo the prime q."""
+    squares = {(x * x) % q for x in range(1, q)}
+    chi = np.array([0] + [1 if a in squares else -1 for a in range(1, q)], dtype=np.int64)
+    idx = (np.arange(q)[None, :] - np.arange(q)[:, None]) % q
+    return chi[idx]
+
+
+def paley1(q: int) -> np.ndarray:
+    """Paley-I Hadamard matrix of order q + 1, q a prime with q = 3 (mod 4):
+    H = I + S with S = [[0, 1^T], [-1, Q]] (S antisymmetric)."""
+    if not _is_prime(q) or q % 4 != 3:
+        raise ValueError("Paley-I needs a prime q = 3 (mod 4)")
+    Q = _jacobsthal(q)
+    S = np.zeros((q + 1, q + 1), dtype=np.int64)
+    S[0, 1:] = 1
+    S[1:, 0] = -1
+    S[1:, 1:] = Q
+    return np.eye(q + 1, dtype=np.int64) + S
+
+
+def paley2(q: int) -> np.ndarray:
+    """Paley-II Hadamard matrix of order 2 (q + 1), q a prime with q = 1 (mod 4):
+    the symmetric conference matrix C = [[0, 1^T], [1, Q]] gives
+    H = C (x) [[1, 1], [1, -1]] + I (x) [[1, -1], [-1, -1]]."""
+    if not _is_prime(q) or q % 4 != 1:
+        raise ValueError("Paley-II needs a prime q = 1 (mod 4)")
+    Q = _jacobsthal(q)
+    Cm = np.zeros((q + 1, q + 1), dtype=np.int64)
+    Cm[0, 1:] = 1
+    Cm[1:, 0] = 1
+    Cm[1:, 1:] = Q
+    A = np.array([[1, 1], [1, -1]], dtype=np.int64)
+    B = np.array([[1, -1], [-1, -1]], dtype=np.int64)
+    return np.kron(Cm, A) + np.kron(np.eye(q + 1, dtype=np.int64), B)
+
+
+def _base_orders(limit: int) -> dict:
+    """Orders <= limit from Sylvester (2^k), Paley-I and Paley-II, each with a
+    constructor (Sylvester preferred, then Paley-I, then Paley-II)."""
+    out = {}
+    m = 1
+    while m <= limit:
+        out[m] = ("sylvester", m)
+        m *= 2
+    for q in range(3, limit):
+        if _is_prime(q):
+            if q % 4 == 3 and q + 1 <= limit and q + 1 not in out:
+                out[q + 1] = ("paley1", q)
+            if q % 4 == 1 and 2 * (q + 1) <= limit and 2 * (q + 1) not in out:
+                out[2 * (q + 1)] = ("paley2", q)
+    return out
+
+
+_ORDERS_CACHE = {}
+
+
+def supported_orders(limit: int = 1024) -> dict:
+    """The set M_H of supported orders <= limit: base orders and Kronecker
+    products of supported orders, each with a recipe (a nested tuple).
+    Recipes only (no matrices), cached per limit."""
+    if limit in _ORDERS_CACHE:
+        return dict(_ORDERS_CACHE[limit])
+    orders = dict(_base_orders(limit))
+    changed = True
+    while changed:
+        changed = False
+        for a in sorted(orders):
+            for b in sorted(orders):
+                if a < 2 or b < 2 or a * b > limit or a * b in orders:
+                    continue
+                orders[a * b] = ("kron", a, b)
+                changed = True
+    _ORDERS_CACHE[limit] = dict(orders)
+    return orders
+
+
+def hadamard_of_order(m: int, orders: dict = None) -> np.ndarray:
+    """An unnormalized Hadamard matrix of a supported order m."""
+    orders = orders or supported_orders(max(1024, m))
+    if m not in orders:
+        raise ValueError(f"order {m} is not supported")
+    r = orders[m]
+    if r[0] == "sylvester":
+        return sylvester(m)
+    if r[0] == "paley1":
+        return paley1(r[1])
+    if r[0] == "paley2":
+        return paley2(r[1])
+    return np.kron(hadamard_of_order(r[1], orders), hadamard_of_order(r[2], orders))
+
+
+def hadamard_order(c: int, limit: int = 4096) -> int:
+    """m(C) of Eq. (hadamard_order): the smallest supported order >= 4 ceil(C / 4)."""
+    c4 = 4 * ((c + 3) // 4)
+    orders = supported_orders(limit)
+    return min(m for m in orders if m >= c4)
+
+
+def padded_transforms(c: int):
+    """T_in = P_C H_m and T_out = P_C H_m^T of Eq. (supp_padded_transforms),
+    with H_m = H~_m / sqrt(m) and P_C = [I_C 0]: [C, m] fp64 each."""
+    m = hadamard_order(c)
+    H = hadamard_of_order(m).astype(np.float64) / math.sqrt(m)
+    return H[:c, :], H.T[:c, :]
+
+
 def blockdiag_transform(c: int, hb: int) -> np.ndarray:
     """Normalized block-diagonal transform T = I_{c/hb} (x) H_hb (reading R1),
     H_hb = H~_hb / sqrt(hb) (Eq. hadamard_properties). Dense fp64 [c, c]."""

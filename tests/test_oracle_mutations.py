@@ -14,7 +14,8 @@ _orig = {k: getattr(O, k) for k in ("sylvester", "transform_real", "transform_in
                                     "fixed_point", "prepare_layer", "epilogue_int", "conv_codes",
                                     "quantize_act_i8", "transform_weights", "quantize_sym",
                                     "act_multiplier", "range_expansion_codes", "select_form",
-                                    "epilogue_general", "phi")}
+                                    "epilogue_general", "phi", "paley1", "padded_transforms",
+                                    "_jacobsthal")}
 
 
 def _sylvester_bad(m):
@@ -128,7 +129,26 @@ def _phi_sign(kind, v):
     return v / (1.0 + math.exp(v)) if kind == "silu" else _orig["phi"](kind, -v)
 
 
+def _paley1_no_identity(q):
+    return _orig["paley1"](q) - np.eye(q + 1, dtype=np.int64)
+
+
+def _jacobsthal_chi0(q):
+    Q = _orig["_jacobsthal"](q).copy()
+    np.fill_diagonal(Q, 1)
+    return Q
+
+
+def _padded_unnormalized(c):
+    T_in, T_out = _orig["padded_transforms"](c)
+    m = T_in.shape[1]
+    return T_in * math.sqrt(m), T_out * math.sqrt(m)
+
+
 MUTATIONS = {
+    "paley1_identity_dropped": ("paley1", _paley1_no_identity),
+    "jacobsthal_chi0": ("_jacobsthal", _jacobsthal_chi0),
+    "padded_unnormalized": ("padded_transforms", _padded_unnormalized),
     "general_M_after_H_out": ("epilogue_general", _general_h_before_m),
     "general_lut_index_shift": ("epilogue_general", _general_lut_shifted),
     "phi_sign": ("phi", _phi_sign),

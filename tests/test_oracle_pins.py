@@ -535,3 +535,64 @@ def test_general_transition_tracks_real_model(form, hb_next, kind):
     y = O.conv_layer(op, p).astype(np.float64) * p.s_y
     assert O.sqnr_db(target, y) > (24.0 if form == "DH" else 18.0)
     assert np.mean(np.abs(O.conv_layer(op, p)) == 127) < 0.1
+
+
+# ------------------------------------------------------- paper-exact orders (Supp. Hadamard construction)
+
+def test_every_supported_order_is_a_hadamard_matrix():
+    """Eq. hadamard_properties for every order of M_H up to 256: entries +-1
+    and H~ H~^T = m I (Sylvester, Paley-I, Paley-II, Kronecker products)."""
+    orders = O.supported_orders(256)
+    assert {4, 8, 12, 20, 24, 28, 36, 44, 192, 224, 240} <= set(orders)
+    for m in orders:
+        H = O.hadamard_of_order(m, orders)
+        assert H.shape == (m, m) and np.all(np.abs(H) == 1)
+        assert np.array_equal(H @ H.T, m * np.eye(m, dtype=np.int64)), m
+
+
+def test_paley_constructions_closed_forms():
+    """Paley-I (q = 3 mod 4) gives order q + 1 from an antisymmetric Jacobsthal
+    matrix, Paley-II (q = 1 mod 4) order 2 (q + 1) from a symmetric one; both
+    reject the other residue class."""
+    Q7 = O._jacobsthal(7)
+    assert np.array_equal(Q7, -Q7.T) and np.all(Q7.sum(axis=1) == 0)
+    Q13 = O._jacobsthal(13)
+    assert np.array_equal(Q13, Q13.T)
+    assert O.paley1(7).shape == (8, 8) and O.paley2(13).shape == (28, 28)
+    for bad in (lambda: O.paley1(13), lambda: O.paley2(7), lambda: O.paley1(15)):
+        with pytest.raises(ValueError):
+            bad()
+
+
+def test_hadamard_order_rule():
+    """Eq. hadamard_order: m(C) = min supported order >= 4 ceil(C / 4); the
+    orders the paper names: m(192) = 192 (Paley-I, q = 191), m(224) = 224
+    (q = 223), m(320) = 320 (a Kronecker product)."""
+    assert O.hadamard_order(192) == 192 and O.supported_orders(256)[192] == ("paley1", 191)
+    assert O.hadamard_order(224) == 224 and O.supported_orders(256)[224] == ("paley1", 223)
+    assert O.hadamard_order(320) == 320 and O.supported_orders(512)[320][0] == "kron"
+    assert O.hadamard_order(3) == 4 and O.hadamard_order(13) == 16 and O.hadamard_order(100) == 104
+    for c in range(1, 300, 7):
+        m = O.hadamard_order(c)
+        assert m >= 4 * ((c + 3) // 4)
+        assert not any(4 * ((c + 3) // 4) <= k < m for k in O.supported_orders(512))
+
+
+@pytest.mark.parametrize("c", [3, 20, 100, 192, 200])
+def test_padded_transforms_are_semi_orthogonal_and_preserve_the_layer(c):
+    """Eqs. supp_padded_transforms, supp_semi_orthogonality: T T^T = I_C for
+    both orientations, so DH (X T_in)(W T_in)^T and WH (X (T_out^T W)^T) T_out^T
+    both reproduce X W^T with padding to m(C)."""
+    T_in, T_out = O.padded_transforms(c)
+    m = O.hadamard_order(c)
+    assert T_in.shape == (c, m) and T_out.shape == (c, m)
+    assert np.allclose(T_in @ T_in.T, np.eye(c), atol=1e-12)
+    assert np.allclose(T_out @ T_out.T, np.eye(c), atol=1e-12)
+    rng = np.random.default_rng(c)
+    X = rng.standard_normal((5, c))
+    W = rng.standard_normal((7, c))
+    assert np.allclose((X @ T_in) @ (W @ T_in).T, X @ W.T, atol=1e-10)
+    Wo = rng.standard_normal((c, 6))                         # C_out = c rows
+    Xo = rng.standard_normal((4, 6))
+    Wbar = T_out.T @ Wo                                      # m x C_in
+    assert np.allclose((Xo @ Wbar.T) @ T_out.T, Xo @ Wo.T, atol=1e-10)
