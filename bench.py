@@ -183,7 +183,7 @@ def run_reference(args, cfg, scales):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * t, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "int64", "data": "synthetic",
             "effective_tops": ops / t / 1e12,
-            "config": {"workload": workload_name(cfg), "global_batch": 8, "seq_len": 0},
+            "config": {"workload": workload_name(cfg), "global_batch": 8},
             "cpu_baseline": {"value": value, "unit": "images/s", "cores": threads, "kind": "oracle", "sample": sample},
             "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -477,10 +477,12 @@ def main():
     line = {
         "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world, "steps": args.steps,
         "warmup": max(3, args.warmup), "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
-        "vs_baseline": None, "dtype": "int8 (exact, fp16 tensor-core operands, int32 accumulate)",
+        "vs_baseline": None, "dtype": "int8",
+        "arithmetic": "INT8 codes as exact fp16 tensor-core operands, fp32 chunk sums below 2^24, int32 totals, "
+                      "int64 requantization",
         "data": "synthetic (seeded LIC-shaped inputs, random-init weights)",
         "effective_tops": world * 2 * macs_step / (ms / 1000.0) / 1e12,
-        "config": {"workload": workload_name(cfg), "global_batch": world * images_step, "seq_len": 0,
+        "config": {"workload": workload_name(cfg), "global_batch": world * images_step,
                    "parallelism": f"replicas x{world}", "l2": "inputs larger than L2 (199 MB image batch)"},
         "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
         "gpu_launches": launches_step * args.steps,
