@@ -199,3 +199,43 @@ def test_general_prepare_rejects_what_it_does_not_cover(lib):
     with pytest.raises(H.HatqError) as e:                       # SiLU through the homogeneous entry point
         H.prepare_weights_host(d, w, None, 0.1, 0.1, "silu", 0)
     assert e.value.status == H.ERR_INVALID_ARG
+
+
+def test_binding_constants_match_the_header():
+    """The Python binding's status, form, activation and input-kind values
+    are the ones include/hatq.h declares."""
+    import re
+    text = open(os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "hatq.h")).read()
+    decl = {k: int(v) for k, v in re.findall(r"\b(HATQ_[A-Z0-9_]+)\s*=\s*(\d+)", text)}
+    expect = {"HATQ_OK": H.OK, "HATQ_ERR_INVALID_ARG": H.ERR_INVALID_ARG, "HATQ_ERR_UNSUPPORTED": H.ERR_UNSUPPORTED,
+              "HATQ_ERR_OVERFLOW": H.ERR_OVERFLOW, "HATQ_ERR_CUDA": H.ERR_CUDA, "HATQ_ERR_TIMEOUT": H.ERR_TIMEOUT,
+              "HATQ_DH": H.DH, "HATQ_WH": H.WH, "HATQ_ACT_NONE": H.ACT_NONE, "HATQ_ACT_RELU": H.ACT_RELU,
+              "HATQ_ACT_SILU": H.ACT_SILU, "HATQ_ACT_GELU": H.ACT_GELU, "HATQ_IN_OPERAND": H.IN_OPERAND,
+              "HATQ_IN_I8": H.IN_I8, "HATQ_IN_F16": H.IN_F16}
+    for name, value in expect.items():
+        assert decl[name] == value, name
+
+
+def test_prepared_struct_mirror_matches_the_c_layout(tmp_path):
+    """The ctypes mirror of hatq_prepared has the size and field offsets the C
+    compiler gives the header's struct (the library writes the whole struct)."""
+    import ctypes
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    fields = ["d", "act", "hb_next", "out_f32", "shift", "k_pad", "gather", "s_x", "s_y", "w_i8", "w_f16", "b_int",
+              "mult", "deq", "s_w", "opaque", "s_z", "s_u", "shift_in", "reserved", "mult_in", "lut"]
+    src = tmp_path / "layout.c"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    src.write_text("#include <stdio.h>\n#include <stddef.h>\n#include \"hatq.h\"\nint main(void) {\n"
+                   "  printf(\"%zu\\n\", sizeof(hatq_prepared));\n"
+                   + "".join(f"  printf(\"%zu\\n\", offsetof(hatq_prepared, {f}));\n" for f in fields)
+                   + "  return 0;\n}\n")
+    exe = tmp_path / "layout"
+    subprocess.run([cc, "-I", inc, str(src), "-o", str(exe)], check=True, capture_output=True)
+    out = [int(v) for v in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()]
+    assert ctypes.sizeof(H.PreparedStruct) == out[0]
+    for f, off in zip(fields, out[1:]):
+        assert getattr(H.PreparedStruct, f).offset == off, f
