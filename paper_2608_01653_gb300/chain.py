@@ -15,8 +15,9 @@ from . import hatq
 class Chain:
     def __init__(self, layers, params, scales, plan, out_f32_last=False, device="cuda"):
         """layers: objects with c_in, c_out, k, stride, pad, form, hb_in, hb_out, act;
-        params: [(w_ohwi float32, bias float32)]; scales: [{'s_x', 's_out'}];
-        plan: per layer the block of the next layer's DH transform fused in its epilogue (0 = none)."""
+        params: [(w_ohwi float32, bias float32)]; scales: [{'s_x', 's_out'}, plus 's_z' and
+        's_u' for a SiLU / GELU layer]; plan: per layer the block of the next layer's DH
+        transform fused in its epilogue (0 = none)."""
         self.layers = list(layers)
         self.plan = list(plan)
         self.prepared = []
@@ -24,7 +25,7 @@ class Chain:
             last = i == len(self.layers) - 1
             self.prepared.append(hatq.prepare_weights(
                 hatq.desc_from_spec(L), w, b, sc["s_x"], sc["s_out"], L.act, self.plan[i],
-                out_f32_last and last, device=device))
+                out_f32_last and last, device=device, s_z=sc.get("s_z"), s_u=sc.get("s_u")))
 
     def input_kinds(self, x_kind, s_in):
         """(kind, scale) of each layer's input, mirroring what each epilogue emits."""
