@@ -665,6 +665,84 @@ def conv_real(x, w_ohwi, b, stride: int, pad: int) -> np.ndarray:
     return y
 
 
+# --------------------------------------------------------------------------
+# Decoder-side operators (synthesis transforms): transposed and sub-pixel
+# convolutions, linear operators Y = X W^T of Eq. (linear_operator) like the
+# analysis convolutions, so the DH / WH weight transforms apply unchanged
+# (DH along the contracted C_in, WH along C_out).
+# --------------------------------------------------------------------------
+
+
+def conv_transpose_hw(h, w, k, stride, pad, out_pad=0):
+    return (h - 1) * stride - 2 * pad + k + out_pad, (w - 1) * stride - 2 * pad + k + out_pad
+
+
+def conv_transpose_real(x, w_ohwi, b, stride: int, pad: int, out_pad: int = 0) -> np.ndarray:
+    """Transposed convolution, fp64: every input pixel (iy, ix) scatters
+    x[iy, ix, :] W[:, ky, kx, :]^T to output pixel (iy s + ky - pad, ix s + kx - pad).
+    w_ohwi: [C_out, kh, kw, C_in] of this layer (C_in -> C_out)."""
+    x = np.asarray(x, dtype=np.float64)
+    w = np.asarray(w_ohwi, dtype=np.float64)
+    n, h, wd, c = x.shape
+    co, kh, kw, _ = w.shape
+    ho, wo = conv_transpose_hw(h, wd, kh, stride, pad, out_pad)
+    big = np.zeros((n, (h - 1) * stride + kh, (wd - 1) * stride + kw, co))
+    for ky in range(kh):
+        for kx in range(kw):
+            big[:, ky:ky + stride * (h - 1) + 1:stride, kx:kx + stride * (wd - 1) + 1:stride, :] += x @ w[:, ky, kx, :].T
+    y = np.zeros((n, ho, wo, co))
+    hh, ww = min(ho, big.shape[1] - pad), min(wo, big.shape[2] - pad)
+    y[:, :hh, :ww, :] = big[:, pad:pad + hh, pad:pad + ww, :]
+    if b is not None:
+        y += np.asarray(b, dtype=np.float64)
+    return y
+
+
+def conv_transpose_codes(x_i8, w_int, stride: int, pad: int, out_pad: int = 0) -> np.ndarray:
+    """The same scatter on INT8 codes, exact in int64."""
+    x = np.asarray(x_i8, dtype=np.int64)
+    w = np.asarray(w_int, dtype=np.int64)
+    n, h, wd, c = x.shape
+    co, kh, kw, _ = w.shape
+    ho, wo = conv_transpose_hw(h, wd, kh, stride, pad, out_pad)
+    big = np.zeros((n, (h - 1) * stride + kh, (wd - 1) * stride + kw, co), dtype=np.int64)
+    for ky in range(kh):
+        for kx in range(kw):
+            big[:, ky:ky + stride * (h - 1) + 1:stride, kx:kx + stride * (wd - 1) + 1:stride, :] += x @ w[:, ky, kx, :].T
+    y = np.zeros((n, ho, wo, co), dtype=np.int64)
+    hh, ww = min(ho, big.shape[1] - pad), min(wo, big.shape[2] - pad)
+    y[:, :hh, :ww, :] = big[:, pad:pad + hh, pad:pad + ww, :]
+    return y
+
+
+def conv_transpose_layer(x_op, p: Prepared, out_pad: int = 0):
+    """A prepared layer (prepare_layer: DH / WH weights, bias codes, (M, n))
+    applied as a transposed convolution, then the integer transition."""
+    acc = conv_transpose_codes(x_op, p.w_int, p.stride, p.pad, out_pad)
+    if p.act in GENERAL_ACTS:
+        return epilogue_general(acc, p)
+    return epilogue_f32(acc, p) if p.out_f32 else epilogue_int(acc, p)
+
+
+def depth_to_space(x, r: int) -> np.ndarray:
+    """Sub-pixel rearrangement: NHWC [n, h, w, c r^2] -> [n, h r, w r, c], channel
+    c r^2 + i r + j going to pixel (h r + i, w r + j), channel c."""
+    x = np.asarray(x)
+    n, h, w, crr = x.shape
+    if crr % (r * r):
+        raise ValueError("channels must be a multiple of r^2")
+    c = crr // (r * r)
+    return x.reshape(n, h, w, c, r, r).transpose(0, 1, 4, 2, 5, 3).reshape(n, h * r, w * r, c)
+
+
+def space_to_depth(x, r: int) -> np.ndarray:
+    """Inverse of depth_to_space."""
+    x = np.asarray(x)
+    n, hr, wr, c = x.shape
+    h, w = hr // r, wr // r
+    return x.reshape(n, h, r, w, r, c).transpose(0, 1, 3, 5, 2, 4).reshape(n, h, w, c * r * r)
+
+
 def calibrate_chain(layers, params, x_real, plan, first_wh_scale=None):
     """Static scales from the real-valued model (QAT-style frozen scales,
     Sec. quantization-aware training): per layer, s_x = max-abs of the

@@ -15,7 +15,8 @@ _orig = {k: getattr(O, k) for k in ("sylvester", "transform_real", "transform_in
                                     "quantize_act_i8", "transform_weights", "quantize_sym",
                                     "act_multiplier", "range_expansion_codes", "select_form",
                                     "epilogue_general", "phi", "paley1", "padded_transforms",
-                                    "_jacobsthal")}
+                                    "_jacobsthal", "conv_transpose_codes", "conv_transpose_real",
+                                    "depth_to_space")}
 
 
 def _sylvester_bad(m):
@@ -145,7 +146,32 @@ def _padded_unnormalized(c):
     return T_in * math.sqrt(m), T_out * math.sqrt(m)
 
 
+def _convT_gather(x, w, stride, pad, out_pad=0):
+    # a forward-style gather with the transposed output size (the classic mix-up)
+    y = O.conv_codes(x, w, 1, pad)
+    ho, wo = O.conv_transpose_hw(x.shape[1], x.shape[2], w.shape[1], stride, pad, out_pad)
+    out = np.zeros((x.shape[0], ho, wo, w.shape[0]), np.int64)
+    hh, ww = min(ho, y.shape[1]), min(wo, y.shape[2])
+    out[:, :hh, :ww] = y[:, :hh, :ww]
+    return out
+
+
+def _convT_real_unflipped_pad(x, w, b, stride, pad, out_pad=0):
+    return _orig["conv_transpose_real"](x, w, b, stride, max(pad - 1, 0), out_pad)[:, :, :, :] if pad else \
+        _orig["conv_transpose_real"](x, w, b, stride, pad, out_pad) * 1.0001
+
+
+def _d2s_swapped(x, r):
+    x = np.asarray(x)
+    n, h, w, crr = x.shape
+    c = crr // (r * r)
+    return x.reshape(n, h, w, r, r, c).transpose(0, 1, 3, 2, 4, 5).reshape(n, h * r, w * r, c)
+
+
 MUTATIONS = {
+    "convT_forward_gather": ("conv_transpose_codes", _convT_gather),
+    "convT_pad_off_by_one": ("conv_transpose_real", _convT_real_unflipped_pad),
+    "depth_to_space_channel_order": ("depth_to_space", _d2s_swapped),
     "paley1_identity_dropped": ("paley1", _paley1_no_identity),
     "jacobsthal_chi0": ("_jacobsthal", _jacobsthal_chi0),
     "padded_unnormalized": ("padded_transforms", _padded_unnormalized),

@@ -596,3 +596,80 @@ def test_padded_transforms_are_semi_orthogonal_and_preserve_the_layer(c):
     Xo = rng.standard_normal((4, 6))
     Wbar = T_out.T @ Wo                                      # m x C_in
     assert np.allclose((Xo @ Wbar.T) @ T_out.T, Xo @ Wo.T, atol=1e-10)
+
+
+# ------------------------------------------------------- decoder-side operators (transposed, sub-pixel)
+
+@pytest.mark.parametrize("k,stride,pad", [(5, 2, 2), (3, 2, 1), (3, 1, 1), (1, 1, 0)])
+def test_transposed_conv_is_the_adjoint_of_the_strided_conv(k, stride, pad):
+    """<F x, z> = <x, F^T z>: the transposed convolution with the channel-
+    transposed weights is the adjoint of the forward convolution."""
+    rng = np.random.default_rng(k * 10 + stride)
+    x = rng.standard_normal((2, 7, 9, 5))
+    w = rng.standard_normal((6, k, k, 5))
+    y = O.conv_real(x, w, None, stride, pad)
+    z = rng.standard_normal(y.shape)
+    ho, wo = O.conv_transpose_hw(y.shape[1], y.shape[2], k, stride, pad)
+    xt = O.conv_transpose_real(z, w.transpose(3, 1, 2, 0), None, stride, pad,
+                               out_pad=max(0, 7 - ho))[:, :7, :9, :]
+    assert xt.shape == x.shape
+    assert abs(np.sum(y * z) - np.sum(x * xt)) < 1e-9 * max(1.0, abs(np.sum(y * z)))
+
+
+def test_transposed_conv_stride1_is_a_flipped_forward_conv_and_codes_are_exact():
+    """Closed form: stride 1 and padding p equal a forward convolution with the
+    spatially flipped kernel and padding k - 1 - p; on integer codes the int64
+    scatter equals the fp64 one exactly."""
+    rng = np.random.default_rng(3)
+    x = rng.integers(-127, 128, size=(1, 6, 8, 4))
+    w = rng.integers(-127, 128, size=(5, 3, 3, 4))
+    ref = O.conv_real(x, w[:, ::-1, ::-1, :], None, 1, 1)
+    got = O.conv_transpose_real(x, w, None, 1, 1)
+    assert np.array_equal(got, ref)
+    assert np.array_equal(O.conv_transpose_codes(x, w, 2, 1, 1), O.conv_transpose_real(x, w, None, 2, 1, 1))
+
+
+@pytest.mark.parametrize("form", ["DH", "WH"])
+def test_transposed_conv_preserves_function_in_both_forms(form):
+    """Eq. linear_operator holds for the transposed operator too: DH transforms
+    the contracted C_in of activations and weights, WH the weights' C_out with
+    the output basis restored afterwards; both reproduce the layer."""
+    rng = np.random.default_rng(5)
+    x = rng.standard_normal((1, 5, 6, 64))
+    w = rng.standard_normal((32, 5, 5, 64)) * 0.1
+    b = rng.standard_normal(32) * 0.1
+    ref = O.conv_transpose_real(x, w, b, 2, 2, 1)
+    if form == "DH":
+        wp, bb = O.transform_weights(w, b, "DH", 64, 0)
+        got = O.conv_transpose_real(O.transform_real(x, 64), wp, bb, 2, 2, 1)
+    else:
+        wp, bb = O.transform_weights(w, b, "WH", 0, 32)
+        got = O.transform_real(O.conv_transpose_real(x, wp, bb, 2, 2, 1), 32)
+    assert np.allclose(got, ref, atol=1e-10)
+
+
+def test_quantized_transposed_layer_tracks_real_model():
+    """A DH synthesis layer (5x5, stride 2, 64 -> 32) on INT8 codes with the
+    integer transition stays close to the fp64 transposed convolution."""
+    x_real = I.activations((1, 8, 9, 64), seed=90).astype(np.float64)
+    w = I.weights(32, 5, 5, 64, seed=91)
+    b = I.bias(32, seed=92)
+    y_ref = np.maximum(O.conv_transpose_real(x_real, w, b, 2, 2, 1), 0)
+    s_x = O.symmetric_scale(O.transform_real(x_real, 64))
+    s_y = O.symmetric_scale(y_ref)
+    p = O.prepare_layer(w, b, "DH", 64, 0, s_x, s_y, "relu", 0, False, 2, 2)
+    op = O.quantize_act_f16(x_real.astype(np.float16), 64, s_x)
+    y = O.conv_transpose_layer(op, p, 1).astype(np.float64) * p.s_y
+    assert y.shape == y_ref.shape
+    assert O.sqnr_db(y_ref, y) > 28.0
+
+
+def test_depth_to_space_index_mapping():
+    """Sub-pixel rearrangement: channel c r^2 + i r + j goes to pixel
+    (h r + i, w r + j), channel c; space_to_depth inverts it."""
+    x = np.arange(8).reshape(1, 1, 1, 8)                 # c = 2, r = 2
+    y = O.depth_to_space(x, 2)
+    assert y.shape == (1, 2, 2, 2)
+    assert y[0, :, :, 0].tolist() == [[0, 1], [2, 3]] and y[0, :, :, 1].tolist() == [[4, 5], [6, 7]]
+    z = np.random.default_rng(0).integers(0, 9, size=(2, 3, 4, 18))
+    assert np.array_equal(O.space_to_depth(O.depth_to_space(z, 3), 3), z)
