@@ -26,6 +26,16 @@ Readings the paper leaves open (the same list is kept with the design notes):
   R6 fixed summation order for real-valued transforms: for output j,
      acc = 0; acc += H[i][j] * x_i for i = 0..hb-1; then acc / sqrt(hb).
 
+  R7 non-homogeneous activations (SiLU, GELU) take the two-step transition of
+     the supplementary's general nonlinearities: both multiplier/shift pairs by
+     R3, the table phi_int in fp64 (math-library exp / erf) rounded by R2.
+  R8 the range-expansion statistic is decided on the INT8 codes a layer
+     receives, exactly: max|H~ x|^2 > hb max|x|^2.
+  R9 Paley constructions are taken over primes q only; any valid construction
+     of an order serves.
+  R10 transposed convolutions use the same prepared weights (DH / WH along
+     C_in / C_out) as a scatter; the integer transition is unchanged.
+
 parity unpinned: the rounding convention R2 and the (M, n) rule R3 are
 conventions of this implementation (the paper fixes neither); the oracle pins
 them against exact rational arithmetic, not against the paper.
