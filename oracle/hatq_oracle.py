@@ -676,6 +676,72 @@ def conv_real(x, w_ohwi, b, stride: int, pad: int) -> np.ndarray:
 
 
 # --------------------------------------------------------------------------
+# Dynamic affine activation quantization (PTQ setting): Eqs. (uniform_q,
+# affine_q); the MACs and transforms use centred codes x_int - z_x
+# (supplementary, affine activation quantization)
+# --------------------------------------------------------------------------
+
+AFFINE_QMIN, AFFINE_QMAX = 0, 255          # unsigned 8-bit grid of Eq. affine_q
+
+
+def affine_params(x):
+    """(s, z) of Eq. affine_q from the tensor's range, zero kept representable:
+    x_min' = min(x_min, 0), x_max' = max(x_max, 0), s = (x_max' - x_min') / 255,
+    z = clamp(round(0 - x_min' / s), 0, 255); a zero range gives (1, 0)."""
+    x = np.asarray(x, dtype=np.float64)
+    lo = min(float(x.min()), 0.0) if x.size else 0.0
+    hi = max(float(x.max()), 0.0) if x.size else 0.0
+    if hi - lo <= 0.0:
+        return 1.0, 0
+    s = (hi - lo) / (AFFINE_QMAX - AFFINE_QMIN)
+    z = int(min(max(round(AFFINE_QMIN - lo / s), AFFINE_QMIN), AFFINE_QMAX))
+    return s, z
+
+
+def quantize_affine(x, s: float, z: int) -> np.ndarray:
+    """x_int = clamp(round(x / s) + z, 0, 255) of Eq. uniform_q."""
+    q = np.rint(np.asarray(x, dtype=np.float64) / s) + z
+    return np.clip(q, AFFINE_QMIN, AFFINE_QMAX).astype(np.int64)
+
+
+def conv_codes_wide(x_int, w_int, stride: int, pad: int) -> np.ndarray:
+    """The integer accumulator for codes wider than INT8 (centred affine codes,
+    |x| <= 255): a library matmul per kernel tap in int64, zero padding."""
+    x = np.asarray(x_int, dtype=np.int64)
+    w = np.asarray(w_int, dtype=np.int64)
+    n, h, wd, c = x.shape
+    co, kh, kw, _ = w.shape
+    ho, wo = out_hw(h, wd, kh, stride, pad)
+    xp = np.zeros((n, h + 2 * pad, wd + 2 * pad, c), dtype=np.int64)
+    xp[:, pad:pad + h, pad:pad + wd, :] = x
+    acc = np.zeros((n, ho, wo, co), dtype=np.int64)
+    for ky in range(kh):
+        for kx in range(kw):
+            patch = xp[:, ky:ky + stride * (ho - 1) + 1:stride, kx:kx + stride * (wo - 1) + 1:stride, :]
+            acc += patch @ w[:, ky, kx, :].T
+    return acc
+
+
+def conv_layer_affine(x_real, p: Prepared):
+    """A prepared layer (out_f32 preparation: DH / WH weights, s_w, bias) on a
+    real input with dynamic affine activation quantization: the input-side
+    operand (T x for DH, x for WH) is quantized with (s, z) from its own range,
+    the convolution runs on the centred codes x_int - z (zero padding is a
+    centred zero), and the output is dequantized:
+    y = H_out(s s_w (.) a) + b_bar, a = sum (x_int - z) w_int.
+    Returns (y, s, z)."""
+    v = transform_real(np.asarray(x_real, dtype=np.float64), p.hb_in) if p.form == "DH" else \
+        np.asarray(x_real, dtype=np.float64)
+    s, z = affine_params(v)
+    centred = quantize_affine(v, s, z) - z
+    acc = conv_codes_wide(centred, p.w_int, p.stride, p.pad)
+    t = (s * p.s_w) * acc.astype(np.float64)
+    y = transform_real(t, p.hb_out) if p.form == "WH" else t
+    y = y + p.bbar if p.form == "DH" else y + transform_real(p.bbar, p.hb_out)
+    return (np.maximum(y, 0.0) if p.act == "relu" else y), s, z
+
+
+# --------------------------------------------------------------------------
 # Decoder-side operators (synthesis transforms): transposed and sub-pixel
 # convolutions, linear operators Y = X W^T of Eq. (linear_operator) like the
 # analysis convolutions, so the DH / WH weight transforms apply unchanged

@@ -16,7 +16,7 @@ _orig = {k: getattr(O, k) for k in ("sylvester", "transform_real", "transform_in
                                     "act_multiplier", "range_expansion_codes", "select_form",
                                     "epilogue_general", "phi", "paley1", "padded_transforms",
                                     "_jacobsthal", "conv_transpose_codes", "conv_transpose_real",
-                                    "depth_to_space")}
+                                    "depth_to_space", "affine_params", "conv_layer_affine")}
 
 
 def _sylvester_bad(m):
@@ -168,7 +168,36 @@ def _d2s_swapped(x, r):
     return x.reshape(n, h, w, r, r, c).transpose(0, 1, 3, 2, 4, 5).reshape(n, h * r, w * r, c)
 
 
+def _affine_z_sign(x):
+    s, z = _orig["affine_params"](x)
+    lo = min(float(np.min(x)), 0.0)
+    return s, int(min(max(round(lo / s), 0), 255)) if s != 1.0 or z else (s, z)
+
+
+def _affine_no_zero_in_range(x):
+    x = np.asarray(x, dtype=np.float64)
+    lo, hi = float(x.min()), float(x.max())
+    if hi - lo <= 0:
+        return 1.0, 0
+    s = (hi - lo) / 255
+    return s, int(min(max(round(-lo / s), 0), 255))
+
+
+def _affine_raw_padding(x_real, p):
+    v = O.transform_real(np.asarray(x_real, dtype=np.float64), p.hb_in) if p.form == "DH" else np.asarray(x_real)
+    s, z = O.affine_params(v)
+    q = O.quantize_affine(v, s, z)
+    acc = O.conv_codes_wide(q, p.w_int, p.stride, p.pad) - z * p.w_int.astype(np.int64).sum(axis=(1, 2, 3))
+    t = (s * p.s_w) * acc.astype(np.float64)
+    y = O.transform_real(t, p.hb_out) if p.form == "WH" else t
+    y = y + p.bbar if p.form == "DH" else y + O.transform_real(p.bbar, p.hb_out)
+    return (np.maximum(y, 0.0) if p.act == "relu" else y), s, z
+
+
 MUTATIONS = {
+    "affine_zero_point_sign": ("affine_params", _affine_z_sign),
+    "affine_zero_not_in_range": ("affine_params", _affine_no_zero_in_range),
+    "affine_padding_raw_code": ("conv_layer_affine", _affine_raw_padding),
     "convT_forward_gather": ("conv_transpose_codes", _convT_gather),
     "convT_pad_off_by_one": ("conv_transpose_real", _convT_real_unflipped_pad),
     "depth_to_space_channel_order": ("depth_to_space", _d2s_swapped),

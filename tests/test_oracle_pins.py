@@ -673,3 +673,55 @@ def test_depth_to_space_index_mapping():
     assert y[0, :, :, 0].tolist() == [[0, 1], [2, 3]] and y[0, :, :, 1].tolist() == [[4, 5], [6, 7]]
     z = np.random.default_rng(0).integers(0, 9, size=(2, 3, 4, 18))
     assert np.array_equal(O.space_to_depth(O.depth_to_space(z, 3), 3), z)
+
+
+# ------------------------------------------------------- dynamic affine activation quantization (PTQ)
+
+def test_affine_params_closed_forms():
+    """Eq. affine_q: s = (max' - min') / 255 and z = round(-min' / s), zero
+    representable exactly; a nonnegative tensor gets z = 0; a zero tensor
+    (1, 0); dequantization error at most s / 2 in range (Eq. uniform_q)."""
+    x = np.array([-1.0, 0.0, 0.5, 2.0])
+    s, z = O.affine_params(x)
+    assert s == pytest.approx(3.0 / 255) and z == 85
+    q = O.quantize_affine(x, s, z)
+    assert q[1] == z and s * (q[1] - z) == 0.0
+    assert np.all(np.abs(s * (q - z) - x) <= s / 2 + 1e-12)
+    assert O.affine_params(np.array([0.2, 3.0])) == pytest.approx((3.0 / 255, 0))
+    assert O.affine_params(np.array([-4.0, -1.0]))[1] == 255
+    assert O.affine_params(np.zeros(5)) == (1.0, 0)
+
+
+def test_wide_code_conv_matches_the_int8_conv_and_fp64():
+    """conv_codes_wide equals the nested-loop C convolution on INT8 codes and
+    the fp64 convolution on centred codes up to +-255 (exact integers)."""
+    rng = np.random.default_rng(4)
+    x8 = rng.integers(-127, 128, size=(2, 7, 6, 16)).astype(np.int8)
+    w = rng.integers(-127, 128, size=(8, 3, 3, 16)).astype(np.int8)
+    assert np.array_equal(O.conv_codes_wide(x8, w, 2, 1), O.conv_codes(x8, w, 2, 1))
+    xw = rng.integers(-255, 256, size=(1, 5, 5, 16))
+    assert np.array_equal(O.conv_codes_wide(xw, w, 1, 1), O.conv_real(xw, w, None, 1, 1).astype(np.int64))
+
+
+@pytest.mark.parametrize("form", ["DH", "WH"])
+def test_dynamic_affine_layer_tracks_real_model_and_pads_with_centred_zero(form):
+    """The PTQ layer: dynamic (s, z) per input, MACs on centred codes,
+    dequantized output; it tracks the fp64 model, and a zero-padded border
+    sees the centred zero (the result equals the layer on an explicitly
+    zero-padded input without padding)."""
+    x_real = I.activations((1, 9, 10, 64), seed=120).astype(np.float64) + 1.5     # shifted, nonzero mean
+    w = I.weights(32, 3, 3, 64, seed=121)
+    b = I.bias(32, seed=122)
+    hb_in, hb_out = (64, 0) if form == "DH" else (0, 32)
+    p = O.prepare_layer(w, b, form, hb_in, hb_out, 1.0, 1.0, "none", 0, True, 1, 1)
+    y, s, z = O.conv_layer_affine(x_real, p)
+    y_ref = O.conv_real(x_real, w, b, 1, 1)
+    assert O.sqnr_db(y_ref, y) > (30.0 if form == "DH" else 22.0)
+    assert z != 0 or form == "WH"
+    xp = np.zeros((1, 11, 12, 64))
+    xp[:, 1:10, 1:11, :] = x_real
+    p0 = O.prepare_layer(w, b, form, hb_in, hb_out, 1.0, 1.0, "none", 0, True, 1, 0)
+    y0, s0, z0 = O.conv_layer_affine(xp, p0)
+    assert (s0, z0) == (s, z) or form == "WH"
+    if form == "DH":
+        assert np.allclose(y0, y, atol=1e-9)
