@@ -35,6 +35,9 @@ Readings the paper leaves open (the same list is kept with the design notes):
      of an order serves.
   R10 transposed convolutions use the same prepared weights (DH / WH along
      C_in / C_out) as a scatter; the integer transition is unchanged.
+  R11 dynamic affine activations: unsigned 8-bit codes (q_min 0, q_max 255),
+     a zero range gives (s, z) = (1, 0), the input-side operand (T x for DH)
+     is quantized and padding is a centred zero.
 
 parity unpinned: the rounding convention R2 and the (M, n) rule R3 are
 conventions of this implementation (the paper fixes neither); the oracle pins
