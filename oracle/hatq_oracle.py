@@ -26,9 +26,10 @@ Readings the paper leaves open (the same list is kept with the design notes):
   R6 fixed summation order for real-valued transforms: for output j,
      acc = 0; acc += H[i][j] * x_i for i = 0..hb-1; then acc / sqrt(hb).
 
-  R7 non-homogeneous activations (SiLU, GELU) take the two-step transition of
-     the supplementary's general nonlinearities: both multiplier/shift pairs by
-     R3, the table phi_int in fp64 (math-library exp / erf) rounded by R2.
+  R7 non-homogeneous activations (SiLU, GELU; GDN, IGDN on the channel
+     vector) take the two-step transition of the supplementary's general
+     nonlinearities: both multiplier/shift pairs by R3, phi_int in fp64
+     (math-library exp / erf, a table for the elementwise ones) rounded by R2.
   R8 the range-expansion statistic is decided on the INT8 codes a layer
      receives, exactly: max|H~ x|^2 > hb max|x|^2.
   R9 Paley constructions are taken over primes q only; any valid construction
@@ -348,6 +349,7 @@ class Prepared:
 
 
 GENERAL_ACTS = ("silu", "gelu")
+VECTOR_ACTS = ("gdn", "igdn")
 
 
 def phi(kind: str, v: float) -> float:
@@ -401,14 +403,14 @@ def prepare_layer(w_ohwi, b, form: str, hb_in: int, hb_out: int, s_x: float,
                     s_x=s_x, s_y=s_y, s_w=s_w, b_int=b_int,
                     w_int=w_int.reshape(wprime.shape).astype(np.int8),
                     a_bound=a_bound, wprime=wprime, bbar=bbar)
-    if act in GENERAL_ACTS:
+    if act in GENERAL_ACTS or act in VECTOR_ACTS:
         if out_f32:
             raise ValueError("the general transition emits INT8 codes")
         s_z = float(np.float32(s_z))
         s_u = float(np.float32(s_u))
         # Eq. supp_general_output_scale: s_A,c / (gamma_out s_z) ~ M_out / 2^n_out, M before H_out
         prep.M, prep.n = fixed_point(s_a / (g_out * s_z), a_bound, hb_out if form == "WH" else 1)
-        prep.lut = activation_lut(act, s_z, s_u)
+        prep.lut = activation_lut(act, s_z, s_u) if act in GENERAL_ACTS else None
         # Eq. supp_general_input_scale: s_u / (gamma_in,next s_x,next) ~ M_in / 2^n_in
         M_in, n_in = fixed_point([s_u / (g_in * s_y)], [QMAX], hb_next if hb_next else 1)
         prep.M_in, prep.n_in = int(M_in[0]), n_in
@@ -583,6 +585,30 @@ def epilogue_general(acc, p: Prepared) -> np.ndarray:
     v = transform_int(t, p.hb_out) if p.hb_out else t
     z = np.clip(rshift_rne(v, p.n), -QMAX, QMAX)
     u = p.lut[z + QMAX]
+    w = p.M_in * u
+    w = transform_int(w, p.hb_next) if p.hb_next else w
+    return np.clip(rshift_rne(w, p.n_in), -QMAX, QMAX).astype(np.int8)
+
+
+def gdn(v, beta, gamma, inverse: bool = False) -> np.ndarray:
+    """Generalized divisive normalization across channels (last axis), fp64:
+    y_i = v_i / sqrt(beta_i + sum_j gamma_ij v_j^2); the inverse (IGDN)
+    multiplies by the same root."""
+    v = np.asarray(v, dtype=np.float64)
+    norm = np.sqrt(np.asarray(beta, np.float64) + (v * v) @ np.asarray(gamma, np.float64).T)
+    return v * norm if inverse else v / norm
+
+
+def epilogue_general_vector(acc, p: Prepared, phi_vec) -> np.ndarray:
+    """The transition of Sec. general nonlinearities for a channel-coupled
+    activation (GDN / IGDN): z as in epilogue_general, then per pixel
+    u = clamp(round(phi(s_z z) / s_u)) with phi on the whole channel vector
+    (fp64, rounded half to even), then the input-side rescale."""
+    a = np.asarray(acc, dtype=np.int64) + p.b_int
+    t = p.M * a
+    v = transform_int(t, p.hb_out) if p.hb_out else t
+    z = np.clip(rshift_rne(v, p.n), -QMAX, QMAX)
+    u = np.clip(np.rint(phi_vec(p.s_z * z.astype(np.float64)) / p.s_u), -QMAX, QMAX).astype(np.int64)
     w = p.M_in * u
     w = transform_int(w, p.hb_next) if p.hb_next else w
     return np.clip(rshift_rne(w, p.n_in), -QMAX, QMAX).astype(np.int8)

@@ -16,7 +16,7 @@ _orig = {k: getattr(O, k) for k in ("sylvester", "transform_real", "transform_in
                                     "act_multiplier", "range_expansion_codes", "select_form",
                                     "epilogue_general", "phi", "paley1", "padded_transforms",
                                     "_jacobsthal", "conv_transpose_codes", "conv_transpose_real",
-                                    "depth_to_space", "affine_params", "conv_layer_affine")}
+                                    "depth_to_space", "affine_params", "conv_layer_affine", "gdn")}
 
 
 def _sylvester_bad(m):
@@ -194,7 +194,19 @@ def _affine_raw_padding(x_real, p):
     return (np.maximum(y, 0.0) if p.act == "relu" else y), s, z
 
 
+def _gdn_unsquared(v, beta, gamma, inverse=False):
+    v = np.asarray(v, dtype=np.float64)
+    norm = np.sqrt(np.asarray(beta, np.float64) + np.abs(v) @ np.asarray(gamma, np.float64).T)
+    return v * norm if inverse else v / norm
+
+
+def _igdn_divides(v, beta, gamma, inverse=False):
+    return _orig["gdn"](v, beta, gamma, False)
+
+
 MUTATIONS = {
+    "gdn_norm_unsquared": ("gdn", _gdn_unsquared),
+    "igdn_divides": ("gdn", _igdn_divides),
     "affine_zero_point_sign": ("affine_params", _affine_z_sign),
     "affine_zero_not_in_range": ("affine_params", _affine_no_zero_in_range),
     "affine_padding_raw_code": ("conv_layer_affine", _affine_raw_padding),

@@ -725,3 +725,45 @@ def test_dynamic_affine_layer_tracks_real_model_and_pads_with_centred_zero(form)
     assert (s0, z0) == (s, z) or form == "WH"
     if form == "DH":
         assert np.allclose(y0, y, atol=1e-9)
+
+
+# ------------------------------------------------------- GDN / IGDN (channel-coupled nonlinearities)
+
+def test_gdn_closed_forms():
+    """gamma = 0: v / sqrt(beta); diagonal gamma: elementwise v / sqrt(beta +
+    g v^2); IGDN inverts GDN when the normalization does not depend on v
+    (gamma = 0), and a single channel satisfies IGDN(GDN(v)) = v exactly in
+    closed form v / r * sqrt(beta + g (v / r)^2) with r = sqrt(beta + g v^2)."""
+    v = np.array([[0.5, -2.0, 3.0]])
+    beta = np.array([1.0, 4.0, 0.25])
+    assert np.allclose(O.gdn(v, beta, np.zeros((3, 3))), v / np.sqrt(beta))
+    g = np.diag([0.5, 1.0, 2.0])
+    assert np.allclose(O.gdn(v, beta, g), v / np.sqrt(beta + np.diag(g) * v * v))
+    assert np.allclose(O.gdn(O.gdn(v, beta, np.zeros((3, 3))), beta, np.zeros((3, 3)), inverse=True), v)
+    one = O.gdn(np.array([[2.0]]), [1.0], [[0.75]])
+    assert one[0, 0] == pytest.approx(2.0 / math.sqrt(1.0 + 0.75 * 4.0))
+    assert np.allclose(O.gdn(v, beta, g, inverse=True), v * np.sqrt(beta + np.diag(g) * v * v))
+
+
+@pytest.mark.parametrize("inverse", [False, True])
+def test_gdn_transition_tracks_real_model(inverse):
+    """A DH layer followed by GDN (or IGDN) through the two-step integer
+    transition stays close to the fp64 model gdn(conv(x))."""
+    rng = np.random.default_rng(9)
+    c = 64
+    x_real = np.maximum(I.activations((1, 7, 8, c), seed=130).astype(np.float64), 0)
+    w = I.weights(c, 3, 3, c, seed=131)
+    b = I.bias(c, seed=132)
+    beta = 1.0 + rng.random(c)
+    gamma = np.abs(rng.standard_normal((c, c))) * 0.01
+    phi_vec = lambda v: O.gdn(v, beta, gamma, inverse)
+    y = O.conv_real(x_real, w, b, 1, 1)
+    u = phi_vec(y)
+    s_x = O.symmetric_scale(O.transform_real(x_real, 64))
+    s_z, s_u = O.symmetric_scale(y), O.symmetric_scale(u)
+    p = O.prepare_layer(w, b, "DH", 64, 0, s_x, s_u, "igdn" if inverse else "gdn", 0, False, 1, 1,
+                        s_z=s_z, s_u=s_u)
+    op = O.quantize_act_f16(x_real.astype(np.float16), 64, s_x)
+    acc = O.conv_codes(op, p.w_int, 1, 1)
+    got = O.epilogue_general_vector(acc, p, phi_vec).astype(np.float64) * p.s_y
+    assert O.sqnr_db(u, got) > 24.0
