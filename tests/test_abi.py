@@ -239,3 +239,22 @@ def test_prepared_struct_mirror_matches_the_c_layout(tmp_path):
     assert ctypes.sizeof(H.PreparedStruct) == out[0]
     for f, off in zip(fields, out[1:]):
         assert getattr(H.PreparedStruct, f).offset == off, f
+
+
+@pytest.mark.parametrize("hb_out", [0, 16, 32, 64, 128])
+def test_chain_fusion_rule_matches_the_library(hb_out):
+    """synth.configs.fusable (used to plan chains) and the library's check of
+    a fused next-layer transform agree for every block pair."""
+    c = 128
+    d = H.make_desc(64, c, 1, 1, 0, "WH", hb_out=hb_out) if hb_out else H.make_desc(64, c, 1, 1, 0, "DH", hb_in=64)
+    w = np.zeros((c, 1, 1, 64), np.float32)
+    w[:, 0, 0, 0] = 0.5
+    for hb_next in (0, 16, 32, 64, 128):
+        ok = C.fusable(hb_out, hb_next)
+        try:
+            H.prepare_weights_host(d, w, None, 0.1, 0.1, "relu", hb_next)
+            lib_ok = True
+        except H.HatqError as e:
+            assert e.status == H.ERR_UNSUPPORTED
+            lib_ok = False
+        assert lib_ok == ok, (hb_out, hb_next)
