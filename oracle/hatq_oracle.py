@@ -654,28 +654,45 @@ def layer_operand(x, x_kind: str, s_in: float, form: str, hb_in: int, s_x: float
     raise ValueError(x_kind)
 
 
-def prepare_chain(layers, params, scales, plan, out_f32_last=False):
-    """layers: LayerSpec-like objects; params: [(w, b)]; scales: [{'s_x','s_out'}];
-    plan: per layer the fused next-layer DH block (0 = none)."""
+def transition_blocks(layers):
+    """Per layer l, the block of the input-side transform H~_in,l+1 that layer
+    l's transition applies after phi (Table integer_transitions): the next
+    layer's input block when it is DH (DH-to-DH, WH-to-DH), 0 when it is WH
+    or there is none (DH-to-WH, WH-to-WH, last layer). Every transition inside
+    a chain is one requantization with one round-shift
+    (Eq. integer_hadamard_transition), whatever the blocks are."""
+    out = []
+    for i in range(len(layers)):
+        nxt = layers[i + 1] if i + 1 < len(layers) else None
+        out.append(nxt.hb_in if nxt is not None and nxt.form == "DH" else 0)
+    return out
+
+
+def prepare_chain(layers, params, scales, out_f32_last=False):
+    """layers: LayerSpec-like objects; params: [(w, b)]; scales: [{'s_x','s_out'}]
+    (s_out: the scale of the next layer's operand, or of the chain output).
+    Each layer is prepared with the input-side block of its transition."""
+    hb_next = transition_blocks(layers)
     preps = []
     for i, (L, (w, b), sc) in enumerate(zip(layers, params, scales)):
         last = i == len(layers) - 1
         preps.append(prepare_layer(w, b, L.form, L.hb_in, L.hb_out, sc["s_x"], sc["s_out"],
-                                   L.act, plan[i], out_f32_last and last, L.stride, L.pad))
+                                   L.act, hb_next[i], out_f32_last and last, L.stride, L.pad))
     return preps
 
 
-def chain_forward(layers, preps, plan, x, x_kind, s_in):
-    """Run a chain on the oracle. Returns the list of per-layer outputs."""
+def chain_forward(layers, preps, x, x_kind, s_in):
+    """Run a chain on the oracle. The chain input enters its first layer through
+    layer_operand; every later layer consumes its producer's output as is (the
+    producer's transition already emitted the operand in the consumer's basis
+    and scale). Returns the list of per-layer outputs."""
     outs = []
     cur, kind, s_cur = x, x_kind, s_in
-    for i, (L, p) in enumerate(zip(layers, preps)):
+    for L, p in zip(layers, preps):
         op = layer_operand(cur, kind, s_cur, L.form, L.hb_in, p.s_x)
         y = conv_layer(op, p)
         outs.append(y)
-        fused = plan[i] != 0
-        cur, s_cur = y, p.s_y
-        kind = "operand" if (fused or (i + 1 < len(layers) and layers[i + 1].form == "WH")) else "i8"
+        cur, kind, s_cur = y, "operand", p.s_y
     return outs
 
 
@@ -848,12 +865,12 @@ def space_to_depth(x, r: int) -> np.ndarray:
     return x.reshape(n, h, r, w, r, c).transpose(0, 1, 3, 5, 2, 4).reshape(n, h, w, c * r * r)
 
 
-def calibrate_chain(layers, params, x_real, plan, first_wh_scale=None):
+def calibrate_chain(layers, params, x_real, first_wh_scale=None):
     """Static scales from the real-valued model (QAT-style frozen scales,
     Sec. quantization-aware training): per layer, s_x = max-abs of the
     operand in its quantizer's basis / 127, and s_out = the scale of what the
-    layer emits (the next operand when fused or next is WH, the
-    original-basis intermediate otherwise, or the final output)."""
+    layer emits: the next layer's operand (in the next layer's input basis,
+    i.e. after H_in,l+1 when the next layer is DH), or the chain output."""
     scales = []
     x = np.asarray(x_real, dtype=np.float64)
     reals = []
@@ -867,10 +884,11 @@ def calibrate_chain(layers, params, x_real, plan, first_wh_scale=None):
         reals.append((x, xn))
         scales.append({"s_x": float(np.float32(s_x))})
         x = xn
+    hb_next = transition_blocks(layers)
     for i, L in enumerate(layers):
         xn = reals[i][1]
-        if plan[i]:
-            s_out = symmetric_scale(transform_real(xn, plan[i]))
+        if hb_next[i]:
+            s_out = symmetric_scale(transform_real(xn, hb_next[i]))
         else:
             s_out = symmetric_scale(xn)
         scales[i]["s_out"] = float(np.float32(s_out))

@@ -4,9 +4,9 @@ blocks and the static per-layer DH/WH profile mask.
 A *chain* is a sequence of convolutions applied one after another; a *config*
 is a list of chains that share nothing but the GPU. Shapes are NHWC, weights
 OHWI. Nothing here computes any part of the quantization method; the only
-structural rule is which DH input transforms are produced inside the previous
-layer's epilogue (`plan_chain`), a property of the deployment that both the
-CUDA path and the oracle follow.
+structural rule is which input-side transform each layer's transition applies
+(`plan_chain`, read off Table integer_transitions for the CUDA path; the
+oracle derives the same from the layers on its own).
 """
 from __future__ import annotations
 
@@ -98,27 +98,15 @@ class ConfigSpec:
     calib_from: str = ""  # scales are taken from this config's calibration
 
 
-def fusable(hb_out: int, hb_next: int) -> bool:
-    """Whether the producer epilogue can apply the next layer's DH input
-    transform itself: at most one 128-wide transform, or both at most 64."""
-    if hb_out == 0 or hb_next == 0:
-        return max(hb_out, hb_next) <= 128
-    return max(hb_out, hb_next) <= 64
-
-
 def plan_chain(chain: ChainSpec):
-    """Per layer l, the block of the next layer's DH transform applied inside
-    layer l's epilogue (0 = none). Where the next layer is DH but the transform
-    cannot be fused, layer l emits original-basis INT8 codes and the next
-    layer starts with a separate transform + requantize pass."""
+    """Per layer l, the block of the next layer's DH input transform that layer
+    l's epilogue applies after phi (0 = none: the next layer is WH, or l is
+    the last layer). Table integer_transitions: DH-to-DH and WH-to-DH apply
+    H_in,l+1; DH-to-WH and WH-to-WH do not. The transition is always fused
+    into the producer, so every layer boundary inside a chain is one
+    requantization."""
     L = chain.layers
-    out = []
-    for i, lay in enumerate(L):
-        if i + 1 < len(L) and L[i + 1].form == DH and fusable(lay.hb_out, L[i + 1].hb_in):
-            out.append(L[i + 1].hb_in)
-        else:
-            out.append(0)
-    return out
+    return [L[i + 1].hb_in if i + 1 < len(L) and L[i + 1].form == DH else 0 for i in range(len(L))]
 
 
 def _cfg0():

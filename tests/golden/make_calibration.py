@@ -34,9 +34,8 @@ def main():
         for ch in cfg.chains:
             x = C.chain_input(ch)
             params = C.chain_params(ch)
-            plan = C.plan_chain(ch)
             first_wh = ch.s_in if (ch.layers[0].form == C.WH and ch.input_kind == "i8") else None
-            scales = O.calibrate_chain(ch.layers, params, real_input(ch, x), plan, first_wh)
+            scales = O.calibrate_chain(ch.layers, params, real_input(ch, x), first_wh)
             chains[ch.name] = scales
             print(name, ch.name, [(round(s["s_x"], 5), round(s["s_out"], 5)) for s in scales], flush=True)
         out["configs"][name] = chains

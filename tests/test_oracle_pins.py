@@ -350,22 +350,22 @@ def test_quantized_layer_approximates_real_layer(form):
 
 
 def test_chain_mixed_forms_tracks_real_model():
-    """A small DH/WH chain with fused and unfused transitions stays close to
-    the real-valued model (Table integer_transitions end to end)."""
-    from synth.configs import layer, plan_chain, ChainSpec
+    """A small DH/WH chain with every transition of Table integer_transitions
+    (WH-to-DH at 64 and 128 blocks, DH-to-WH) stays close to the real-valued
+    model end to end."""
+    from synth.configs import layer, ChainSpec
     layers = (layer("a", 16, 64, 3, 1, 1, "WH", "relu", hb_out=64),
               layer("b", 64, 64, 3, 2, 1, "DH", "relu", hb_in=64),
               layer("c", 64, 128, 3, 1, 1, "WH", "relu", hb_out=128),
               layer("d", 128, 32, 1, 1, 0, "DH", "none", hb_in=128))
     ch = ChainSpec("t", layers, 1, 12, 12, "i8", 0.05, 80, 81)
-    plan = plan_chain(ch)
-    assert plan == [64, 0, 0, 0]                        # WH(64)->DH(64) fused; WH(128)->DH(128) not
+    assert O.transition_blocks(layers) == [64, 0, 128, 0]
     x = I.activations_i8((1, 12, 12, 16), seed=80, s_in=0.05)
     params = [(I.weights(L.c_out, L.k, L.k, L.c_in, 90 + i), I.bias(L.c_out, 95 + i)) for i, L in enumerate(layers)]
     x_real = x.astype(np.float64) * float(np.float32(0.05))
-    scales = O.calibrate_chain(layers, params, x_real, plan)
-    preps = O.prepare_chain(layers, params, scales, plan)
-    outs = O.chain_forward(layers, preps, plan, x, "i8", 0.05)
+    scales = O.calibrate_chain(layers, params, x_real)
+    preps = O.prepare_chain(layers, params, scales)
+    outs = O.chain_forward(layers, preps, x, "i8", 0.05)
     ref = x_real
     for L, (w, b) in zip(layers, params):
         ref = O.conv_real(ref, w, b, L.stride, L.pad)
