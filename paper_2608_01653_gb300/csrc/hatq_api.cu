@@ -105,11 +105,6 @@ hatq_status check_desc(const hatq_conv_desc *d) {
     return HATQ_OK;
 }
 
-bool fusable(int hb_out, int hb_next) {
-    if (hb_out == 0 || hb_next == 0) return (hb_out > hb_next ? hb_out : hb_next) <= 128;
-    return hb_out <= 64 && hb_next <= 64;
-}
-
 hatq_status geometry(const hatq_conv_desc *d, int hb_next, Geometry *g) {
     // Packed reduction order. c_in % 16 == 0: (ky, kx, ci) with ci padded to a
     // multiple of 64 per tap. Otherwise (small c_in): kernel row ky holds the
@@ -205,10 +200,6 @@ hatq_status validate_prepare(const hatq_conv_desc *d, const float *w_ohwi, float
     if (hb_next != 0 && (!pow2(hb_next) || hb_next < 2 || hb_next > 128 || d->c_out % hb_next))
         return fail(HATQ_ERR_INVALID_ARG, "hb_next must be 0 or a power of two in 2..128 dividing c_out");
     if (out_f32 && hb_next) return fail(HATQ_ERR_INVALID_ARG, "a float32 output has no next-layer transform");
-    const int hb_out = d->form == HATQ_WH ? d->hb_out : 0;
-    if (!fusable(hb_out, hb_next))
-        return fail(HATQ_ERR_UNSUPPORTED, "output block %d and next-layer block %d cannot both be applied in the epilogue",
-                    hb_out, hb_next);
     return geometry(d, hb_next, g);
 }
 
@@ -576,10 +567,12 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     // of the reduction accumulating in region g & 1, then the ring of fp16
     // A-operand slots. Without drains the two epilogue warpgroups alternate
     // tiles (nbuf = 2); with drains both take every chunk, each for half of
-    // the columns, keeping int32 partials in registers (nbuf = 1).
+    // the columns, keeping int32 partials in registers (nbuf = 1). A
+    // 128-column transform group (n_t = 128) is always shared by both
+    // warpgroups, one half each (nbuf = 1).
     const bool drains = a.num_kb > a.chunk_kb;
     a.buf_cols = a.n_t;
-    a.nbuf = drains ? 1 : 2;
+    a.nbuf = (drains || g.G == 128) ? 1 : 2;
     a.tmem_cols = 512;
     a.a_col = 2 * a.n_t;
     a.seg = g.seg;
@@ -621,6 +614,9 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     a.const_off = (bar_bytes + table_bytes + 127) & ~127;
     a.win_off = a.const_off + const_bytes;
     const int smem_bytes = a.stages * a.stage_bytes + a.staging_bytes + 1024 + a.win_off + win_bytes;
+    // the exchange of a 128-wide next-layer transform uses the output tile: 2 x 128 rows x 64 bytes
+    if (g.G == 128 && L->hb_next == 128 && a.staging_bytes < 2 * kTileRows * 64)
+        return fail(HATQ_ERR_UNSUPPORTED, "output tile too small for the 128-wide transition exchange");
     if (smem_bytes > 227 * 1024 - 1024) return fail(HATQ_ERR_UNSUPPORTED, "shared memory budget exceeded (%d bytes)", smem_bytes);
     a.x = x;
     a.b_int = L->b_int;
@@ -707,6 +703,19 @@ hatq_status hatq_profile_range(const int8_t *x, int n, int h, int w, int c, int 
     a.maxima = maxima;
     cudaError_t e = hatq::launch_profile(a, expands, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "profiling launch");
+    return HATQ_OK;
+}
+
+hatq_status hatq_select_form(const uint8_t *expands, int n, int tau_num, int tau_den, int *form, int *expanded) {
+    if (!expands || !form) return fail(HATQ_ERR_INVALID_ARG, "null argument");
+    if (n < 1) return fail(HATQ_ERR_INVALID_ARG, "at least one profiled image is required");
+    if (tau_den < 1 || tau_num < 0 || tau_num > tau_den)
+        return fail(HATQ_ERR_INVALID_ARG, "tau_sel must be a fraction in [0, 1] with a positive denominator");
+    long long count = 0;
+    for (int k = 0; k < n; ++k) count += expands[k] != 0;
+    // p_l = count / n > tau_num / tau_den, cross-multiplied (no rounding)
+    *form = count * (long long)tau_den > (long long)n * tau_num ? HATQ_WH : HATQ_DH;
+    if (expanded) *expanded = (int)count;
     return HATQ_OK;
 }
 

@@ -423,61 +423,116 @@ __device__ __forceinline__ void epi_group(const EpiCtx &e, const ConvArgs &a, in
     }
 }
 
-// A 128-column group with exactly one 128-wide transform (H~_out or H~_next):
-// H~_128 [x_lo; x_hi] = [H~_64 (x_lo + x_hi); H~_64 (x_lo - x_hi)], evaluated
-// as two register-resident passes of 64 outputs each.
-__device__ __forceinline__ void epi_group128(const EpiCtx &e, const ConvArgs &a, int col) {
-    const bool pre_relu = a.act && a.hb_out == 0;     // phi before H~_next
-    const bool post_relu = a.act && a.hb_out != 0;    // phi after H~_out
-#pragma unroll 1
-    for (int pass = 0; pass < 2; ++pass) {
-        if (!a.out_f32) {
-            long long s[64];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                int v[16];
-                long long x[16];
-                load_acc16(e, col + 16 * q, v);
-                scale_i64(e, col + 16 * q, v, x);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) s[16 * q + i] = pre_relu ? relu(x[i]) : x[i];
-                load_acc16(e, col + 64 + 16 * q, v);
-                scale_i64(e, col + 64 + 16 * q, v, x);
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    const long long x1 = pre_relu ? relu(x[i]) : x[i];
-                    s[16 * q + i] = pass == 0 ? s[16 * q + i] + x1 : s[16 * q + i] - x1;
-                }
-            }
-            fwht_fixed<64, 64>(s);
-            if (post_relu) {
-#pragma unroll
-                for (int i = 0; i < 64; ++i) s[i] = relu(s[i]);
-            }
-            store_codes<64>(a, e.row, col + 64 * pass, s);
-        } else {
-            float s[64];
+// A 128-column group (n_t = 128, nbuf = 1) shared by the two epilogue
+// warpgroups: warpgroup wg produces outputs 64 wg .. 64 wg + 63 of the
+// transition of Eq. integer_hadamard_transition.
+//   before phi: p = H~_out (M (.) a) on this half. For hb_out = 128,
+//     H~_128 [t_lo; t_hi] = [H~_64 (t_lo + t_hi); H~_64 (t_lo - t_hi)]
+//     (both halves of the accumulator are read); smaller blocks lie inside
+//     the half.
+//   after phi: for hb_next = 128 the two halves u_0, u_1 of phi(p) are
+//     exchanged through shared memory (eight int64 per thread and round)
+//     and H~_128 [u_0; u_1] = [H~_64 (u_0 + u_1); H~_64 (u_0 - u_1)] gives
+//     this half; smaller blocks again lie inside the half.
+// One round-shift at the end, as in every other group. Every thread of both
+// warpgroups runs the integer path with its exchange barriers, also after an
+// abort (ok false: the values are then meaningless but stay in this CTA's
+// tensor and shared memory, and the copy-out is skipped), so the named
+// barrier always completes.
+__device__ __forceinline__ void epi_split128(const EpiCtx &e, const ConvArgs &a, int wg, bool ok, uint8_t *xbuf,
+                                             int row) {
+    const int half = 64 * wg;
+    if (a.out_f32) {
+        if (!ok) return;
+        float p[64];
+        if (a.hb_out == 128) {
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
                 int v[16];
                 float x[16];
-                load_acc16(e, col + 16 * q, v);
-                scale_f32(e, col + 16 * q, v, x);
+                load_acc16(e, 16 * q, v);
+                scale_f32(e, 16 * q, v, x);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) s[16 * q + i] = x[i];
-                load_acc16(e, col + 64 + 16 * q, v);
-                scale_f32(e, col + 64 + 16 * q, v, x);
+                for (int i = 0; i < 16; ++i) p[16 * q + i] = x[i];
+                load_acc16(e, 64 + 16 * q, v);
+                scale_f32(e, 64 + 16 * q, v, x);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) s[16 * q + i] = pass == 0 ? s[16 * q + i] + x[i] : s[16 * q + i] - x[i];
+                for (int i = 0; i < 16; ++i) p[16 * q + i] = wg ? p[16 * q + i] - x[i] : p[16 * q + i] + x[i];
             }
-            fwht_fixed<64, 64>(s);
-            if (post_relu || pre_relu) {
+            fwht_fixed<64, 64>(p);
+        } else {
 #pragma unroll
-                for (int i = 0; i < 64; ++i) s[i] = relu(s[i]);
+            for (int q = 0; q < 4; ++q) {
+                int v[16];
+                load_acc16(e, half + 16 * q, v);
+                scale_f32(e, half + 16 * q, v, p + 16 * q);
             }
-            store_f32<64>(e.gout, col + 64 * pass, s);
+            if (a.hb_out) fwht<64>(p, a.hb_out);
         }
+        if (a.act) {
+#pragma unroll
+            for (int i = 0; i < 64; ++i) p[i] = relu(p[i]);
+        }
+        store_f32<64>(e.gout, half, p);
+        return;
     }
+    long long p[64];
+    if (a.hb_out == 128) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            int v[16];
+            long long x[16];
+            load_acc16(e, 16 * q, v);
+            scale_i64(e, 16 * q, v, x);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) p[16 * q + i] = x[i];
+            load_acc16(e, 64 + 16 * q, v);
+            scale_i64(e, 64 + 16 * q, v, x);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) p[16 * q + i] = wg ? p[16 * q + i] - x[i] : p[16 * q + i] + x[i];
+        }
+        fwht_fixed<64, 64>(p);
+    } else {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            int v[16];
+            load_acc16(e, half + 16 * q, v);
+            scale_i64(e, half + 16 * q, v, p + 16 * q);
+        }
+        if (a.hb_out) fwht<64>(p, a.hb_out);
+    }
+    if (a.act) {
+#pragma unroll
+        for (int i = 0; i < 64; ++i) p[i] = relu(p[i]);
+    }
+    if (a.hb_next == 128) {
+        // [warpgroup][pair k][row] in 16-byte units: a warp's accesses are 512 contiguous bytes
+        int4 *mine = reinterpret_cast<int4 *>(xbuf) + wg * 512 + row;
+        const int4 *theirs = reinterpret_cast<const int4 *>(xbuf) + (wg ^ 1) * 512 + row;
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const long long u0 = p[8 * r + 2 * k], u1 = p[8 * r + 2 * k + 1];
+                mine[k * 128] = make_int4((int)u0, (int)(u0 >> 32), (int)u1, (int)(u1 >> 32));
+            }
+            asm volatile("bar.sync 4, 256;" ::: "memory");
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int4 v = theirs[k * 128];
+                const long long o0 = (long long)(((unsigned long long)(uint32_t)v.y << 32) | (uint32_t)v.x);
+                const long long o1 = (long long)(((unsigned long long)(uint32_t)v.w << 32) | (uint32_t)v.z);
+                const int i0 = 8 * r + 2 * k;
+                p[i0] = wg ? o0 - p[i0] : p[i0] + o0;               // u_0 - u_1 on the upper half, u_0 + u_1 on the lower
+                p[i0 + 1] = wg ? o1 - p[i0 + 1] : p[i0 + 1] + o1;
+            }
+            asm volatile("bar.sync 4, 256;" ::: "memory");
+        }
+        fwht_fixed<64, 64>(p);
+    } else if (a.hb_next) {
+        fwht<64>(p, a.hb_next);
+    }
+    store_codes<64>(a, e.row, half, p);
 }
 
 // ------------------------------------------------------------------ kernel
@@ -906,7 +961,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int k = 0; k < 4; ++k)
 #pragma unroll
                     for (int i = 0; i < 32; ++i) part[k][i] = 0u;
-                if (ok) {
                 EpiCtx e;
                 e.b_int = cb + n0;
                 e.mult = cb + a.co + n0;
@@ -921,13 +975,17 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (oy < a.ho && ox < a.wo)
                         e.gout = static_cast<float *>(a.y) + (((long long)img * a.ho + oy) * a.wo + ox) * a.co + n0;
                 }
-                int gi = 0;
-                for (int col = 0; col < a.n_t; col += G, ++gi) {
-                    if (nbuf == 1 && (gi & 1) != wg) continue;
-                    if (G == 32) epi_group<32>(e, a, col);
-                    else if (G == 64) epi_group<64>(e, a, col);
-                    else epi_group128(e, a, col);
-                }
+                if (G == 128) {
+                    // n_t == 128, nbuf == 1: the warpgroups share the group; the shared-memory
+                    // output tile is free until the codes are stored and serves as the exchange buffer
+                    epi_split128(e, a, wg, ok, stage_tile, row);
+                } else if (ok) {
+                    int gi = 0;
+                    for (int col = 0; col < a.n_t; col += G, ++gi) {
+                        if (nbuf == 1 && (gi & 1) != wg) continue;
+                        if (G == 32) epi_group<32>(e, a, col);
+                        else epi_group<64>(e, a, col);
+                    }
                 }
                 tc_fence_before();
                 mbar_arrive(acc_empty(reg));           // TMEM reads of this region are complete

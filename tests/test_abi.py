@@ -45,6 +45,65 @@ def test_profile_range_checks_arguments_on_the_host(lib):
     assert "null" in H.last_error()
 
 
+def test_select_form_decides_exactly(lib):
+    """Eq. layerwise_hadamard_selection through the C ABI: WH iff p_l > tau_sel
+    (strict), with p_l the exact fraction of expanding images."""
+    from fractions import Fraction
+    assert H.select_form([1, 1, 1, 1, 0]) == ("DH", Fraction(4, 5))          # p_l = tau_sel: not above it
+    assert H.select_form([1] * 5) == ("WH", Fraction(1))
+    assert H.select_form([1] * 81 + [0] * 19) == ("WH", Fraction(81, 100))
+    assert H.select_form([0, 1], tau=(1, 4)) == ("WH", Fraction(1, 2))
+    assert H.select_form([0, 0, 0]) == ("DH", Fraction(0))
+    assert H.select_form(np.array([0, 7, 255], np.uint8)) == ("DH", Fraction(2, 3))  # nonzero means expands
+    for ind in ([1, 0, 1, 1, 1, 1], [1] * 9 + [0], [0] * 7, [1, 1, 1, 1, 1, 0, 0]):
+        form, p = H.select_form(ind)
+        assert (form, p) == (O.select_form(O.expansion_probability(ind)), O.expansion_probability(ind))
+    for bad in (([], (4, 5)), ([1], (6, 5)), ([1], (1, 0)), ([1], (-1, 5))):
+        with pytest.raises(H.HatqError) as e:
+            H.select_form(*bad)
+        assert e.value.status == H.ERR_INVALID_ARG
+
+
+class _FakeLayer:
+    """The attributes the binding's argument checks read from a prepared layer."""
+    c_in, out_f32 = 64, False
+
+    @staticmethod
+    def out_shape(n, h, w):
+        return (n, h, w, 32)
+
+
+@pytest.mark.parametrize("call", ["layer", "layer_noalloc", "conv2d_i8"])
+def test_binding_rejects_mismatched_tensors_before_the_library(call):
+    """Tensors that do not match the layer (channels, dtype for the input kind,
+    layout, output shape or dtype) raise ValueError in the binding, before any
+    library call could read or write past them."""
+    import torch
+    L = _FakeLayer()
+    fn = getattr(H, call)
+
+    def go(x, kind=H.IN_I8, y=None):
+        return fn(x, y=y, L=L) if call == "conv2d_i8" else fn(x, kind, 0.05, L, y=y)
+    x8 = torch.zeros((1, 4, 4, 64), dtype=torch.int8)
+    with pytest.raises(ValueError, match="channels"):
+        go(torch.zeros((1, 4, 4, 48), dtype=torch.int8))
+    with pytest.raises(ValueError, match="int8"):
+        go(torch.zeros((1, 4, 4, 64), dtype=torch.float16))
+    if call != "conv2d_i8":
+        with pytest.raises(ValueError, match="float16"):
+            go(x8, kind=H.IN_F16)
+    with pytest.raises(ValueError, match="contiguous"):
+        go(torch.zeros((1, 4, 64, 4), dtype=torch.int8).permute(0, 1, 3, 2))
+    with pytest.raises(ValueError, match="shape"):
+        go(x8, y=torch.zeros((1, 4, 4, 64), dtype=torch.int8))
+    with pytest.raises(ValueError, match="int8"):
+        go(x8, y=torch.zeros((1, 4, 4, 32), dtype=torch.float32))
+    with pytest.raises(ValueError, match="4-D"):
+        go(torch.zeros((4, 4, 64), dtype=torch.int8))
+    with pytest.raises(ValueError, match="CUDA"):
+        go(x8)
+
+
 def test_version_and_last_error(lib):
     assert H.version() == 1
     d = H.make_desc(64, 48, 3, 1, 1, "DH", hb_in=64)          # c_out not a multiple of 32
@@ -84,12 +143,9 @@ def test_invalid_descriptors_rejected(bad):
     assert e.value.status in (H.ERR_INVALID_ARG, H.ERR_UNSUPPORTED)
 
 
-def test_prepare_rejects_unfusable_pair_and_bad_scales():
+def test_prepare_rejects_bad_scales_and_float_output_with_a_next_transform():
     d = H.make_desc(64, 128, 3, 1, 1, "WH", hb_out=128)
     w = np.zeros((128, 3, 3, 64), np.float32)
-    with pytest.raises(H.HatqError) as e:
-        H.prepare_weights_host(d, w, None, 0.1, 0.1, "relu", hb_next=128)
-    assert e.value.status == H.ERR_UNSUPPORTED
     with pytest.raises(H.HatqError):
         H.prepare_weights_host(d, w, None, -1.0, 0.1)
     with pytest.raises(H.HatqError):
@@ -214,6 +270,8 @@ def test_binding_constants_match_the_header():
               "HATQ_IN_I8": H.IN_I8, "HATQ_IN_F16": H.IN_F16}
     for name, value in expect.items():
         assert decl[name] == value, name
+    m = re.search(r"#define\s+HATQ_NOALLOC_MAX_BYTES\s+\((\d+)u\s*<<\s*(\d+)\)", text)
+    assert m and (int(m.group(1)) << int(m.group(2))) == H.NOALLOC_MAX_BYTES
 
 
 def test_prepared_struct_mirror_matches_the_c_layout(tmp_path):
@@ -242,19 +300,24 @@ def test_prepared_struct_mirror_matches_the_c_layout(tmp_path):
 
 
 @pytest.mark.parametrize("hb_out", [0, 16, 32, 64, 128])
-def test_chain_fusion_rule_matches_the_library(hb_out):
-    """synth.configs.fusable (used to plan chains) and the library's check of
-    a fused next-layer transform agree for every block pair."""
+def test_every_transition_block_pair_is_accepted(hb_out):
+    """Every WH output block and next-layer DH input block of Table
+    integer_transitions up to 128 is one fused transition in the library
+    (the paper's single requantization, Eq. integer_hadamard_transition)."""
     c = 128
     d = H.make_desc(64, c, 1, 1, 0, "WH", hb_out=hb_out) if hb_out else H.make_desc(64, c, 1, 1, 0, "DH", hb_in=64)
     w = np.zeros((c, 1, 1, 64), np.float32)
     w[:, 0, 0, 0] = 0.5
     for hb_next in (0, 16, 32, 64, 128):
-        ok = C.fusable(hb_out, hb_next)
-        try:
-            H.prepare_weights_host(d, w, None, 0.1, 0.1, "relu", hb_next)
-            lib_ok = True
-        except H.HatqError as e:
-            assert e.status == H.ERR_UNSUPPORTED
-            lib_ok = False
-        assert lib_ok == ok, (hb_out, hb_next)
+        got = H.prepare_weights_host(d, w, None, 0.1, 0.1, "relu", hb_next)
+        ref = O.prepare_layer(w, None, "WH" if hb_out else "DH", 0 if hb_out else 64, hb_out, 0.1, 0.1, "relu",
+                              hb_next, False, 1, 0)
+        assert got.shift == ref.n and np.array_equal(got.mult.astype(np.int64), ref.M), (hb_out, hb_next)
+
+
+def test_chain_plan_is_the_oracles_transition_plan():
+    """The CUDA path's chain planner (synth.configs.plan_chain) and the
+    oracle's own reading of Table integer_transitions agree on every chain."""
+    for cfg in C.CONFIGS.values():
+        for ch in cfg.chains:
+            assert C.plan_chain(ch) == O.transition_blocks(ch.layers), ch.name

@@ -142,13 +142,23 @@ LAYER_CASES = [
     ("dh3x3_k1728_drain", C.layer("a", 192, 192, 3, 1, 1, "DH", "relu", hb_in=64), (2, 13, 37), 64),
     ("dh5x5s2_ragged", C.layer("a", 192, 192, 5, 2, 2, "DH", "none", hb_in=64), (3, 19, 45), 0),
     ("wh5x5s2_c3_gather", C.layer("a", 3, 192, 5, 2, 2, "WH", "relu", hb_out=64), (1, 40, 50), 64),
-    ("wh3x3_hb128_twopass", C.layer("a", 224, 128, 3, 1, 1, "WH", "relu", hb_out=128), (1, 12, 20), 0),
+    ("wh3x3_hb128_split", C.layer("a", 224, 128, 3, 1, 1, "WH", "relu", hb_out=128), (1, 12, 20), 0),
     ("dh3x3_c32_box", C.layer("a", 32, 224, 3, 1, 1, "DH", "relu", hb_in=32), (2, 9, 17), 0),
-    ("dh3x3_next128_twopass", C.layer("a", 128, 128, 3, 1, 1, "DH", "relu", hb_in=128), (1, 10, 33), 128),
+    ("dh3x3_next128_split", C.layer("a", 128, 128, 3, 1, 1, "DH", "relu", hb_in=128), (1, 10, 33), 128),
     ("dh3x3_c640_n160", C.layer("a", 320, 640, 3, 1, 1, "DH", "relu", hb_in=64), (1, 6, 9), 0),
     ("wh1x1_c640", C.layer("a", 640, 640, 1, 1, 0, "WH", "none", hb_out=128), (1, 7, 11), 0),
     ("dh3x3_next32", C.layer("a", 224, 128, 3, 1, 1, "DH", "relu", hb_in=32), (1, 8, 8), 32),
     ("wh3x3_fused_16", C.layer("a", 64, 64, 3, 2, 1, "WH", "relu", hb_out=16), (1, 16, 24), 16),
+    # WH-to-DH transitions with a 128-wide transform on either side (Table integer_transitions):
+    # one requantization, the two epilogue warpgroups exchanging halves for the next transform
+    ("wh3x3_128_next128_drain", C.layer("a", 224, 128, 3, 1, 1, "WH", "relu", hb_out=128), (2, 11, 21), 128),
+    ("wh1x1_128_next128_nodrain", C.layer("a", 128, 128, 1, 1, 0, "WH", "relu", hb_out=128), (1, 13, 29), 128),
+    ("wh3x3_128_next64", C.layer("a", 64, 128, 3, 1, 1, "WH", "relu", hb_out=128), (1, 9, 14), 64),
+    ("wh3x3_64_next128", C.layer("a", 64, 128, 3, 1, 1, "WH", "relu", hb_out=64), (1, 9, 14), 128),
+    ("wh3x3_32_next128", C.layer("a", 96, 128, 3, 2, 1, "WH", "relu", hb_out=32), (1, 17, 23), 128),
+    ("dh1x1_next128_nodrain", C.layer("a", 64, 128, 1, 1, 0, "DH", "relu", hb_in=64), (1, 12, 12), 128),
+    ("wh3x3_c640_128_next128", C.layer("a", 320, 640, 3, 1, 1, "WH", "relu", hb_out=128), (1, 7, 10), 128),
+    ("wh5x5s2_c3_next128", C.layer("a", 3, 128, 5, 2, 2, "WH", "relu", hb_out=128), (1, 30, 44), 128),
 ]
 
 
@@ -243,8 +253,8 @@ def run_chain(H, ch, scales):
     chain = Chain(ch.layers, params, scales, plan, ch.out_f32)
     outs = chain.forward(dev(x), kind, ch.s_in)
     H.sync_status()
-    preps = O.prepare_chain(ch.layers, params, scales, plan, ch.out_f32)
-    refs = O.chain_forward(ch.layers, preps, plan, x, ch.input_kind, ch.s_in)
+    preps = O.prepare_chain(ch.layers, params, scales, ch.out_f32)
+    refs = O.chain_forward(ch.layers, preps, x, ch.input_kind, ch.s_in)
     return [host(o) for o in outs], refs
 
 
