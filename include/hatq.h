@@ -285,6 +285,20 @@ hatq_status hatq_sync_status(hatq_stream stream);
 hatq_status hatq_profile_range(const int8_t *x, int n, int h, int w, int c, int hb, int32_t *maxima,
                                uint8_t *expands, hatq_stream stream);
 
+/* Layer-wise strategy selection (Eqs. hadamard_sensitivity,
+ * layerwise_hadamard_selection) from the per-image indicators of
+ * hatq_profile_range.
+ *   expands   HOST uint8 [n], nonzero where image k's range expands; n >= 1.
+ *   tau_num / tau_den   the threshold tau_sel as an exact fraction
+ *             (0 <= tau_num <= tau_den, tau_den > 0; the paper uses 4 / 5).
+ *   form      out: HATQ_WH when p_l > tau_sel (strict), else HATQ_DH, with
+ *             p_l = (number of expanding images) / n decided exactly in
+ *             integers: count * tau_den > n * tau_num.
+ *   expanded  out (may be NULL): the number of expanding images, so that
+ *             p_l = *expanded / n.
+ * Host only, synchronous; HATQ_ERR_INVALID_ARG for a bad argument. */
+hatq_status hatq_select_form(const uint8_t *expands, int n, int tau_num, int tau_den, int *form, int *expanded);
+
 /* Failure-detection self test (the paper has no counterpart): launches one
  * thread that waits, through the same bounded mbarrier wait the convolution
  * pipeline uses, on a barrier nothing arrives at. The wait expires after

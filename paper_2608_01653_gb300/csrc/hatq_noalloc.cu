@@ -12,6 +12,8 @@
 // the GPU (different streams without ordering between them) race on it.
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include "hatq.h"
 #include "hatq_internal.h"
 
@@ -21,17 +23,23 @@ static __device__ __align__(256) int8_t g_noalloc_operand[HATQ_NOALLOC_MAX_BYTES
 
 // Device address of g_noalloc_operand per device, looked up once with that
 // device current (in host code the symbol itself is only a host-side stand-in).
-int8_t *g_operand_ptr[64] = {nullptr};
+// Host threads may call concurrently: each slot is an atomic, and two threads
+// that race on the first lookup store the same address. The cached address
+// belongs to the device's primary context: after cudaDeviceReset() it is
+// stale, as is every other device pointer the caller held.
+std::atomic<int8_t *> g_operand_ptr[64];
 
 hatq_status operand_buffer(int8_t **out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return HATQ_ERR_CUDA;
-    if (!g_operand_ptr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_noalloc_operand) != cudaSuccess || p == nullptr) return HATQ_ERR_CUDA;
-        g_operand_ptr[dev] = static_cast<int8_t *>(p);
+    int8_t *p = g_operand_ptr[dev].load(std::memory_order_acquire);
+    if (!p) {
+        void *q = nullptr;
+        if (cudaGetSymbolAddress(&q, g_noalloc_operand) != cudaSuccess || q == nullptr) return HATQ_ERR_CUDA;
+        p = static_cast<int8_t *>(q);
+        g_operand_ptr[dev].store(p, std::memory_order_release);
     }
-    *out = g_operand_ptr[dev];
+    *out = p;
     return HATQ_OK;
 }
 

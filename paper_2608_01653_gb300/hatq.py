@@ -81,6 +81,8 @@ def load(build: bool = True) -> ctypes.CDLL:
             "hatq_sync_status": (_I, [_P]),
             "hatq_selftest_wait": (_I, [ctypes.c_ulonglong, _P]),
             "hatq_profile_range": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P]),
+            "hatq_select_form": (_I, [_P, _I, _I, _I, ctypes.POINTER(_I), ctypes.POINTER(_I)]),
+            "hatq_layer_noalloc": (_I, [_P, _I, _F, _I, _I, _I, ctypes.POINTER(PreparedStruct), _P, _P]),
             "hatq_version": (_I, []),
         }
         for name, (res, args) in sig.items():
@@ -270,11 +272,59 @@ def prepare_weights_general_host(desc: ConvDesc, w_ohwi, bias, s_x, s_z, s_u, s_
     return HostGeneral(w_i8.reshape(desc.c_out, -1), b_int, mult, s_w, shift.value, mult_in.value, shift_in.value, lut)
 
 
+_KIND_DTYPE = {IN_OPERAND: "int8", IN_I8: "int8", IN_F16: "float16"}
+
+
+def _check_tensor(t, what, dtype=None, shape=None):
+    """Shape, dtype, layout and device of a tensor handed to the library: the
+    entry points read and write exactly the elements these describe."""
+    import torch
+    if not isinstance(t, torch.Tensor):
+        raise ValueError(f"{what} must be a torch tensor")
+    if dtype is not None and t.dtype != getattr(torch, dtype):
+        raise ValueError(f"{what} must be {dtype}, got {t.dtype}")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{what} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+    if not t.is_contiguous():
+        raise ValueError(f"{what} must be contiguous (NHWC, C innermost)")
+
+
+def _check_cuda(*named):
+    for what, t in named:
+        if t is not None and not t.is_cuda:
+            raise ValueError(f"{what} must be on a CUDA device")
+
+
+def _check_layer_io(x, x_kind, L, y=None, scratch=None):
+    """The input of a layer call (kind, dtype, 4-D NHWC with L.c_in channels)
+    and, when given, its output and scratch buffers."""
+    if x_kind not in _KIND_DTYPE:
+        raise ValueError(f"unknown input kind {x_kind}")
+    if getattr(x, "dim", lambda: 0)() != 4:
+        raise ValueError("x must be a 4-D NHWC tensor")
+    n, h, w, c = x.shape
+    if c != L.c_in:
+        raise ValueError(f"x has {c} channels, the layer takes {L.c_in}")
+    _check_tensor(x, "x", _KIND_DTYPE[x_kind])
+    if y is not None:
+        _check_tensor(y, "y", "float32" if L.out_f32 else "int8", L.out_shape(n, h, w))
+    if scratch is not None:
+        _check_tensor(scratch, "scratch", "int8")
+    _check_cuda(("x", x), ("y", y), ("scratch", scratch))
+    return n, h, w, c
+
+
 def quantize_act(x, x_kind, s_in, hb, s_out, y=None, s_used=None, workspace=None, stream=None):
     """hatq_quantize_act on a CUDA NHWC tensor (int8 codes or fp16 values).
     s_out <= 0 selects the dynamic mode (s_used: 1-element float32 CUDA tensor)."""
     torch = _torch()
+    if x_kind not in (IN_I8, IN_F16) or getattr(x, "dim", lambda: 0)() != 4:
+        raise ValueError("x must be a 4-D NHWC tensor of kind IN_I8 or IN_F16")
+    _check_tensor(x, "x", _KIND_DTYPE[x_kind])
     n, h, w, c = x.shape
+    if y is not None:
+        _check_tensor(y, "y", "int8", (n, h, w, c))
+    _check_cuda(("x", x), ("y", y))
     if y is None:
         y = torch.empty((n, h, w, c), dtype=torch.int8, device=x.device)
     if s_out <= 0:
@@ -289,10 +339,8 @@ def quantize_act(x, x_kind, s_in, hb, s_out, y=None, s_used=None, workspace=None
 
 def conv2d_i8(x, L: PreparedLayer, y=None, stream=None):
     """hatq_conv2d_i8: convolution + fused requantize epilogue on the INT8 operand x (NHWC)."""
+    n, h, w, c = _check_layer_io(x, IN_OPERAND, L, y)
     torch = _torch()
-    n, h, w, c = x.shape
-    if c != L.c_in:
-        raise ValueError("channel mismatch")
     if y is None:
         y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32 if L.out_f32 else torch.int8, device=x.device)
     _check(load().hatq_conv2d_i8(_ptr(x), n, h, w, ctypes.byref(L.struct), _ptr(y), _stream(stream)))
@@ -301,8 +349,8 @@ def conv2d_i8(x, L: PreparedLayer, y=None, stream=None):
 
 def layer(x, x_kind, s_in, L: PreparedLayer, y=None, scratch=None, stream=None):
     """hatq_layer: input transform/quantize (when needed) + conv in one call."""
+    n, h, w, c = _check_layer_io(x, x_kind, L, y, scratch)
     torch = _torch()
-    n, h, w, c = x.shape
     if y is None:
         y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32 if L.out_f32 else torch.int8, device=x.device)
     nbytes = 0
@@ -337,19 +385,16 @@ def profile_range(x, hb: int, stream=None):
     return maxima, expands
 
 
-def expansion_probability(expands):
-    """p_l: the fraction of profiled images whose range expands (exact)."""
+def select_form(expands, tau=(4, 5)):
+    """hatq_select_form: the DH/WH decision of Eq. layerwise_hadamard_selection
+    from the per-image indicators (host array or tensor) and tau_sel given as
+    (numerator, denominator). Returns (form 'DH' or 'WH', p_l as a Fraction)."""
     from fractions import Fraction
-    vals = [int(v) for v in (expands.tolist() if hasattr(expands, "tolist") else expands)]
-    if not vals:
-        raise ValueError("no profiled images")
-    return Fraction(sum(vals), len(vals))
-
-
-def select_form(p, tau=0.8) -> str:
-    """pi_l: WH when p_l > tau_sel, else DH."""
-    from fractions import Fraction
-    return "WH" if Fraction(p) > Fraction(str(tau)) else "DH"
+    e = np.ascontiguousarray(expands.cpu().numpy() if hasattr(expands, "cpu") else expands, dtype=np.uint8).ravel()
+    form, count = ctypes.c_int(), ctypes.c_int()
+    _check(load().hatq_select_form(e.ctypes.data if e.size else None, int(e.size), int(tau[0]), int(tau[1]),
+                                   ctypes.byref(form), ctypes.byref(count)))
+    return ("WH" if form.value == WH else "DH"), Fraction(count.value, int(e.size))
 
 
 def selftest_wait(limit_cycles: int, stream=None):
@@ -366,14 +411,12 @@ def layer_noalloc(x, x_kind, s_in, L: PreparedLayer, y=None, stream=None):
     """hatq_layer_noalloc: hatq_layer for callers that cannot allocate device
     memory; the staged INT8 operand lives in the library's fixed device array
     (at most HATQ_NOALLOC_MAX_BYTES bytes, shared by all calls)."""
+    n, h, w, c = _check_layer_io(x, x_kind, L, y)
     torch = _torch()
-    fn = load().hatq_layer_noalloc
-    fn.restype = _I
-    fn.argtypes = [_P, _I, _F, _I, _I, _I, ctypes.POINTER(PreparedStruct), _P, _P]
-    n, h, w, c = x.shape
     if y is None:
         y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32 if L.out_f32 else torch.int8, device=x.device)
-    _check(fn(_ptr(x), int(x_kind), float(s_in), n, h, w, ctypes.byref(L.struct), _ptr(y), _stream(stream)))
+    _check(load().hatq_layer_noalloc(_ptr(x), int(x_kind), float(s_in), n, h, w, ctypes.byref(L.struct), _ptr(y),
+                                     _stream(stream)))
     return y
 
 

@@ -30,9 +30,8 @@ def _check(H, x, hb):
     got = maxima.cpu().numpy()
     assert np.array_equal(got[:, 0], mx) and np.array_equal(got[:, 1], mh)
     assert np.array_equal(expands.cpu().numpy(), ind)
-    assert H.expansion_probability(expands.cpu()) == O.expansion_probability(ind)
     p = O.expansion_probability(ind)
-    assert H.select_form(p) == O.select_form(p)
+    assert H.select_form(expands) == (O.select_form(p), p)          # Eq. layerwise_hadamard_selection, C ABI
     return ind
 
 
