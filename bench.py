@@ -52,9 +52,10 @@ def parse():
     p.add_argument("--steps", type=int, default=10)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--workload", default="cfg4", choices=["cfg4", "cfg2", "cfg1", "fwht", "profile"],
+    p.add_argument("--workload", default="cfg4", choices=["cfg4", "cfg2", "cfg1", "fwht", "profile", "int8mm"],
                    help="fwht: the INT8 transform+requantize pass alone on the config-4 ga2 input; "
-                        "profile: the range-expansion profiling pass on the same tensor")
+                        "profile: the range-expansion profiling pass on the same tensor; "
+                        "int8mm: torch._int_mm 8192^3, the library INT8 GEMM as a reference point")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--layer", default="", help="time one layer of the config-4 chains (e.g. ga2, h1, s0a)")
@@ -150,10 +151,9 @@ def oracle_sample(cfg, scales, threads=None, hw=CPU_SAMPLE_HW, latent=CPU_SAMPLE
         sub = ch.with_batch(1, h, w, ch.input_seed)
         x = C.chain_input(sub)
         params = C.chain_params(ch)
-        plan = C.plan_chain(ch)
-        preps = O.prepare_chain(ch.layers, params, scales[ch.name], plan, ch.out_f32)
+        preps = O.prepare_chain(ch.layers, params, scales[ch.name], ch.out_f32)
         t0 = time.perf_counter()
-        O.chain_forward(ch.layers, preps, plan, x, ch.input_kind, ch.s_in)
+        O.chain_forward(ch.layers, preps, x, ch.input_kind, ch.s_in)
         t_total += time.perf_counter() - t0
         ops += 2 * sub.macs()
         if ch.name == "analysis":
@@ -165,7 +165,7 @@ def run_reference(args, cfg, scales):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
-    for _ in range(args.warmup if args.warmup < 1 else 1):
+    for _ in range(args.warmup):
         oracle_sample(cfg, scales, hw=REF_SAMPLE_HW, latent=REF_SAMPLE_LATENT)
     times = []
     frac = ops = threads = None
@@ -274,23 +274,47 @@ def run_layer_mode(args, cfg, scales):
     raise SystemExit(f"unknown layer {args.layer}")
 
 
-def run_fwht_mode(args):
+def fwht_pass(batch, steps, warmup, device="cuda"):
     """The INT8-entry transform + requantize pass (hb 64) on an NHWC tensor
-    shaped like the config-4 ga2 input: 1 byte read + 1 byte written per element."""
+    shaped like the config-4 ga2 input (8 x 1080 x 1920 x 192 at batch 8,
+    3.2 GB, larger than L2): 1 byte read + 1 byte written per element. Returns
+    (ms per pass, algorithmic bytes per pass, shape)."""
     import torch
     from paper_2608_01653_gb300 import hatq as H
-    H.load()
-    shape = (args.batch, 1080, 1920, 192)
-    x = torch.from_numpy(I.uniform_codes(shape, seed=9)).cuda()
+    shape = (batch, 1080, 1920, 192)
+    g = torch.Generator(device=device)
+    g.manual_seed(9)
+    x = torch.randint(-127, 128, shape, dtype=torch.int8, device=device, generator=g)
     y = torch.empty_like(x)
-    ms = time_events(lambda: H.quantize_act(x, H.IN_I8, 0.05, 64, 0.07, y=y), args.steps, args.warmup)
+    ms = time_events(lambda: H.quantize_act(x, H.IN_I8, 0.05, 64, 0.07, y=y), steps, warmup)
     H.sync_status()
-    nbytes = 2 * x.numel()
+    return ms, 2 * x.numel(), shape
+
+
+def run_fwht_mode(args):
+    from paper_2608_01653_gb300 import hatq as H
+    H.load()
+    ms, nbytes, shape = fwht_pass(args.batch, args.steps, args.warmup)
     peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
     peak = peaks.get("hbm_gbs", FALLBACK_HBM_GBS)
     gbs = nbytes / (ms / 1000) / 1e9
     print(json.dumps({"mode": "fwht", "shape": list(shape), "hb": 64, "ms": ms, "GB/s": gbs, "peak_hbm_gbs": peak,
                       "frac": gbs / peak}), flush=True)
+
+
+def run_int8mm_mode(args):
+    """torch._int_mm (the library INT8 GEMM, int32 output) on 8192^3, CUDA
+    events: the measured INT8 tensor-core reference point of this GPU."""
+    import torch
+    n = 8192
+    a = torch.randint(-127, 128, (n, n), dtype=torch.int8, device="cuda")
+    b = torch.randint(-127, 128, (n, n), dtype=torch.int8, device="cuda")
+    ms = time_events(lambda: torch._int_mm(a, b), args.steps, args.warmup)
+    af = a.to(torch.float16)
+    bf = b.to(torch.float16)
+    ms16 = time_events(lambda: torch.matmul(af, bf), args.steps, args.warmup)
+    print(json.dumps({"mode": "int8mm", "n": n, "int8_ms": ms, "int8_tops": 2 * n ** 3 / (ms / 1000) / 1e12,
+                      "f16_ms": ms16, "f16_tflops": 2 * n ** 3 / (ms16 / 1000) / 1e12}), flush=True)
 
 
 def run_profile_mode(args):
@@ -331,6 +355,9 @@ def main():
     if args.workload == "profile":
         run_profile_mode(args)
         return
+    if args.workload == "int8mm":
+        run_int8mm_mode(args)
+        return
 
     import torch
     from paper_2608_01653_gb300 import hatq as H
@@ -360,17 +387,17 @@ def main():
     macs_step = sum(c["spec"].macs() for c in chains)
     images_step = cfg.images
 
-    # conv launches of one step with their algorithmic flops, timed by event pairs
+    # conv launches of one step, each timed by an event pair on the launching stream
     def step(record=None):
-        for c in chains:
+        for ci, c in enumerate(chains):
             chain, ch = c["chain"], c["spec"]
             kinds = chain.input_kinds(c["kind"], ch.s_in)
             cur = c["x_dev"]
             n, h, w = ch.n, ch.h, ch.w
-            for i, (P, L) in enumerate(zip(chain.prepared, ch.layers)):
+            for i, P in enumerate(chain.prepared):
                 k, s_in = kinds[i]
                 if H.layer_launches(k, s_in, P) > 1:
-                    hb = L.hb_in if L.form == "DH" else 1
+                    hb = ch.layers[i].hb_in if ch.layers[i].form == "DH" else 1
                     op = c["scratch"][: n * h * w * P.c_in].view(n, h, w, P.c_in)
                     H.quantize_act(cur, k, s_in, hb, P.s_x, y=op)
                     cur = op
@@ -381,7 +408,7 @@ def main():
                 H.conv2d_i8(cur, P, y=c["outs"][i])
                 if record is not None:
                     e1.record(stream)
-                    record.append((e0, e1, 2 * L.macs(n, h, w)))
+                    record.append((ci, i, e0, e1))
                 cur = c["outs"][i]
                 _, h, w, _ = c["outs"][i].shape
 
@@ -410,28 +437,106 @@ def main():
         dist.barrier()
     clocks = sampler.stop()
     H.sync_status()
-    conv_ms = sum(e0.elapsed_time(e1) for e0, e1, _ in records)
-    conv_flops = sum(f for _, _, f in records)
-    n_conv = len(records)
 
-    # --- end to end through the public API with host buffers
+    peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
+    tc_peak, tc_src = peaks.get("bf16_tflops"), "measured bf16 burst (fp16 operands run at the bf16 rate)"
+    if tc_peak is None:
+        tc_peak, tc_src = FALLBACK_BF16_TFLOPS, "fallback bf16"
+    hbm_peak, hbm_src = peaks.get("hbm_gbs"), "measured HBM copy"
+    if hbm_peak is None:
+        hbm_peak, hbm_src = FALLBACK_HBM_GBS, "fallback HBM"
+
+    # per layer: algorithmic flops (2 MACs of the unpadded reduction) and bytes
+    # (INT8 input + INT8 output + INT8 weights, each once); its roofline is the
+    # larger of the tensor-core and the HBM time
+    per_layer = {}
+    for ci, i, e0, e1 in records:
+        per_layer.setdefault((ci, i), []).append(e0.elapsed_time(e1))
+    layers = []
+    for (ci, i), times in sorted(per_layer.items()):
+        ch = chains[ci]["spec"]
+        L = ch.layers[i]
+        n, h, w = ch.shapes()[i]
+        ho, wo = L.out_hw(h, w)
+        flops = 2 * L.macs(n, h, w)
+        nbytes = n * h * w * L.c_in + n * ho * wo * L.c_out + L.c_out * L.k * L.k * L.c_in
+        lms = sum(times) / len(times)
+        t_tc, t_hbm = flops / (tc_peak * 1e12), nbytes / (hbm_peak * 1e9)
+        bound = "tensor" if t_tc >= t_hbm else "hbm"
+        layers.append({"layer": L.name, "chain": ch.name, "ms": lms, "bound": bound,
+                       "tflops": flops / (lms / 1000) / 1e12, "gbs": nbytes / (lms / 1000) / 1e9,
+                       "flops": flops, "bytes": nbytes, "frac": max(t_tc, t_hbm) * 1000 / lms})
+    conv_ms = sum(x["ms"] for x in layers)
+    conv_flops = sum(x["flops"] for x in layers)
+    n_conv = len(layers)
+    achieved = conv_flops / (conv_ms / 1000.0) / 1e12
+    traffic = None
+    prof = os.path.join(ROOT, "profiles", "conv_cfg4_traffic.json")
+    if os.path.exists(prof):
+        traffic = json.load(open(prof)).get("dram_bytes_per_launch")
+    roofline = {"bound": "tensor", "achieved": achieved, "peak": tc_peak, "unit": "TFLOP/s", "frac": achieved / tc_peak,
+                "traffic": traffic, "kernel": "hatq conv_kernel (tcgen05 kind::f16, exact INT8)",
+                "launches": n_conv, "avg_launch_ms": conv_ms / max(n_conv, 1), "peak_source": tc_src,
+                "note": "all conv launches of the step; per-layer bounds in roofline_layers"}
+
+    # the INT8-entry transform + requantize pass on the config-4 ga2-shaped input (not part of the step:
+    # every transition inside a chain is fused into its producer)
+    f_ms, f_bytes, f_shape = fwht_pass(8, max(5, args.steps), 3, dev)
+    roofline_fwht = {"bound": "hbm", "achieved": f_bytes / (f_ms / 1000) / 1e9, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": f_bytes / (f_ms / 1000) / 1e9 / hbm_peak, "ms": f_ms, "bytes": f_bytes,
+                     "shape": list(f_shape), "hb": 64, "peak_source": hbm_src,
+                     "kernel": "hatq act_quant_kernel (INT8 entry, int32 butterfly, 64-bit requantization)"}
+
+    # --- end to end through the public API (Chain.forward) with pinned host buffers: every step copies its
+    # inputs in and its chain outputs back. Two input and two output slots per chain; copies run on their own
+    # stream, so step k's copies overlap the compute of steps k - 1 and k + 1.
     e2e = None
     if not args.no_e2e:
-        def e2e_step():
-            for c in chains:
-                c["x_dev"].copy_(c["x_pin"], non_blocking=True)
-                c["chain"].forward(c["x_dev"], c["kind"], c["spec"].s_in, c["outs"], c["scratch"])
-                c["out_pin"].copy_(c["outs"][-1], non_blocking=True)
-        for _ in range(2):
-            e2e_step()
+        cstream = torch.cuda.Stream(dev)
+        for c in chains:
+            c["x_slots"] = [c["x_dev"], torch.empty_like(c["x_dev"])]
+            c["y_slots"] = [c["outs"][-1], torch.empty_like(c["outs"][-1])]
+            c["out_pins"] = [c["out_pin"], torch.empty_like(c["out_pin"]).pin_memory()]
+        ev = lambda: torch.cuda.Event()  # noqa: E731
+        x_free = [ev(), ev()]
+        y_free = [ev(), ev()]
+        for e in x_free + y_free:
+            e.record(stream)
+
+        def e2e_steps(k_steps):
+            for k in range(k_steps):
+                sl = k % 2
+                loaded = ev()
+                with torch.cuda.stream(cstream):
+                    cstream.wait_event(x_free[sl])
+                    for c in chains:
+                        c["x_slots"][sl].copy_(c["x_pin"], non_blocking=True)
+                    loaded.record(cstream)
+                stream.wait_event(loaded)
+                stream.wait_event(y_free[sl])
+                for c in chains:
+                    outs = c["outs"][:-1] + [c["y_slots"][sl]]
+                    c["chain"].forward(c["x_slots"][sl], c["kind"], c["spec"].s_in, outs, c["scratch"], stream)
+                done = ev()
+                done.record(stream)
+                x_free[sl] = done
+                with torch.cuda.stream(cstream):
+                    cstream.wait_event(done)
+                    for c in chains:
+                        c["out_pins"][sl].copy_(c["y_slots"][sl], non_blocking=True)
+                    fin = ev()
+                    fin.record(cstream)
+                y_free[sl] = fin
+        e2e_steps(2)
         torch.cuda.synchronize()
         if dist:
             dist.barrier()
         s0 = torch.cuda.Event(enable_timing=True)
         s1 = torch.cuda.Event(enable_timing=True)
         s0.record(stream)
-        for _ in range(args.steps):
-            e2e_step()
+        cstream.wait_stream(stream)
+        e2e_steps(args.steps)
+        stream.wait_stream(cstream)
         s1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = job_step_time(s0.elapsed_time(s1) / args.steps, dist, dev)
@@ -439,26 +544,13 @@ def main():
         h2d = sum(c["x_pin"].numel() * c["x_pin"].element_size() for c in chains)
         d2h = sum(c["out_pin"].numel() * c["out_pin"].element_size() for c in chains)
         e2e = {"value": job_throughput(images_step, world, e2e_ms), "unit": "images/s", "h2d_bytes_per_step": h2d,
-               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms}
+               "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
+               "api": "Chain.forward -> hatq_layer (C ABI); copies on a second stream, double-buffered"}
 
     if rank != 0:
         if dist:
             dist.destroy_process_group()
         return
-
-    peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
-    peak = peaks.get("bf16_tflops_sustained")
-    peak_src = "measured bf16 sustained (fp16 operands run at the bf16 rate)"
-    if peak is None:
-        peak, peak_src = FALLBACK_BF16_TFLOPS, "fallback bf16"
-    achieved = conv_flops / (conv_ms / 1000.0) / 1e12
-    traffic = None
-    prof = os.path.join(ROOT, "profiles", "conv_cfg4_traffic.json")
-    if os.path.exists(prof):
-        traffic = json.load(open(prof)).get("dram_bytes_per_launch")
-    roofline = {"bound": "tensor", "achieved": achieved, "peak": peak, "unit": "TFLOP/s", "frac": achieved / peak,
-                "traffic": traffic, "kernel": "hatq conv_kernel (tcgen05 kind::f16, exact INT8)",
-                "launches": n_conv, "avg_launch_ms": conv_ms / max(n_conv, 1), "peak_source": peak_src}
 
     cpu = None
     if not args.no_cpu and world >= 1:
@@ -483,7 +575,8 @@ def main():
         "effective_tops": world * 2 * macs_step / (ms / 1000.0) / 1e12,
         "config": {"workload": workload_name(cfg), "global_batch": world * images_step,
                    "parallelism": f"replicas x{world}", "l2": "inputs larger than L2 (199 MB image batch)"},
-        "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
+        "roofline": roofline, "roofline_layers": layers, "roofline_fwht": roofline_fwht,
+        "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
         "gpu_launches": launches_step * args.steps,
     }
     print(json.dumps(line), flush=True)
