@@ -342,7 +342,7 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile") else args.workload)
+    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile", "int8mm") else args.workload)
     if args.impl == "reference":
         run_reference(args, cfg, scales)
         return
@@ -489,10 +489,12 @@ def main():
 
     # --- end to end through the public API (Chain.forward) with pinned host buffers: every step copies its
     # inputs in and its chain outputs back. Two input and two output slots per chain; copies run on their own
-    # stream, so step k's copies overlap the compute of steps k - 1 and k + 1.
+    # streams (host-to-device and device-to-host each on its own, so neither waits behind the other), and
+    # step k's copies overlap the compute of steps k - 1 and k + 1.
     e2e = None
     if not args.no_e2e:
-        cstream = torch.cuda.Stream(dev)
+        in_stream = torch.cuda.Stream(dev)
+        out_stream = torch.cuda.Stream(dev)
         for c in chains:
             c["x_slots"] = [c["x_dev"], torch.empty_like(c["x_dev"])]
             c["y_slots"] = [c["outs"][-1], torch.empty_like(c["outs"][-1])]
@@ -507,11 +509,11 @@ def main():
             for k in range(k_steps):
                 sl = k % 2
                 loaded = ev()
-                with torch.cuda.stream(cstream):
-                    cstream.wait_event(x_free[sl])
+                with torch.cuda.stream(in_stream):
+                    in_stream.wait_event(x_free[sl])
                     for c in chains:
                         c["x_slots"][sl].copy_(c["x_pin"], non_blocking=True)
-                    loaded.record(cstream)
+                    loaded.record(in_stream)
                 stream.wait_event(loaded)
                 stream.wait_event(y_free[sl])
                 for c in chains:
@@ -520,12 +522,12 @@ def main():
                 done = ev()
                 done.record(stream)
                 x_free[sl] = done
-                with torch.cuda.stream(cstream):
-                    cstream.wait_event(done)
+                with torch.cuda.stream(out_stream):
+                    out_stream.wait_event(done)
                     for c in chains:
                         c["out_pins"][sl].copy_(c["y_slots"][sl], non_blocking=True)
                     fin = ev()
-                    fin.record(cstream)
+                    fin.record(out_stream)
                 y_free[sl] = fin
         e2e_steps(2)
         torch.cuda.synchronize()
@@ -534,9 +536,11 @@ def main():
         s0 = torch.cuda.Event(enable_timing=True)
         s1 = torch.cuda.Event(enable_timing=True)
         s0.record(stream)
-        cstream.wait_stream(stream)
+        in_stream.wait_stream(stream)
+        out_stream.wait_stream(stream)
         e2e_steps(args.steps)
-        stream.wait_stream(cstream)
+        stream.wait_stream(in_stream)
+        stream.wait_stream(out_stream)
         s1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = job_step_time(s0.elapsed_time(s1) / args.steps, dist, dev)
@@ -545,7 +549,7 @@ def main():
         d2h = sum(c["out_pin"].numel() * c["out_pin"].element_size() for c in chains)
         e2e = {"value": job_throughput(images_step, world, e2e_ms), "unit": "images/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms,
-               "api": "Chain.forward -> hatq_layer (C ABI); copies on a second stream, double-buffered"}
+               "api": "Chain.forward -> hatq_layer (C ABI); H2D and D2H on their own streams, double-buffered"}
 
     if rank != 0:
         if dist:
