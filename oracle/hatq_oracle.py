@@ -32,8 +32,11 @@ Readings the paper leaves open (the same list is kept with the design notes):
      (math-library exp / erf, a table for the elementwise ones) rounded by R2.
   R8 the range-expansion statistic is decided on the INT8 codes a layer
      receives, exactly: max|H~ x|^2 > hb max|x|^2.
-  R9 Paley constructions are taken over primes q only; any valid construction
-     of an order serves.
+  R9 Paley constructions are taken over primes q only. Where an order has
+     several constructions (the paper fixes none) the matrix is the first of:
+     Sylvester (a power of two), Paley-I (q = m - 1), Paley-II (q = m / 2 - 1),
+     else H~_a (x) H~_(m/a) with a the smallest supported order >= 2 whose
+     cofactor m / a is supported, each factor by the same rule.
   R10 transposed convolutions use the same prepared weights (DH / WH along
      C_in / C_out) as a scatter; the integer transition is unchanged.
   R11 dynamic affine activations: unsigned 8-bit codes (q_min 0, q_max 255),
@@ -129,19 +132,17 @@ def paley2(q: int) -> np.ndarray:
 
 
 def _base_orders(limit: int) -> dict:
-    """Orders <= limit from Sylvester (2^k), Paley-I and Paley-II, each with a
-    constructor (Sylvester preferred, then Paley-I, then Paley-II)."""
+    """Orders <= limit with a direct construction, each with its constructor by
+    reading R9: Sylvester for a power of two, else Paley-I (q = m - 1 a prime,
+    q = 3 mod 4), else Paley-II (q = m / 2 - 1 a prime, q = 1 mod 4)."""
     out = {}
-    m = 1
-    while m <= limit:
-        out[m] = ("sylvester", m)
-        m *= 2
-    for q in range(3, limit):
-        if _is_prime(q):
-            if q % 4 == 3 and q + 1 <= limit and q + 1 not in out:
-                out[q + 1] = ("paley1", q)
-            if q % 4 == 1 and 2 * (q + 1) <= limit and 2 * (q + 1) not in out:
-                out[2 * (q + 1)] = ("paley2", q)
+    for m in range(1, limit + 1):
+        if m & (m - 1) == 0:
+            out[m] = ("sylvester", m)
+        elif _is_prime(m - 1) and (m - 1) % 4 == 3:
+            out[m] = ("paley1", m - 1)
+        elif m % 2 == 0 and _is_prime(m // 2 - 1) and (m // 2 - 1) % 4 == 1:
+            out[m] = ("paley2", m // 2 - 1)
     return out
 
 
@@ -150,26 +151,33 @@ _ORDERS_CACHE = {}
 
 def supported_orders(limit: int = 1024) -> dict:
     """The set M_H of supported orders <= limit: base orders and Kronecker
-    products of supported orders, each with a recipe (a nested tuple).
-    Recipes only (no matrices), cached per limit."""
+    products of supported orders, each with its recipe under reading R9 (a
+    nested tuple; recipes only, no matrices), cached per limit."""
     if limit in _ORDERS_CACHE:
         return dict(_ORDERS_CACHE[limit])
-    orders = dict(_base_orders(limit))
+    base = _base_orders(limit)
+    members = set(base)
     changed = True
     while changed:
         changed = False
-        for a in sorted(orders):
-            for b in sorted(orders):
-                if a < 2 or b < 2 or a * b > limit or a * b in orders:
-                    continue
-                orders[a * b] = ("kron", a, b)
-                changed = True
+        for a in sorted(members):
+            for b in sorted(members):
+                if a >= 2 and b >= 2 and a * b <= limit and a * b not in members:
+                    members.add(a * b)
+                    changed = True
+    orders = {}
+    for m in sorted(members):
+        if m in base:
+            orders[m] = base[m]
+        else:
+            a = min(f for f in members if f >= 2 and m % f == 0 and m // f in members)
+            orders[m] = ("kron", a, m // a)
     _ORDERS_CACHE[limit] = dict(orders)
     return orders
 
 
 def hadamard_of_order(m: int, orders: dict = None) -> np.ndarray:
-    """An unnormalized Hadamard matrix of a supported order m."""
+    """The unnormalized Hadamard matrix of a supported order m (reading R9)."""
     orders = orders or supported_orders(max(1024, m))
     if m not in orders:
         raise ValueError(f"order {m} is not supported")
@@ -240,6 +248,30 @@ def transform_real(x: np.ndarray, hb: int, normalize: bool = True) -> np.ndarray
     if normalize:
         acc = acc / math.sqrt(hb)
     return acc.reshape(x.shape)
+
+
+def transform_order_real(x: np.ndarray, m: int) -> np.ndarray:
+    """x T_in with T_in = P_C H_m of Eq. (supp_padded_transforms): the last
+    axis (C channels) is zero-padded to the order m >= C and multiplied by the
+    normalized H_m of reading R9, in the fixed order of reading R6:
+    y_j = (sum_{i=0}^{C-1} H~[i][j] x_i) / sqrt(m). Returns [..., m] fp64."""
+    x = np.asarray(x, dtype=np.float64)
+    c = x.shape[-1]
+    if m < c:
+        raise ValueError("the order must be at least the channel count")
+    H = hadamard_of_order(m).astype(np.float64)
+    acc = np.zeros(x.shape[:-1] + (m,))
+    for i in range(c):
+        acc += H[i][None, :] * x[..., i:i + 1]
+    return acc / math.sqrt(m)
+
+
+def transform_order_int(x_i8, m: int) -> np.ndarray:
+    """Unnormalized integer transform of the zero-padded channel vector,
+    y_j = sum_{i<C} H~[i][j] x_i, exact in int64: [..., m]."""
+    x = np.asarray(x_i8, dtype=np.int64)
+    H = hadamard_of_order(m)
+    return x @ H[:x.shape[-1], :]
 
 
 # --------------------------------------------------------------------------
@@ -376,16 +408,26 @@ def activation_lut(kind: str, s_z: float, s_u: float) -> np.ndarray:
 
 def prepare_layer(w_ohwi, b, form: str, hb_in: int, hb_out: int, s_x: float,
                   s_y: float, act: str, hb_next: int, out_f32: bool,
-                  stride: int, pad: int, s_z: float = None, s_u: float = None) -> Prepared:
+                  stride: int, pad: int, s_z: float = None, s_u: float = None,
+                  order_in: int = 0) -> Prepared:
     """Offline preparation of one layer (Sec. deployment realization).
     s_x: scale of the INT8 operand this layer consumes; s_y: scale of the
     INT8 operand the next layer consumes (or of this layer's output).
     A non-homogeneous act ('silu', 'gelu') takes the two-step transition of
     Sec. general nonlinearities with preactivation scale s_z and activation
-    scale s_u."""
+    scale s_u. order_in > 0 (DH only): the input side takes the paper's
+    single order m = order_in instead of blocks, W' = W (I (x) P_C H_m)
+    (Eqs. supp_padded_transforms, supp_padded_dh); the layer then consumes an
+    operand of m channels."""
     s_x = float(np.float32(s_x))
     s_y = float(np.float32(s_y))
-    wprime, bbar = transform_weights(w_ohwi, b, form, hb_in, hb_out)
+    if order_in:
+        if form != "DH":
+            raise ValueError("a paper-order input transform belongs to a DH layer")
+        wprime = transform_order_real(w_ohwi, order_in)
+        bbar = np.zeros(wprime.shape[0]) if b is None else np.asarray(b, dtype=np.float64).copy()
+    else:
+        wprime, bbar = transform_weights(w_ohwi, b, form, hb_in, hb_out)
     co = wprime.shape[0]
     flat = wprime.reshape(co, -1)
     maxabs = np.max(np.abs(flat), axis=1)
@@ -398,7 +440,7 @@ def prepare_layer(w_ohwi, b, form: str, hb_in: int, hb_out: int, s_x: float,
     a_bound = QMAX * np.sum(np.abs(w_int), axis=1) + np.abs(b_int)
     if int(np.max(a_bound)) >= 2 ** 31:
         raise OverflowError("int32 accumulator bound exceeded")
-    prep = Prepared(form=form, hb_in=hb_in, hb_out=hb_out if form == "WH" else 0,
+    prep = Prepared(form=form, hb_in=hb_in, hb_out=hb_out if form == "WH" else 0, order_in=order_in,
                     hb_next=hb_next, act=act, out_f32=out_f32, stride=stride, pad=pad,
                     s_x=s_x, s_y=s_y, s_w=s_w, b_int=b_int,
                     w_int=w_int.reshape(wprime.shape).astype(np.int8),
@@ -453,6 +495,19 @@ def quantize_act_i8(x_i8, hb: int, s_in: float, s_x: float) -> np.ndarray:
     M, n = act_multiplier(hb, s_in, s_x)
     y = transform_int(x_i8, hb)
     return np.clip(rshift_rne(M * y, n), -QMAX, QMAX).astype(np.int8)
+
+
+def quantize_act_order_i8(x_i8, m: int, s_in: float, s_x: float) -> np.ndarray:
+    """INT8 entry into the paper's order-m basis (the activation side of
+    Eq. supp_padded_dh): y = x_int P_C H~_m exactly, codes =
+    clamp(round(M_q y / 2^n_q)) with M_q / 2^n_q ~ s_in / (sqrt(m) s_x) by
+    reading R3 over the bound |y| <= 127 C. Returns [..., m] int8."""
+    x = np.asarray(x_i8, dtype=np.int64)
+    c = x.shape[-1]
+    rho = float(np.float32(s_in)) / (math.sqrt(m) * float(np.float32(s_x)))
+    M, n = fixed_point([rho], [QMAX * c], 1)
+    y = transform_order_int(x, m)
+    return np.clip(rshift_rne(int(M[0]) * y, n), -QMAX, QMAX).astype(np.int8)
 
 
 def quantize_act_dynamic_i8(x_i8, hb: int, s_in: float):

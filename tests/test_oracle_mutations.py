@@ -16,7 +16,9 @@ _orig = {k: getattr(O, k) for k in ("sylvester", "transform_real", "transform_in
                                     "act_multiplier", "range_expansion_codes", "select_form",
                                     "epilogue_general", "phi", "paley1", "padded_transforms",
                                     "_jacobsthal", "conv_transpose_codes", "conv_transpose_real",
-                                    "depth_to_space", "affine_params", "conv_layer_affine", "gdn")}
+                                    "depth_to_space", "affine_params", "conv_layer_affine", "gdn",
+                                    "transform_order_real", "transform_order_int", "quantize_act_order_i8",
+                                    "hadamard_of_order")}
 
 
 def _sylvester_bad(m):
@@ -204,7 +206,36 @@ def _igdn_divides(v, beta, gamma, inverse=False):
     return _orig["gdn"](v, beta, gamma, False)
 
 
+def _order_real_by_sqrt_c(x, m):
+    c = np.shape(x)[-1]
+    return _orig["transform_order_real"](x, m) * math.sqrt(m) / math.sqrt(c)
+
+
+def _order_int_transposed(x, m):
+    x = np.asarray(x, dtype=np.int64)
+    H = _orig["hadamard_of_order"](m)
+    return x @ H.T[:x.shape[-1], :]
+
+
+def _order_quant_sqrt_c(x_i8, m, s_in, s_x):
+    x = np.asarray(x_i8, dtype=np.int64)
+    rho = float(np.float32(s_in)) / (math.sqrt(x.shape[-1]) * float(np.float32(s_x)))
+    M, n = O.fixed_point([rho], [127 * x.shape[-1]], 1)
+    y = O.transform_order_int(x, m)
+    return np.clip(O.rshift_rne(int(M[0]) * y, n), -127, 127).astype(np.int8)
+
+
+def _orders_paley2_first(m, orders=None):
+    if m == 12:
+        return _orig["paley2"](5)
+    return _orig["hadamard_of_order"](m, orders)
+
+
 MUTATIONS = {
+    "order_normalized_by_sqrt_c": ("transform_order_real", _order_real_by_sqrt_c),
+    "order_transposed": ("transform_order_int", _order_int_transposed),
+    "order_paley2_first": ("hadamard_of_order", _orders_paley2_first),
+    "order_quantizer_sqrt_c": ("quantize_act_order_i8", _order_quant_sqrt_c),
     "gdn_norm_unsquared": ("gdn", _gdn_unsquared),
     "igdn_divides": ("gdn", _igdn_divides),
     "affine_zero_point_sign": ("affine_params", _affine_z_sign),

@@ -598,6 +598,84 @@ def test_padded_transforms_are_semi_orthogonal_and_preserve_the_layer(c):
     assert np.allclose((Xo @ Wbar.T) @ T_out.T, Xo @ Wo.T, atol=1e-10)
 
 
+def test_construction_rule_prefers_paley1_and_smallest_kronecker_factor():
+    """Reading R9: Paley-I before Paley-II where both exist (12 = Paley-I(11),
+    not Paley-II(5)); Paley-II where Paley-I does not (28, q = 13); a product
+    order takes the smallest supported left factor (320 = H~_2 (x) H~_160)."""
+    o = O.supported_orders(1024)
+    assert o[12] == ("paley1", 11) and o[28] == ("paley2", 13) and o[36] == ("paley2", 17)
+    assert o[320] == ("kron", 2, 160) and o[160] == ("kron", 2, 80) and o[80] == ("paley1", 79)
+    assert np.array_equal(O.hadamard_of_order(320), np.kron(O.sylvester(4), O.paley1(79)))
+
+
+def test_paley1_transform_of_a_constant_vector():
+    """Closed form that fixes the orientation: with H~ = I + S, S = [[0, 1^T],
+    [-1, Q]] and zero column sums of the Jacobsthal matrix Q, the input-side
+    transform y_j = sum_i H~[i][j] x_i of x = mu 1 is mu (2 - m) at j = 0 and
+    2 mu elsewhere (the transposed matrix would give mu m, 0, ..., 0)."""
+    m, mu = 192, 3
+    y = O.transform_order_int(np.full((2, m), mu, np.int8), m)
+    assert np.all(y[:, 0] == mu * (2 - m)) and np.all(y[:, 1:] == 2 * mu)
+    yr = O.transform_order_real(np.full((1, m), 1.0), m) * math.sqrt(m)
+    assert np.allclose(yr[0, 0], 2 - m) and np.allclose(yr[0, 1:], 2.0)
+
+
+@pytest.mark.parametrize("c", [20, 100, 190, 192, 320])
+def test_order_transforms_are_semi_orthogonal_and_exact(c):
+    """Eq. supp_semi_orthogonality for the loop-order transform
+    (rows of T_in = P_C H_m orthonormal), the padded DH identity of
+    Eq. supp_padded_dh, and the integer transform equal to sqrt(m) times the
+    real one on codes."""
+    m = O.hadamard_order(c)
+    T = O.transform_order_real(np.eye(c), m)
+    assert T.shape == (c, m) and np.allclose(T @ T.T, np.eye(c), atol=1e-12)
+    rng = np.random.default_rng(c)
+    x = rng.standard_normal((1, 6, 5, c))
+    w = rng.standard_normal((4, 3, 3, c))
+    assert np.allclose(O.conv_real(O.transform_order_real(x, m), O.transform_order_real(w, m), None, 1, 1),
+                       O.conv_real(x, w, None, 1, 1), atol=1e-10)
+    codes = rng.integers(-127, 128, size=(3, 7, c)).astype(np.int8)
+    yi = O.transform_order_int(codes, m)
+    assert np.array_equal(yi.astype(np.float64), np.rint(O.transform_order_real(codes, m) * math.sqrt(m)))
+
+
+def test_order_quantizer_tracks_the_real_quantizer():
+    """INT8 entry into the order-m basis: equal to the real-valued quantizer
+    Q(x T_in) up to the (M, n) approximation (at most one code, rarely), zero
+    stays zero, and the codes span the range."""
+    c, m, s_in = 190, 192, 0.05
+    x = I.activations_i8((2, 9, 11, c), seed=41, s_in=s_in)
+    y_real = O.transform_order_real(x.astype(np.float64) * float(np.float32(s_in)), m)
+    s_x = float(np.float32(O.symmetric_scale(y_real)))
+    got = O.quantize_act_order_i8(x, m, s_in, s_x).astype(np.int64)
+    ref = O.quantize_sym(y_real, s_x)
+    d = np.abs(got - ref)
+    assert got.shape[-1] == m and d.max() <= 1 and np.mean(d > 0) < 1e-3
+    assert np.abs(got).max() == 127
+    assert not O.quantize_act_order_i8(np.zeros((1, 2, 2, c), np.int8), m, s_in, s_x).any()
+
+
+def test_order_layer_tracks_the_real_model():
+    """A DH layer in the paper's order (Eq. supp_padded_dh) on the quantized
+    operand stays close to the fp64 model."""
+    c = 190
+    m = O.hadamard_order(c)
+    x_real = np.maximum(I.activations((1, 12, 12, c), seed=42).astype(np.float64), 0)
+    w, b = I.weights(64, 3, 3, c, seed=43), I.bias(64, seed=44)
+    y_ref = O.conv_real(x_real, w, b, 1, 1)
+    s_in = float(np.float32(O.symmetric_scale(x_real)))
+    x_i8 = O.quantize_sym(x_real, s_in).astype(np.int8)
+    s_x = float(np.float32(O.symmetric_scale(O.transform_order_real(x_real, m))))
+    p = O.prepare_layer(w, b, "DH", 0, 0, s_x, float(np.float32(O.symmetric_scale(y_ref))), "none", 0, False, 1, 1,
+                        order_in=m)
+    assert p.w_int.shape == (64, 3, 3, m)
+    y = O.conv_layer(O.quantize_act_order_i8(x_i8, m, s_in, s_x), p).astype(np.float64) * p.s_y
+    # against the model on the INT8 input it was given (transform-domain and weight quantization only),
+    # and against the model on the real input (plus the original-domain input quantization)
+    assert O.sqnr_db(O.conv_real(x_i8.astype(np.float64) * s_in, w, b, 1, 1), y) > 25.0
+    assert O.sqnr_db(y_ref, y) > 18.0
+
+
 # ------------------------------------------------------- decoder-side operators (transposed, sub-pixel)
 
 @pytest.mark.parametrize("k,stride,pad", [(5, 2, 2), (3, 2, 1), (3, 1, 1), (1, 1, 0)])
