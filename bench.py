@@ -52,10 +52,12 @@ def parse():
     p.add_argument("--steps", type=int, default=10)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    p.add_argument("--workload", default="cfg4", choices=["cfg4", "cfg2", "cfg1", "fwht", "profile", "int8mm"],
+    p.add_argument("--workload", default="cfg4",
+                   choices=["cfg4", "cfg2", "cfg1", "fwht", "profile", "int8mm", "orders"],
                    help="fwht: the INT8 transform+requantize pass alone on the config-4 ga2 input; "
                         "profile: the range-expansion profiling pass on the same tensor; "
-                        "int8mm: torch._int_mm 8192^3, the library INT8 GEMM as a reference point")
+                        "int8mm: torch._int_mm 8192^3, the library INT8 GEMM as a reference point; "
+                        "orders: the paper's order-192 transform layer and ga2 in that basis at batch 8")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--layer", default="", help="time one layer of the config-4 chains (e.g. ga2, h1, s0a)")
@@ -302,6 +304,46 @@ def run_fwht_mode(args):
                       "frac": gbs / peak}), flush=True)
 
 
+def run_orders_mode(args, cfg, scales):
+    """The paper's single order on the config-4 ga2 layer: the activation-side
+    transform into the Paley-I order 192 as a 1x1 tensor-core layer on the
+    8 x 1080 x 1920 x 192 INT8 input, then ga2 (5x5 s2, 192 -> 192) prepared
+    in that basis. CUDA events, inputs larger than L2."""
+    import torch
+    from paper_2608_01653_gb300 import hatq as H
+    H.load()
+    ch = cfg.chains[0]
+    L = ch.layers[1]
+    n, h, w = ch.shapes()[1]
+    g = torch.Generator(device="cuda")
+    g.manual_seed(11)
+    x = torch.randint(-127, 128, (n, h, w, L.c_in), dtype=torch.int8, device="cuda", generator=g)
+    sc = scales[ch.name][1]
+    T = H.prepare_order_transform(L.c_in, 0.05, sc["s_x"])
+    m = T.c_out
+    op = torch.empty((n, h, w, m), dtype=torch.int8, device="cuda")
+    w_, b_ = C.chain_params(ch)[1]
+    P = H.prepare_weights_order(H.make_desc(L.c_in, L.c_out, L.k, L.stride, L.pad, "DH"), w_, b_, sc["s_x"],
+                                sc["s_out"], L.act, 0)
+    y = torch.empty(P.out_shape(n, h, w), dtype=torch.int8, device="cuda")
+    t_ms = time_events(lambda: H.conv2d_i8(x, T, y=op), args.steps, args.warmup)
+    c_ms = time_events(lambda: H.conv2d_i8(op, P, y=y), args.steps, args.warmup)
+    H.sync_status()
+    peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
+    tc, hbm = peaks.get("bf16_tflops", FALLBACK_BF16_TFLOPS), peaks.get("hbm_gbs", FALLBACK_HBM_GBS)
+    t_flops, t_bytes = 2 * n * h * w * L.c_in * m, n * h * w * (L.c_in + m) + m * L.c_in
+    ho, wo = L.out_hw(h, w)
+    c_flops = 2 * n * ho * wo * L.c_out * L.k * L.k * L.c_in
+    print(json.dumps({
+        "mode": "orders", "order": m, "construction": "Paley-I q = %d" % (m - 1), "batch": n, "in_hw": [h, w],
+        "transform": {"ms": t_ms, "tflops": t_flops / (t_ms / 1000) / 1e12, "gbs": t_bytes / (t_ms / 1000) / 1e9,
+                      "bound": "hbm" if t_bytes / hbm / 1e9 > t_flops / tc / 1e12 else "tensor",
+                      "frac": max(t_bytes / (hbm * 1e9), t_flops / (tc * 1e12)) * 1000 / t_ms},
+        "ga2_order": {"ms": c_ms, "tflops": c_flops / (c_ms / 1000) / 1e12,
+                      "frac": c_flops / (tc * 1e12) * 1000 / c_ms},
+        "peaks": {"bf16_tflops": tc, "hbm_gbs": hbm}}), flush=True)
+
+
 def run_int8mm_mode(args):
     """torch._int_mm (the library INT8 GEMM, int32 output) on 8192^3, CUDA
     events: the measured INT8 tensor-core reference point of this GPU."""
@@ -342,7 +384,8 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile", "int8mm") else args.workload)
+    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile", "int8mm", "orders")
+                                  else args.workload)
     if args.impl == "reference":
         run_reference(args, cfg, scales)
         return
@@ -357,6 +400,9 @@ def main():
         return
     if args.workload == "int8mm":
         run_int8mm_mode(args)
+        return
+    if args.workload == "orders":
+        run_orders_mode(args, cfg, scales)
         return
 
     import torch

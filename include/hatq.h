@@ -52,7 +52,11 @@ typedef enum {
     HATQ_ERR_TIMEOUT = 5        /* a bounded device-side wait expired */
 } hatq_status;
 
-typedef enum { HATQ_DH = 0, HATQ_WH = 1 } hatq_form;
+/* DH, WH: Eqs. double_hadamard_quantization, weight_only_hadamard_quantization.
+ * TRANSFORM: the activation-side transform of the paper's single order m(C)
+ * as a bias-free 1x1 convolution (supplementary, deployment realization),
+ * prepared only by hatq_prepare_order_transform. */
+typedef enum { HATQ_DH = 0, HATQ_WH = 1, HATQ_TRANSFORM = 2 } hatq_form;
 /* Activation between layers. NONE and RELU are positively homogeneous and
  * fold into the single requantization of Eq. integer_hadamard_transition;
  * SILU and GELU are not and take the two-step transition of Sec. general
@@ -73,7 +77,9 @@ typedef struct {
     int kh, kw;           /* kernel size */
     int stride, pad;      /* stride >= 1, symmetric zero padding */
     int form;             /* hatq_form, from the static profile mask (Eq. layerwise_hadamard_selection) */
-    int hb_in;            /* DH: Hadamard block along c_in (16..256, power of two); 0 for WH */
+    int hb_in;            /* DH: Hadamard block along c_in (2..256, power of two), or c_in itself for a
+                             layer in the paper's single order (c_in = m, see hatq_prepare_weights_order);
+                             0 for WH */
     int hb_out;           /* WH: Hadamard block along c_out (16..128); 0 for DH */
 } hatq_conv_desc;
 
@@ -284,6 +290,55 @@ hatq_status hatq_sync_status(hatq_stream stream);
  * n == 0 is a no-op. */
 hatq_status hatq_profile_range(const int8_t *x, int n, int h, int w, int c, int hb, int32_t *maxima,
                                uint8_t *expands, hatq_stream stream);
+
+/*
+ * The paper's single Hadamard order per channel axis (Supp. Hadamard
+ * construction; Eqs. supp_hadamard_order, supp_padded_transforms,
+ * supp_padded_dh). The supported orders M_H are the Sylvester orders 2^k,
+ * the Paley-I orders q + 1 (q prime, q = 3 mod 4), the Paley-II orders
+ * 2 (q + 1) (q prime, q = 1 mod 4) and Kronecker products of supported
+ * orders, up to 4096. Where an order has several constructions the matrix is
+ * the first of Sylvester, Paley-I, Paley-II, else H~_a (x) H~_(m/a) with a the
+ * smallest supported order >= 2 whose cofactor is supported.
+ */
+/* m(C) = the smallest supported order >= 4 ceil(C / 4) (Eq. supp_hadamard_order);
+ * HATQ_ERR_UNSUPPORTED if there is none up to 4096. Host only. */
+hatq_status hatq_hadamard_order(int c, int *m);
+/* The unnormalized matrix H~_m (+-1 entries) into host memory, row-major
+ * [m][m]; HATQ_ERR_UNSUPPORTED for an order outside M_H. Host only. */
+hatq_status hatq_hadamard_matrix(int m, int8_t *h);
+/*
+ * A DH layer whose input side takes the paper's order m = m(c_in) over the
+ * whole channel axis: W' = W (I_{KhKw} (x) P_C H_m) (Eq. supp_padded_dh, with
+ * zero padding from c_in to m). d->form = HATQ_DH, d->c_in = C (the real
+ * channel count), d->hb_in = 0 or m. The prepared layer consumes an operand
+ * of m channels: out->d gets c_in = hb_in = m, and its device buffers are
+ * sized by hatq_prepared_sizes on that descriptor. Every other argument, rule
+ * and error as hatq_prepare_weights. The operand comes from the transform
+ * layer of hatq_prepare_order_transform (or is already in the order-m basis).
+ */
+hatq_status hatq_prepare_weights_order(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                       float s_y, int act, int hb_next, int out_f32, hatq_prepared *out,
+                                       hatq_stream stream);
+/* The host arithmetic of hatq_prepare_weights_order into host arrays sized for
+ * the order-m operand (c_out * k_pad and c_out entries). */
+hatq_status hatq_prepare_weights_order_host(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                            float s_y, int act, int hb_next, int out_f32, int8_t *w_i8,
+                                            uint16_t *w_f16, int32_t *b_int, int32_t *mult, float *deq, float *s_w,
+                                            int *shift);
+/*
+ * The activation-side transform into the paper's order m = m(c) as a
+ * bias-free 1x1 convolution (supplementary, deployment realization), run by
+ * hatq_conv2d_i8 (or hatq_layer with HATQ_IN_I8) on the tensor cores: for
+ * INT8 codes x at scale s_in with c channels,
+ *   y_j = clamp(round(M_q (sum_{i<c} H~_m[i][j] x_i) / 2^n_q)),  j < m,
+ * M_q / 2^n_q ~ s_in / (sqrt(m) s_out) by the (M, n) rule of
+ * hatq_prepare_weights with the bound |sum| <= 127 c. The layer is
+ * {c_in = c, c_out = m, 1x1, stride 1, form HATQ_TRANSFORM}; its device
+ * buffers are sized by hatq_prepared_sizes on that descriptor (m must be a
+ * multiple of 32). s_in, s_out > 0.
+ */
+hatq_status hatq_prepare_order_transform(int c, float s_in, float s_out, hatq_prepared *out, hatq_stream stream);
 
 /* Layer-wise strategy selection (Eqs. hadamard_sensitivity,
  * layerwise_hadamard_selection) from the per-image indicators of

@@ -57,6 +57,115 @@ bool pow2(int v) { return v > 0 && (v & (v - 1)) == 0; }
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 int sylvester_sign(int i, int j) { return (__builtin_popcount((unsigned)(i & j)) & 1) ? -1 : 1; }
 
+// ------------------------------------------------------------ Hadamard orders (Supp. Hadamard construction)
+//
+// The supported set M_H: Sylvester orders 2^k, Paley-I orders q + 1 (q a
+// prime, q = 3 mod 4), Paley-II orders 2 (q + 1) (q a prime, q = 1 mod 4) and
+// Kronecker products of supported orders. Where an order has several
+// constructions the matrix is the first of Sylvester, Paley-I, Paley-II, else
+// H~_a (x) H~_(m/a) with a the smallest supported order >= 2 whose cofactor is
+// supported (each factor by the same rule).
+
+constexpr int kMaxOrder = 4096;
+
+bool is_prime(int q) {
+    if (q < 2) return false;
+    for (int f = 2; f * f <= q; ++f)
+        if (q % f == 0) return false;
+    return true;
+}
+
+// 1 Sylvester, 2 Paley-I, 3 Paley-II, 0 none
+int base_kind(int m) {
+    if (m >= 1 && (m & (m - 1)) == 0) return 1;
+    if (is_prime(m - 1) && (m - 1) % 4 == 3) return 2;
+    if (m % 2 == 0 && is_prime(m / 2 - 1) && (m / 2 - 1) % 4 == 1) return 3;
+    return 0;
+}
+
+const std::vector<char> &supported_table() {
+    static const std::vector<char> sup = [] {
+        std::vector<char> t(kMaxOrder + 1, 0);
+        for (int m = 1; m <= kMaxOrder; ++m) {
+            if (base_kind(m)) { t[m] = 1; continue; }
+            for (int a = 2; a < m && !t[m]; ++a)
+                if (m % a == 0 && t[a] && t[m / a]) t[m] = 1;
+        }
+        return t;
+    }();
+    return sup;
+}
+
+bool order_supported(int m) { return m >= 1 && m <= kMaxOrder && supported_table()[m]; }
+
+// quadratic character modulo the prime q
+std::vector<int> quadratic_character(int q) {
+    std::vector<int> chi(q, -1);
+    chi[0] = 0;
+    for (int x = 1; x < q; ++x) chi[(long long)x * x % q] = 1;
+    return chi;
+}
+
+// H~_m row-major into h (m * m entries of +-1)
+void build_hadamard(int m, int8_t *h) {
+    const int kind = base_kind(m);
+    if (kind == 1) {
+        for (int i = 0; i < m; ++i)
+            for (int j = 0; j < m; ++j) h[(size_t)i * m + j] = (int8_t)sylvester_sign(i, j);
+        return;
+    }
+    if (kind == 2) {
+        // H = I + S, S = [[0, 1^T], [-1, Q]], Q[i][j] = chi(j - i)
+        const int q = m - 1;
+        const std::vector<int> chi = quadratic_character(q);
+        for (int i = 0; i < m; ++i)
+            for (int j = 0; j < m; ++j) {
+                int v;
+                if (i == 0) v = j == 0 ? 0 : 1;
+                else if (j == 0) v = -1;
+                else v = chi[((j - i) % q + q) % q];
+                h[(size_t)i * m + j] = (int8_t)(v + (i == j ? 1 : 0));
+            }
+        return;
+    }
+    if (kind == 3) {
+        // C = [[0, 1^T], [1, Q]] symmetric; H = C (x) [[1, 1], [1, -1]] + I (x) [[1, -1], [-1, -1]]
+        const int q = m / 2 - 1, n = q + 1;
+        const std::vector<int> chi = quadratic_character(q);
+        const int A[2][2] = {{1, 1}, {1, -1}}, B[2][2] = {{1, -1}, {-1, -1}};
+        for (int i = 0; i < n; ++i)
+            for (int j = 0; j < n; ++j) {
+                int c;
+                if (i == 0) c = j == 0 ? 0 : 1;
+                else if (j == 0) c = 1;
+                else c = chi[((j - i) % q + q) % q];
+                for (int k = 0; k < 2; ++k)
+                    for (int l = 0; l < 2; ++l)
+                        h[(size_t)(2 * i + k) * m + (2 * j + l)] = (int8_t)(c * A[k][l] + (i == j ? B[k][l] : 0));
+            }
+        return;
+    }
+    int a = 2;
+    while (!(m % a == 0 && order_supported(a) && order_supported(m / a))) ++a;
+    const int b = m / a;
+    std::vector<int8_t> ha((size_t)a * a), hb((size_t)b * b);
+    build_hadamard(a, ha.data());
+    build_hadamard(b, hb.data());
+    for (int i = 0; i < a; ++i)
+        for (int j = 0; j < a; ++j)
+            for (int k = 0; k < b; ++k)
+                for (int l = 0; l < b; ++l)
+                    h[(size_t)(i * b + k) * m + (j * b + l)] = (int8_t)(ha[(size_t)i * a + j] * hb[(size_t)k * b + l]);
+}
+
+// m(C) of Eq. supp_hadamard_order: the smallest supported order >= 4 ceil(C / 4); 0 if none <= kMaxOrder
+int hadamard_order_of(int c) {
+    if (c < 1) return 0;
+    for (int m = 4 * ((c + 3) / 4); m <= kMaxOrder; ++m)
+        if (order_supported(m)) return m;
+    return 0;
+}
+
 // ------------------------------------------------------------ tensor maps
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -92,9 +201,17 @@ hatq_status check_desc(const hatq_conv_desc *d) {
     if (d->pad < 0 || d->pad >= d->kh || d->pad >= d->kw) return fail(HATQ_ERR_INVALID_ARG, "padding out of range");
     if (d->form == HATQ_DH) {
         if (d->hb_out != 0) return fail(HATQ_ERR_INVALID_ARG, "a DH layer has no output block");
-        if (!pow2(d->hb_in) || d->hb_in < 2 || d->hb_in > 256 || d->c_in % d->hb_in)
-            return fail(HATQ_ERR_INVALID_ARG, "DH block hb_in must be a power of two in 2..256 dividing c_in");
+        const bool block = pow2(d->hb_in) && d->hb_in >= 2 && d->hb_in <= 256 && d->c_in % d->hb_in == 0;
+        const bool order = d->hb_in == d->c_in && order_supported(d->hb_in);   // the paper's single order
+        if (!block && !order)
+            return fail(HATQ_ERR_INVALID_ARG, "DH block hb_in must be a power of two in 2..256 dividing c_in, or c_in "
+                                              "itself when c_in is a supported Hadamard order");
         if (d->c_in % 16) return fail(HATQ_ERR_UNSUPPORTED, "a DH layer needs c_in % 16 == 0");
+    } else if (d->form == HATQ_TRANSFORM) {
+        if (d->kh != 1 || d->kw != 1 || d->stride != 1 || d->pad != 0 || d->hb_in != 0 || d->hb_out != 0)
+            return fail(HATQ_ERR_INVALID_ARG, "a transform layer is a 1x1 stride-1 convolution without blocks");
+        if (!order_supported(d->c_out) || d->c_out < d->c_in)
+            return fail(HATQ_ERR_INVALID_ARG, "a transform layer maps c_in channels to a supported order >= c_in");
     } else if (d->form == HATQ_WH) {
         if (d->hb_in != 0) return fail(HATQ_ERR_INVALID_ARG, "a WH layer has no input block");
         if (!pow2(d->hb_out) || d->hb_out < 2 || d->hb_out > 128 || d->c_out % d->hb_out)
@@ -192,6 +309,8 @@ hatq_status validate_prepare(const hatq_conv_desc *d, const float *w_ohwi, float
                                     int hb_next, int out_f32, Geometry *g) {
     hatq_status st = check_desc(d);
     if (st != HATQ_OK) return st;
+    if (d->form == HATQ_TRANSFORM)
+        return fail(HATQ_ERR_INVALID_ARG, "transform layers are prepared with hatq_prepare_order_transform");
     if (!w_ohwi) return fail(HATQ_ERR_INVALID_ARG, "null weights");
     if (!(s_x > 0.f) || !std::isfinite(s_x)) return fail(HATQ_ERR_INVALID_ARG, "s_x must be positive");
     if (!out_f32 && (!(s_y > 0.f) || !std::isfinite(s_y))) return fail(HATQ_ERR_INVALID_ARG, "s_y must be positive");
@@ -232,12 +351,36 @@ hatq_status validate_general(const hatq_conv_desc *d, int act, int hb_next, int 
     return HATQ_OK;
 }
 
+// The descriptor of the operand a layer consumes: for a DH layer in the
+// paper's single order (order > 0) the operand has m = order channels and the
+// block is the whole axis; otherwise the caller's descriptor.
+hatq_status operand_desc(const hatq_conv_desc *d, int order, hatq_conv_desc *op) {
+    if (!d) return fail(HATQ_ERR_INVALID_ARG, "null descriptor");
+    *op = *d;
+    if (!order) {
+        if (d->form == HATQ_DH && !pow2(d->hb_in))
+            return fail(HATQ_ERR_INVALID_ARG, "a paper-order DH layer is prepared with hatq_prepare_weights_order");
+        return HATQ_OK;
+    }
+    if (d->form != HATQ_DH) return fail(HATQ_ERR_UNSUPPORTED, "the paper's single order is implemented for DH layers");
+    if (d->c_in < 1 || (d->hb_in != 0 && d->hb_in != order))
+        return fail(HATQ_ERR_INVALID_ARG, "hb_in of a paper-order layer must be 0 or m(c_in) = %d", order);
+    op->c_in = order;
+    op->hb_in = order;
+    return HATQ_OK;
+}
+
 hatq_status prepare_core(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x, float s_y,
-                         int act, int hb_next, int out_f32, GeneralParams *gen, int8_t *w_i8_out,
+                         int act, int hb_next, int out_f32, GeneralParams *gen, int order, int8_t *w_i8_out,
                          uint16_t *w_f16_out, int32_t *b_int_out, int32_t *mult_out, float *deq_out, float *s_w_out,
                          int *shift_out) {
+    hatq_conv_desc dop;
+    hatq_status st = operand_desc(d, order, &dop);
+    if (st != HATQ_OK) return st;
+    const int c_src = d->c_in;                      // channels of the real-valued weights
+    d = &dop;
     Geometry g;
-    hatq_status st = validate_prepare(d, w_ohwi, s_x, s_y, act, hb_next, out_f32, &g);
+    st = validate_prepare(d, w_ohwi, s_x, s_y, act, hb_next, out_f32, &g);
     if (st != HATQ_OK) return st;
     if (general_act(act) != (gen != nullptr))
         return fail(HATQ_ERR_INVALID_ARG, "SiLU / GELU layers are prepared with hatq_prepare_weights_general");
@@ -251,7 +394,22 @@ hatq_status prepare_core(const hatq_conv_desc *d, const float *w_ohwi, const flo
     std::vector<double> bbar(co, 0.0);
     if (bias)
         for (int o = 0; o < co; ++o) bbar[o] = (double)bias[o];
-    if (d->form == HATQ_DH) {
+    if (order) {
+        // Eq. supp_padded_dh: W' = W (I (x) P_C H_m), output j of a tap in the fixed order
+        // acc = 0; acc += +-w_i, i = 0..C-1; acc / sqrt(m)
+        std::vector<int8_t> h((size_t)order * order);
+        build_hadamard(order, h.data());
+        const double sq = std::sqrt((double)order);
+        for (long long r = 0; r < (long long)co * taps; ++r)
+            for (int j = 0; j < order; ++j) {
+                double acc = 0.0;
+                for (int i = 0; i < c_src; ++i) {
+                    const double x = (double)w_ohwi[r * c_src + i];
+                    acc += h[(size_t)i * order + j] > 0 ? x : -x;
+                }
+                wp[r * ci + j] = acc / sq;
+            }
+    } else if (d->form == HATQ_DH) {
         const int hb = d->hb_in;
         for (long long r = 0; r < (long long)co * taps; ++r)
             for (int blk = 0; blk < ci / hb; ++blk) {
@@ -365,7 +523,17 @@ hatq_status hatq_prepare_weights_host(const hatq_conv_desc *d, const float *w_oh
                                       float s_y, int act, int hb_next, int out_f32, int8_t *w_i8_out,
                                       uint16_t *w_f16_out, int32_t *b_int_out, int32_t *mult_out, float *deq_out,
                                       float *s_w_out, int *shift_out) {
-    return prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, nullptr, w_i8_out, w_f16_out, b_int_out,
+    return prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, nullptr, 0, w_i8_out, w_f16_out, b_int_out,
+                        mult_out, deq_out, s_w_out, shift_out);
+}
+
+hatq_status hatq_prepare_weights_order_host(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                            float s_y, int act, int hb_next, int out_f32, int8_t *w_i8_out,
+                                            uint16_t *w_f16_out, int32_t *b_int_out, int32_t *mult_out,
+                                            float *deq_out, float *s_w_out, int *shift_out) {
+    const int m = d ? hadamard_order_of(d->c_in) : 0;
+    if (d && !m) return fail(HATQ_ERR_UNSUPPORTED, "no supported Hadamard order for c_in=%d", d->c_in);
+    return prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, nullptr, m, w_i8_out, w_f16_out, b_int_out,
                         mult_out, deq_out, s_w_out, shift_out);
 }
 
@@ -380,7 +548,7 @@ hatq_status hatq_prepare_weights_general_host(const hatq_conv_desc *d, const flo
     GeneralParams gen;
     gen.s_z = s_z;
     gen.s_u = s_u;
-    hatq_status st = prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, 0, &gen, w_i8_out, w_f16_out, b_int_out,
+    hatq_status st = prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, 0, &gen, 0, w_i8_out, w_f16_out, b_int_out,
                                   mult_out, deq.data(), s_w_out, shift_out);
     if (st != HATQ_OK) return st;
     *mult_in_out = gen.mult_in;
@@ -393,35 +561,41 @@ hatq_status hatq_prepare_weights_general_host(const hatq_conv_desc *d, const flo
 
 namespace {
 
-hatq_status prepare_device(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x, float s_y,
-                           int act, int hb_next, int out_f32, GeneralParams *gen, hatq_prepared *out,
-                           hatq_stream stream) {
-    Geometry g;
-    hatq_status st = validate_prepare(d, w_ohwi, s_x, s_y, act, hb_next, out_f32, &g);
-    if (st != HATQ_OK) return st;
+// Host arrays of a prepared layer in the library's packed layout.
+struct HostLayer {
+    std::vector<int8_t> w_i8;
+    std::vector<uint16_t> w_f16;
+    std::vector<int32_t> b_int, mult;
+    std::vector<float> deq, s_w;
+    int shift = 0;
+    HostLayer(int co, int k_pad) : w_i8((size_t)co * k_pad), w_f16((size_t)co * k_pad), b_int(co), mult(co), deq(co),
+                                   s_w(co) {}
+};
+
+hatq_status check_out_buffers(const hatq_prepared *out) {
     if (!out) return fail(HATQ_ERR_INVALID_ARG, "null output struct");
     if (!out->w_i8 || !out->w_f16 || !out->b_int || !out->mult || !out->deq || !out->s_w)
         return fail(HATQ_ERR_INVALID_ARG, "prepared-layer device buffers must be set before preparation");
     if (!aligned16(out->w_i8) || !aligned16(out->w_f16) || !aligned16(out->b_int) || !aligned16(out->mult) ||
         !aligned16(out->deq) || !aligned16(out->s_w))
         return fail(HATQ_ERR_INVALID_ARG, "prepared-layer device buffers must be 16-byte aligned");
-    const int co = d->c_out;
-    std::vector<int8_t> w_i8((size_t)co * g.k_pad);
-    std::vector<uint16_t> w_f16((size_t)co * g.k_pad);
-    std::vector<int32_t> b_int(co), mult(co);
-    std::vector<float> deq(co), s_w(co);
-    int shift = 0;
-    st = prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, gen, w_i8.data(), w_f16.data(), b_int.data(),
-                      mult.data(), deq.data(), s_w.data(), &shift);
-    if (st != HATQ_OK) return st;
+    return HATQ_OK;
+}
+
+// Copies the host arrays to the caller's device buffers, encodes the weight
+// tensor map and fills the struct (dop: the descriptor of the operand).
+hatq_status upload_layer(const hatq_conv_desc &dop, const Geometry &g, const HostLayer &hl, int act, int hb_next,
+                         int out_f32, float s_x, float s_y, const GeneralParams *gen, hatq_prepared *out,
+                         hatq_stream stream) {
+    const int co = dop.c_out;
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     cudaError_t e;
-    if ((e = cudaMemcpyAsync(out->w_i8, w_i8.data(), w_i8.size(), cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(out->w_f16, w_f16.data(), w_f16.size() * 2, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(out->b_int, b_int.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(out->mult, mult.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(out->deq, deq.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
-        (e = cudaMemcpyAsync(out->s_w, s_w.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+    if ((e = cudaMemcpyAsync(out->w_i8, hl.w_i8.data(), hl.w_i8.size(), cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->w_f16, hl.w_f16.data(), hl.w_f16.size() * 2, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->b_int, hl.b_int.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->mult, hl.mult.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->deq, hl.deq.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->s_w, hl.s_w.data(), co * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess)
         return cuda_fail(e, "upload of prepared weights");
     if ((e = cudaStreamSynchronize(s)) != cudaSuccess) return cuda_fail(e, "upload of prepared weights");
     // weight tensor map: [c_out][k_pad] fp16, 64 x n_t box, 128-byte swizzle
@@ -439,11 +613,11 @@ hatq_status prepare_device(const hatq_conv_desc *d, const float *w_ohwi, const f
     static_assert(sizeof(CUtensorMap) <= sizeof(out->opaque), "opaque area too small");
     std::memcpy(out->opaque, &tm, sizeof tm);
 
-    out->d = *d;
+    out->d = dop;
     out->act = act;
     out->hb_next = hb_next;
     out->out_f32 = out_f32 ? 1 : 0;
-    out->shift = shift;
+    out->shift = hl.shift;
     out->k_pad = g.k_pad;
     out->gather = g.gather;
     out->s_x = s_x;
@@ -458,6 +632,63 @@ hatq_status prepare_device(const hatq_conv_desc *d, const float *w_ohwi, const f
     return HATQ_OK;
 }
 
+hatq_status prepare_device(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x, float s_y,
+                           int act, int hb_next, int out_f32, GeneralParams *gen, int order, hatq_prepared *out,
+                           hatq_stream stream) {
+    hatq_conv_desc dop;
+    hatq_status st = operand_desc(d, order, &dop);
+    if (st != HATQ_OK) return st;
+    Geometry g;
+    if ((st = validate_prepare(&dop, w_ohwi, s_x, s_y, act, hb_next, out_f32, &g)) != HATQ_OK) return st;
+    if ((st = check_out_buffers(out)) != HATQ_OK) return st;
+    HostLayer hl(dop.c_out, g.k_pad);
+    st = prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, gen, order, hl.w_i8.data(), hl.w_f16.data(),
+                      hl.b_int.data(), hl.mult.data(), hl.deq.data(), hl.s_w.data(), &hl.shift);
+    if (st != HATQ_OK) return st;
+    return upload_layer(dop, g, hl, act, hb_next, out_f32, s_x, s_y, gen, out, stream);
+}
+
+// The activation-side transform of the paper's order m = m(c) as a 1x1
+// convolution (Sec. deployment realization): c input channels (codes in the
+// original basis at s_in), m output channels, weights w[j][i] = H~_m[i][j],
+// zero bias, one multiplier M_q / 2^n_q ~ s_in / (sqrt(m) s_out) by the
+// (M, n) rule over |y| <= 127 c.
+hatq_status transform_core(int c, float s_in, float s_out, hatq_conv_desc *dt, Geometry *g, HostLayer **out) {
+    const int m = hadamard_order_of(c);
+    if (!m) return fail(HATQ_ERR_UNSUPPORTED, "no supported Hadamard order for c=%d", c);
+    if (!(s_in > 0.f) || !std::isfinite(s_in) || !(s_out > 0.f) || !std::isfinite(s_out))
+        return fail(HATQ_ERR_INVALID_ARG, "s_in and s_out must be positive");
+    *dt = hatq_conv_desc{c, m, 1, 1, 1, 0, HATQ_TRANSFORM, 0, 0};
+    hatq_status st = check_desc(dt);
+    if (st != HATQ_OK) return st;
+    if ((st = geometry(dt, 0, g)) != HATQ_OK) return st;
+    std::vector<int8_t> h((size_t)m * m);
+    build_hadamard(m, h.data());
+    HostLayer *hl = new HostLayer(m, g->k_pad);
+    for (int j = 0; j < m; ++j) {
+        for (int k = 0; k < g->k_pad; ++k) hl->w_f16[(size_t)j * g->k_pad + k] = f16_bits(0);
+        for (int i = 0; i < c; ++i) {       // 1x1: reduction index i in both packings
+            hl->w_i8[(size_t)j * g->k_pad + i] = h[(size_t)i * m + j];
+            hl->w_f16[(size_t)j * g->k_pad + i] = f16_bits(h[(size_t)i * m + j]);
+        }
+    }
+    std::vector<int32_t> M;
+    const double rho = (double)s_in / (std::sqrt((double)m) * (double)s_out);
+    if ((st = fixed_point(std::vector<double>(1, rho), std::vector<long long>(1, 127LL * c), 1, M, hl->shift)) !=
+        HATQ_OK) {
+        delete hl;
+        return st;
+    }
+    for (int j = 0; j < m; ++j) {
+        hl->mult[j] = M[0];
+        hl->b_int[j] = 0;
+        hl->deq[j] = 0.f;
+        hl->s_w[j] = 1.f;
+    }
+    *out = hl;
+    return HATQ_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -465,7 +696,42 @@ extern "C" {
 hatq_status hatq_prepare_weights(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
                                  float s_y, int act, int hb_next, int out_f32, hatq_prepared *out,
                                  hatq_stream stream) {
-    return prepare_device(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, nullptr, out, stream);
+    return prepare_device(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, nullptr, 0, out, stream);
+}
+
+hatq_status hatq_hadamard_order(int c, int *m) {
+    if (!m) return fail(HATQ_ERR_INVALID_ARG, "null output");
+    if (c < 1) return fail(HATQ_ERR_INVALID_ARG, "c must be positive");
+    *m = hadamard_order_of(c);
+    if (!*m) return fail(HATQ_ERR_UNSUPPORTED, "no supported Hadamard order >= 4 ceil(c / 4) up to %d", kMaxOrder);
+    return HATQ_OK;
+}
+
+hatq_status hatq_hadamard_matrix(int m, int8_t *h) {
+    if (!h) return fail(HATQ_ERR_INVALID_ARG, "null output");
+    if (!order_supported(m)) return fail(HATQ_ERR_UNSUPPORTED, "order %d is not supported", m);
+    build_hadamard(m, h);
+    return HATQ_OK;
+}
+
+hatq_status hatq_prepare_weights_order(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
+                                       float s_y, int act, int hb_next, int out_f32, hatq_prepared *out,
+                                       hatq_stream stream) {
+    const int m = d ? hadamard_order_of(d->c_in) : 0;
+    if (d && !m) return fail(HATQ_ERR_UNSUPPORTED, "no supported Hadamard order for c_in=%d", d->c_in);
+    return prepare_device(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, nullptr, m, out, stream);
+}
+
+hatq_status hatq_prepare_order_transform(int c, float s_in, float s_out, hatq_prepared *out, hatq_stream stream) {
+    hatq_status st = check_out_buffers(out);
+    if (st != HATQ_OK) return st;
+    hatq_conv_desc dt;
+    Geometry g;
+    HostLayer *hl = nullptr;
+    if ((st = transform_core(c, s_in, s_out, &dt, &g, &hl)) != HATQ_OK) return st;
+    st = upload_layer(dt, g, *hl, HATQ_ACT_NONE, 0, 0, s_in, s_out, nullptr, out, stream);
+    delete hl;
+    return st;
 }
 
 hatq_status hatq_prepare_weights_general(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x,
@@ -474,7 +740,7 @@ hatq_status hatq_prepare_weights_general(const hatq_conv_desc *d, const float *w
     GeneralParams gen;
     gen.s_z = s_z;
     gen.s_u = s_u;
-    return prepare_device(d, w_ohwi, bias, s_x, s_y, act, hb_next, 0, &gen, out, stream);
+    return prepare_device(d, w_ohwi, bias, s_x, s_y, act, hb_next, 0, &gen, 0, out, stream);
 }
 
 hatq_status hatq_quantize_act(const void *x, int x_kind, float s_in, int n, int h, int w, int c, int hb, float s_out,
@@ -660,6 +926,8 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
 int hatq_layer_launches(int x_kind, float s_in, const hatq_prepared *L) {
     if (!L) return -1;
     if (x_kind == HATQ_IN_OPERAND) return 1;
+    if (L->d.form == HATQ_TRANSFORM) return x_kind == HATQ_IN_I8 ? 1 : -1;
+    if (L->d.form == HATQ_DH && !pow2(L->d.hb_in)) return -1;   // paper order: operand from the transform layer
     if (x_kind == HATQ_IN_I8) return (L->d.form == HATQ_WH && s_in == L->s_x) ? 1 : 2;
     if (x_kind == HATQ_IN_F16) return 2;
     return -1;
@@ -671,9 +939,14 @@ hatq_status hatq_layer(const void *x, int x_kind, float s_in, int n, int h, int 
     if (n == 0 && h >= 1 && w >= 1) return HATQ_OK;                    // empty batch: nothing to do
     if (!x || !y) return fail(HATQ_ERR_INVALID_ARG, "null argument");
     const hatq_conv_desc *d = &L->d;
-    if (x_kind == HATQ_IN_OPERAND || (x_kind == HATQ_IN_I8 && d->form == HATQ_WH && s_in == L->s_x))
+    if (x_kind == HATQ_IN_OPERAND || (x_kind == HATQ_IN_I8 && d->form == HATQ_WH && s_in == L->s_x) ||
+        (x_kind == HATQ_IN_I8 && d->form == HATQ_TRANSFORM))
         return hatq_conv2d_i8(static_cast<const int8_t *>(x), n, h, w, L, y, stream);
     if (x_kind != HATQ_IN_I8 && x_kind != HATQ_IN_F16) return fail(HATQ_ERR_INVALID_ARG, "unknown input kind %d", x_kind);
+    if (d->form == HATQ_TRANSFORM) return fail(HATQ_ERR_INVALID_ARG, "a transform layer takes INT8 codes");
+    if (d->form == HATQ_DH && !pow2(d->hb_in))
+        return fail(HATQ_ERR_UNSUPPORTED, "a paper-order layer consumes the output of its transform layer "
+                                          "(hatq_prepare_order_transform) as HATQ_IN_OPERAND");
     const size_t need = (size_t)n * h * w * d->c_in;
     if (!scratch || scratch_bytes < need) return fail(HATQ_ERR_INVALID_ARG, "scratch must hold %zu bytes", need);
     if (d->c_in % 16) return fail(HATQ_ERR_UNSUPPORTED, "an input transform needs c_in % 16 == 0");

@@ -16,7 +16,7 @@ import numpy as np
 from . import build as _build
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_OVERFLOW, ERR_CUDA, ERR_TIMEOUT = range(6)
-DH, WH = 0, 1
+DH, WH, TRANSFORM = 0, 1, 2
 ACT_NONE, ACT_RELU, ACT_SILU, ACT_GELU = 0, 1, 2, 3
 IN_OPERAND, IN_I8, IN_F16 = 0, 1, 2
 
@@ -82,6 +82,13 @@ def load(build: bool = True) -> ctypes.CDLL:
             "hatq_selftest_wait": (_I, [ctypes.c_ulonglong, _P]),
             "hatq_profile_range": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P]),
             "hatq_select_form": (_I, [_P, _I, _I, _I, ctypes.POINTER(_I), ctypes.POINTER(_I)]),
+            "hatq_hadamard_order": (_I, [_I, ctypes.POINTER(_I)]),
+            "hatq_hadamard_matrix": (_I, [_I, _P]),
+            "hatq_prepare_weights_order": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _I, _I, _I,
+                                                ctypes.POINTER(PreparedStruct), _P]),
+            "hatq_prepare_weights_order_host": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _I, _I, _I,
+                                                     _P, _P, _P, _P, _P, _P, ctypes.POINTER(_I)]),
+            "hatq_prepare_order_transform": (_I, [_I, _F, _F, ctypes.POINTER(PreparedStruct), _P]),
             "hatq_layer_noalloc": (_I, [_P, _I, _F, _I, _I, _I, ctypes.POINTER(PreparedStruct), _P, _P]),
             "hatq_version": (_I, []),
         }
@@ -240,6 +247,71 @@ def prepare_weights(desc: ConvDesc, w_ohwi, bias, s_x, s_y, act="none", hb_next=
     _check(load().hatq_prepare_weights(ctypes.byref(desc), w.ctypes.data, bp, float(s_x), float(s_y),
                                        _ACTS.get(act, act), int(hb_next), int(bool(out_f32)),
                                        ctypes.byref(L.struct), _stream(stream)))
+    return L
+
+
+def hadamard_order(c: int) -> int:
+    """hatq_hadamard_order: m(C) of Eq. supp_hadamard_order."""
+    m = ctypes.c_int()
+    _check(load().hatq_hadamard_order(int(c), ctypes.byref(m)))
+    return m.value
+
+
+def hadamard_matrix(m: int) -> np.ndarray:
+    """hatq_hadamard_matrix: the library's unnormalized H~_m as an int8 [m, m] array."""
+    h = np.zeros((m, m), np.int8)
+    _check(load().hatq_hadamard_matrix(int(m), h.ctypes.data))
+    return h
+
+
+def order_desc(desc: ConvDesc) -> ConvDesc:
+    """The operand descriptor of a DH layer in the paper's order: c_in = hb_in = m(c_in)."""
+    m = hadamard_order(desc.c_in)
+    return ConvDesc(m, desc.c_out, desc.kh, desc.kw, desc.stride, desc.pad, desc.form, m, 0)
+
+
+def prepare_weights_order_host(desc: ConvDesc, w_ohwi, bias, s_x, s_y, act="none", hb_next=0, out_f32=False):
+    """hatq_prepare_weights_order_host: a paper-order DH layer prepared into host arrays."""
+    if desc.form != DH:                             # the library rejects it before touching any buffer
+        _check(load().hatq_prepare_weights_order_host(ctypes.byref(desc), None, None, float(s_x), float(s_y), 0, 0,
+                                                      0, None, None, None, None, None, None, None))
+    dop = order_desc(desc)
+    w_elems, ch = prepared_sizes(dop)
+    w = np.ascontiguousarray(w_ohwi, dtype=np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    out = HostPrepared(np.zeros(w_elems, np.int8), np.zeros(w_elems, np.uint16), np.zeros(ch, np.int32),
+                       np.zeros(ch, np.int32), np.zeros(ch, np.float32), np.zeros(ch, np.float32), 0)
+    shift = ctypes.c_int()
+    _check(load().hatq_prepare_weights_order_host(
+        ctypes.byref(desc), w.ctypes.data, None if b is None else b.ctypes.data, float(s_x), float(s_y),
+        _ACTS.get(act, act), int(hb_next), int(bool(out_f32)), out.w_i8.ctypes.data, out.w_f16.ctypes.data,
+        out.b_int.ctypes.data, out.mult.ctypes.data, out.deq.ctypes.data, out.s_w.ctypes.data, ctypes.byref(shift)))
+    out.shift = shift.value
+    out.w_i8 = out.w_i8.reshape(desc.c_out, -1)
+    out.w_f16 = out.w_f16.reshape(desc.c_out, -1)
+    return out
+
+
+def prepare_weights_order(desc: ConvDesc, w_ohwi, bias, s_x, s_y, act="none", hb_next=0, out_f32=False,
+                          stream=None, device="cuda") -> "PreparedLayer":
+    """hatq_prepare_weights_order: a DH layer whose input side takes the paper's
+    order m(c_in); the returned layer consumes an operand of m channels."""
+    L = PreparedLayer(order_desc(desc), device)
+    w = np.ascontiguousarray(w_ohwi, dtype=np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    _check(load().hatq_prepare_weights_order(ctypes.byref(desc), w.ctypes.data, None if b is None else b.ctypes.data,
+                                             float(s_x), float(s_y), _ACTS.get(act, act), int(hb_next),
+                                             int(bool(out_f32)), ctypes.byref(L.struct), _stream(stream)))
+    return L
+
+
+def prepare_order_transform(c: int, s_in, s_out, stream=None, device="cuda") -> "PreparedLayer":
+    """hatq_prepare_order_transform: the activation-side transform into the
+    order m(c) as a 1x1 layer (c -> m channels), run with conv2d_i8 or layer."""
+    m = hadamard_order(c)
+    L = PreparedLayer(ConvDesc(c, m, 1, 1, 1, 0, TRANSFORM, 0, 0), device)
+    _check(load().hatq_prepare_order_transform(int(c), float(s_in), float(s_out), ctypes.byref(L.struct),
+                                               _stream(stream)))
     return L
 
 

@@ -321,3 +321,56 @@ def test_chain_plan_is_the_oracles_transition_plan():
     for cfg in C.CONFIGS.values():
         for ch in cfg.chains:
             assert C.plan_chain(ch) == O.transition_blocks(ch.layers), ch.name
+
+
+# ------------------------------------------------------------------ the paper's single order (f2)
+
+def test_library_orders_and_matrices_match_the_oracle():
+    """The library builds the same M_H, m(C) and H~_m as the oracle (two
+    independent implementations of the supplementary's constructions under
+    the same choice rule)."""
+    for c in range(1, 700):
+        assert H.hadamard_order(c) == O.hadamard_order(c), c
+    orders = O.supported_orders(1024)
+    for m in [k for k in sorted(orders) if k <= 512] + [576, 640, 768, 1024]:
+        assert np.array_equal(H.hadamard_matrix(m).astype(np.int64), O.hadamard_of_order(m, orders)), m
+    with pytest.raises(H.HatqError):
+        H.hadamard_matrix(100)                     # not in M_H (Paley needs a prime q)
+
+
+ORDER_CASES = [
+    ("dh5x5s2_c192_m192", C.layer("a", 192, 192, 5, 2, 2, "DH", "relu", hb_in=64), 0),
+    ("dh3x3_c190_m192_pad", C.layer("a", 190, 64, 3, 1, 1, "DH", "none", hb_in=2), 0),
+    ("dh3x3_c320_m320_kron", C.layer("a", 320, 640, 3, 1, 1, "DH", "relu", hb_in=64), 128),
+    ("dh3x3_c224_m224_next32", C.layer("a", 224, 128, 3, 1, 1, "DH", "relu", hb_in=32), 32),
+]
+
+
+@pytest.mark.parametrize("case", ORDER_CASES, ids=lambda c: c[0])
+def test_order_host_prepare_matches_oracle_bit_exact(case):
+    name, L, hb_next = case
+    m = O.hadamard_order(L.c_in)
+    w, b = I.weights(L.c_out, L.k, L.k, L.c_in, seed=61), I.bias(L.c_out, seed=62)
+    desc = H.make_desc(L.c_in, L.c_out, L.k, L.stride, L.pad, "DH")
+    got = H.prepare_weights_order_host(desc, w, b, 0.07, 0.05, L.act, hb_next)
+    ref = O.prepare_layer(w, b, "DH", 0, 0, 0.07, 0.05, L.act, hb_next, False, L.stride, L.pad, order_in=m)
+    dop = H.order_desc(desc)
+    assert dop.c_in == m and dop.hb_in == m
+    assert np.array_equal(got.w_i8, _oracle_packed(ref, dop, got.w_i8.shape[1]))
+    assert np.array_equal(got.b_int, ref.b_int)
+    assert got.shift == ref.n and np.array_equal(got.mult.astype(np.int64), ref.M)
+
+
+def test_order_layers_reject_what_they_do_not_cover(lib):
+    w = np.zeros((64, 3, 3, 192), np.float32)
+    with pytest.raises(H.HatqError) as e:          # a block prepare with a non-power-of-two block
+        H.prepare_weights_host(H.make_desc(192, 64, 3, 1, 1, "DH", hb_in=192), w, None, 0.1, 0.1)
+    assert e.value.status == H.ERR_INVALID_ARG
+    with pytest.raises(H.HatqError) as e:          # the single order is built for DH layers
+        H.prepare_weights_order_host(H.make_desc(192, 64, 3, 1, 1, "WH", hb_out=64), w, None, 0.1, 0.1)
+    assert e.value.status == H.ERR_UNSUPPORTED
+    w_elems, ch = H.prepared_sizes(H.ConvDesc(190, 192, 1, 1, 1, 0, H.TRANSFORM, 0, 0))
+    assert ch == 192 and w_elems == 192 * 192      # 1x1 with c = 190 -> packed reduction 192
+    for bad in (H.ConvDesc(192, 192, 3, 3, 1, 1, H.TRANSFORM, 0, 0), H.ConvDesc(192, 100, 1, 1, 1, 0, H.TRANSFORM, 0, 0)):
+        with pytest.raises(H.HatqError):
+            H.prepared_sizes(bad)
