@@ -53,11 +53,12 @@ def parse():
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="cfg4",
-                   choices=["cfg4", "cfg2", "cfg1", "fwht", "profile", "int8mm", "orders"],
+                   choices=["cfg4", "cfg2", "cfg1", "fwht", "profile", "int8mm", "orders", "decoder"],
                    help="fwht: the INT8 transform+requantize pass alone on the config-4 ga2 input; "
                         "profile: the range-expansion profiling pass on the same tensor; "
                         "int8mm: torch._int_mm 8192^3, the library INT8 GEMM as a reference point; "
-                        "orders: the paper's order-192 transform layer and ga2 in that basis at batch 8")
+                        "orders: the paper's order-192 transform layer and ga2 in that basis at batch 8; "
+                        "decoder: a synthesis-side transposed 5x5 s2 layer and a sub-pixel layer at batch 8")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--layer", default="", help="time one layer of the config-4 chains (e.g. ga2, h1, s0a)")
@@ -344,6 +345,43 @@ def run_orders_mode(args, cfg, scales):
         "peaks": {"bf16_tflops": tc, "hbm_gbs": hbm}}), flush=True)
 
 
+def run_decoder_mode(args):
+    """Decoder-side operators at the config-4 latent size (batch 8): a
+    synthesis transposed convolution 320 -> 192 (5x5, stride 2, pad 2, output
+    padding 1, WH 64 output block, ReLU) on the 8 x 135 x 240 latent, and a
+    sub-pixel layer 192 -> 768 (3x3, DH 64, ReLU) with factor 2 on its
+    8 x 270 x 480 output. Random INT8 operands, CUDA events."""
+    import torch
+    from paper_2608_01653_gb300 import hatq as H
+    H.load()
+    peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
+    tc = peaks.get("bf16_tflops", FALLBACK_BF16_TFLOPS)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(13)
+    n, h, w = 8, 135, 240
+    Lt = C.layer("gs1", 320, 192, 5, 2, 2, "WH", "relu", hb_out=64)
+    T = H.prepare_weights_transposed(H.desc_from_spec(Lt), 1, I.weights(192, 5, 5, 320, 31), I.bias(192, 32), 0.1,
+                                     0.05, "relu", 0)
+    x = torch.randint(-127, 128, (n, h, w, 320), dtype=torch.int8, device="cuda", generator=g)
+    y = torch.empty(T.out_shape(n, h, w), dtype=torch.int8, device="cuda")
+    t_ms = time_events(lambda: H.conv_transpose2d_i8(x, T, y=y), args.steps, args.warmup)
+    _, ho, wo, _ = y.shape
+    t_flops = 2 * n * h * w * 320 * 192 * 25                   # every input pixel meets every tap once
+    Ls = C.layer("gs2", 192, 768, 3, 1, 1, "DH", "relu", hb_in=64)
+    P = H.prepare_weights(H.desc_from_spec(Ls), I.weights(768, 3, 3, 192, 33), I.bias(768, 34), 0.1, 0.05, "relu", 0)
+    z = torch.empty((n, ho * 2, wo * 2, 192), dtype=torch.int8, device="cuda")
+    s_ms = time_events(lambda: H.conv2d_i8_subpixel(y, P, 2, y=z), args.steps, args.warmup)
+    H.sync_status()
+    s_flops = 2 * n * ho * wo * 768 * 9 * 192
+    print(json.dumps({
+        "mode": "decoder", "batch": n,
+        "transposed": {"layer": "320->192 5x5 s2 p2 q1 WH64 ReLU", "in_hw": [h, w], "out_hw": [ho, wo], "ms": t_ms,
+                       "tflops": t_flops / (t_ms / 1000) / 1e12, "frac": t_flops / (tc * 1e12) * 1000 / t_ms},
+        "subpixel": {"layer": "192->768 3x3 DH64 ReLU, r = 2", "in_hw": [ho, wo], "out_hw": [2 * ho, 2 * wo],
+                     "ms": s_ms, "tflops": s_flops / (s_ms / 1000) / 1e12, "frac": s_flops / (tc * 1e12) * 1000 / s_ms},
+        "peak_bf16_burst": tc}), flush=True)
+
+
 def run_int8mm_mode(args):
     """torch._int_mm (the library INT8 GEMM, int32 output) on 8192^3, CUDA
     events: the measured INT8 tensor-core reference point of this GPU."""
@@ -384,7 +422,7 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile", "int8mm", "orders")
+    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile", "int8mm", "orders", "decoder")
                                   else args.workload)
     if args.impl == "reference":
         run_reference(args, cfg, scales)
@@ -403,6 +441,9 @@ def main():
         return
     if args.workload == "orders":
         run_orders_mode(args, cfg, scales)
+        return
+    if args.workload == "decoder":
+        run_decoder_mode(args)
         return
 
     import torch

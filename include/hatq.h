@@ -340,6 +340,59 @@ hatq_status hatq_prepare_weights_order_host(const hatq_conv_desc *d, const float
  */
 hatq_status hatq_prepare_order_transform(int c, float s_in, float s_out, hatq_prepared *out, hatq_stream stream);
 
+/*
+ * Decoder-side operators (synthesis transforms). A transposed convolution and
+ * a sub-pixel convolution are linear operators Y = X W^T like the analysis
+ * convolutions (Eq. linear_operator), so the DH / WH weight transforms and
+ * the integer transition apply unchanged.
+ *
+ * Transposed convolution with kernel kh x kw, stride s (1 or 2), padding p and
+ * output padding q (0 <= q < s): input pixel (iy, ix) contributes
+ * x W[:, ky, kx, :]^T to output pixel (iy s + ky - p, ix s + kx - p); the
+ * output is ho = (h - 1) s - 2 p + kh + q rows (likewise wo). It runs as s^2
+ * stride-1 sub-convolutions, one per output parity class (py, px): class
+ * pixels (s r + py, s c + px) take the taps ky = py + p (mod s) in decreasing
+ * order, kx likewise, and each class writes its pixels in place (the output
+ * index remap is in the copy-out). kh, kw >= s.
+ */
+#define HATQ_MAX_TRANSPOSED_CLASSES 4
+typedef struct {
+    hatq_conv_desc d;      /* the transposed convolution (stride s, padding p, form and blocks as for a conv) */
+    int out_pad;           /* q, set by the caller */
+    int classes;           /* written: s * s */
+    int pad_y[HATQ_MAX_TRANSPOSED_CLASSES];   /* written: the sub-convolutions' row / column offsets: class */
+    int pad_x[HATQ_MAX_TRANSPOSED_CLASSES];   /* pixel r reads input row r - pad_y + j at its tap j (may be < 0) */
+    hatq_prepared sub[HATQ_MAX_TRANSPOSED_CLASSES];   /* class py * s + px; the caller sets each one's six
+                                                         device pointers (sizes from hatq_transposed_sizes) */
+} hatq_prepared_transposed;
+
+/* Device buffer sizes of class cls (0 <= cls < s * s) of a transposed
+ * convolution: w_elems for w_i8 / w_f16, ch_elems (= c_out) for the others. */
+hatq_status hatq_transposed_sizes(const hatq_conv_desc *d, int cls, size_t *w_elems, size_t *ch_elems);
+
+/* Offline preparation of a transposed convolution: the weights are transformed
+ * and quantized exactly as by hatq_prepare_weights (per-output-channel scales,
+ * bias codes and (M, n) over the whole kernel), then each class's taps are
+ * packed into its sub-layer. Same arguments and rules as hatq_prepare_weights;
+ * out->d and out->out_pad are the caller's. Synchronizes `stream`. */
+hatq_status hatq_prepare_weights_transposed(const hatq_conv_desc *d, int out_pad, const float *w_ohwi, const float *bias,
+                                            float s_x, float s_y, int act, int hb_next, int out_f32,
+                                            hatq_prepared_transposed *out, hatq_stream stream);
+
+/* The transposed convolution with the fused requantize epilogue on its INT8
+ * operand x [n][h][w][c_in]: y [n][ho][wo][c_out], int8 or float32 as
+ * prepared. s^2 launches on `stream`. */
+hatq_status hatq_conv_transpose2d_i8(const int8_t *x, int n, int h, int w, const hatq_prepared_transposed *T, void *y,
+                                     hatq_stream stream);
+
+/* hatq_conv2d_i8 followed by the sub-pixel rearrangement with factor r
+ * (2 <= r <= 4): channel c r^2 + i r + j of output pixel (oy, ox) is written
+ * to channel c of pixel (oy r + i, ox r + j) of y [n][ho r][wo r][c_out / r^2],
+ * in the copy-out. INT8 output only; c_out and the layer's output tile must
+ * hold whole 16-channel groups per sub-pixel (HATQ_ERR_UNSUPPORTED otherwise). */
+hatq_status hatq_conv2d_i8_subpixel(const int8_t *x, int n, int h, int w, const hatq_prepared *L, int r, void *y,
+                                    hatq_stream stream);
+
 /* Layer-wise strategy selection (Eqs. hadamard_sensitivity,
  * layerwise_hadamard_selection) from the per-image indicators of
  * hatq_profile_range.

@@ -788,7 +788,19 @@ hatq_status hatq_quantize_act(const void *x, int x_kind, float s_in, int n, int 
     return HATQ_OK;
 }
 
-hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prepared *L, void *y, hatq_stream stream) {
+}  // extern "C"
+
+namespace {
+
+// Where a launch's output pixels come from and go to (see ConvArgs): a plain
+// convolution, one output parity class of a transposed convolution, or a
+// convolution followed by the sub-pixel rearrangement.
+struct OutGrid {
+    int pad_y, pad_x, ho, wo, y_h, y_w, ostride, ooy, oox, d2s;
+};
+
+hatq_status conv_launch(const int8_t *x, int n, int h, int w, const hatq_prepared *L, void *y, hatq_stream stream,
+                        const OutGrid *og) {
     if (!L) return fail(HATQ_ERR_INVALID_ARG, "null layer");
     if (n == 0 && h >= 1 && w >= 1) return HATQ_OK;                    // empty batch: nothing to do
     if (!x || !y) return fail(HATQ_ERR_INVALID_ARG, "null argument");
@@ -797,10 +809,17 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     hatq_status st = check_desc(d);
     if (st != HATQ_OK) return st;
     if (n < 0 || h < 1 || w < 1) return fail(HATQ_ERR_INVALID_ARG, "bad input shape");
-    const int ho = (h + 2 * d->pad - d->kh) / d->stride + 1;
-    const int wo = (w + 2 * d->pad - d->kw) / d->stride + 1;
-    if (h + 2 * d->pad < d->kh || w + 2 * d->pad < d->kw || ho < 1 || wo < 1)
-        return fail(HATQ_ERR_INVALID_ARG, "input smaller than the kernel");
+    int ho, wo;
+    if (og) {
+        ho = og->ho;
+        wo = og->wo;
+    } else {
+        ho = (h + 2 * d->pad - d->kh) / d->stride + 1;
+        wo = (w + 2 * d->pad - d->kw) / d->stride + 1;
+        if (h + 2 * d->pad < d->kh || w + 2 * d->pad < d->kw || ho < 1 || wo < 1)
+            return fail(HATQ_ERR_INVALID_ARG, "input smaller than the kernel");
+    }
+    if (ho < 1 || wo < 1) return HATQ_OK;
     if ((long long)n * h * w * d->c_in >= (1LL << 40)) return fail(HATQ_ERR_UNSUPPORTED, "input too large");
     if (n == 0) return HATQ_OK;
     Geometry g;
@@ -811,12 +830,29 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     hatq::ConvArgs a{};
     a.n = n; a.h = h; a.w = w; a.c = d->c_in;
     a.ho = ho; a.wo = wo; a.co = d->c_out;
-    a.kh = d->kh; a.kw = d->kw; a.stride = d->stride; a.pad = d->pad;
+    a.kh = d->kh; a.kw = d->kw; a.stride = d->stride;
+    a.pad_y = og ? og->pad_y : d->pad;
+    a.pad_x = og ? og->pad_x : d->pad;
+    a.y_h = og ? og->y_h : ho;
+    a.y_w = og ? og->y_w : wo;
+    a.ostride = og ? og->ostride : 1;
+    a.ooy = og ? og->ooy : 0;
+    a.oox = og ? og->oox : 0;
+    a.d2s = og ? og->d2s : 0;
     choose_mtile(ho, wo, d->stride, &a.tw, &a.th);
     a.tiles_w = (wo + a.tw - 1) / a.tw;
     a.tiles_h = (ho + a.th - 1) / a.th;
     if ((long long)n * a.tiles_w * a.tiles_h >= (1LL << 31)) return fail(HATQ_ERR_UNSUPPORTED, "grid too large");
     a.n_t = g.n_t;
+    if (a.d2s) {
+        const int r2 = a.d2s * a.d2s;
+        if (L->out_f32) return fail(HATQ_ERR_UNSUPPORTED, "the sub-pixel rearrangement is built for INT8 output");
+        if (L->hb_next)   // the next layer's channel axis is the rearranged one, not this layer's output axis
+            return fail(HATQ_ERR_UNSUPPORTED, "a sub-pixel layer takes no fused next-layer transform");
+        if (d->c_out % r2 || a.n_t % (16 * r2))
+            return fail(HATQ_ERR_UNSUPPORTED, "sub-pixel factor %d needs c_out %% r^2 == 0 and an output tile (%d "
+                                              "channels) of whole 16-channel groups per sub-pixel", a.d2s, a.n_t);
+    }
     a.num_kb = g.k_pad / 64;
     a.cin_kb = g.cin_pad / 64;
     a.gather = g.gather;
@@ -920,6 +956,146 @@ hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prep
     }
     cudaError_t e = hatq::launch_conv(tmA, tmB, a, smem_bytes, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "convolution launch");
+    return HATQ_OK;
+}
+
+// Output parity class p of a transposed convolution (kernel k, stride s,
+// padding pad): its taps are ky = p + pad (mod s); sub-convolution tap j is
+// kernel tap ky_max - s j and reads input row r + j - off for class pixel r,
+// with off = (ky_max - p - pad) / s.
+struct TClass {
+    int taps, ky_max, off;
+};
+
+TClass transposed_class(int k, int s, int pad, int p) {
+    for (int ky = k - 1; ky >= 0; --ky)
+        if (((ky - p - pad) % s + s) % s == 0) return TClass{ky / s + 1, ky, (ky - p - pad) / s};
+    return TClass{0, 0, 0};
+}
+
+hatq_status transposed_sub_desc(const hatq_conv_desc *d, int cls, hatq_conv_desc *sub, TClass *ty, TClass *tx) {
+    hatq_status st = check_desc(d);
+    if (st != HATQ_OK) return st;
+    if (d->form == HATQ_TRANSFORM || (d->form == HATQ_DH && !pow2(d->hb_in)))
+        return fail(HATQ_ERR_UNSUPPORTED, "transposed convolutions take DH / WH layers with block transforms");
+    const int s = d->stride;
+    if (d->kh < s || d->kw < s) return fail(HATQ_ERR_UNSUPPORTED, "a transposed convolution needs kh, kw >= stride");
+    if (cls < 0 || cls >= s * s) return fail(HATQ_ERR_INVALID_ARG, "class %d out of range for stride %d", cls, s);
+    *ty = transposed_class(d->kh, s, d->pad, cls / s);
+    *tx = transposed_class(d->kw, s, d->pad, cls % s);
+    *sub = *d;
+    sub->kh = ty->taps;
+    sub->kw = tx->taps;
+    sub->stride = 1;
+    sub->pad = 0;
+    return HATQ_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+hatq_status hatq_conv2d_i8(const int8_t *x, int n, int h, int w, const hatq_prepared *L, void *y, hatq_stream stream) {
+    return conv_launch(x, n, h, w, L, y, stream, nullptr);
+}
+
+hatq_status hatq_conv2d_i8_subpixel(const int8_t *x, int n, int h, int w, const hatq_prepared *L, int r, void *y,
+                                    hatq_stream stream) {
+    if (!L) return fail(HATQ_ERR_INVALID_ARG, "null layer");
+    if (r < 2 || r > 4) return fail(HATQ_ERR_INVALID_ARG, "sub-pixel factor must be 2..4");
+    const hatq_conv_desc *d = &L->d;
+    if (h < 1 || w < 1) return fail(HATQ_ERR_INVALID_ARG, "bad input shape");
+    const int ho = (h + 2 * d->pad - d->kh) / d->stride + 1, wo = (w + 2 * d->pad - d->kw) / d->stride + 1;
+    if (h + 2 * d->pad < d->kh || w + 2 * d->pad < d->kw || ho < 1 || wo < 1)
+        return fail(HATQ_ERR_INVALID_ARG, "input smaller than the kernel");
+    const OutGrid og{d->pad, d->pad, ho, wo, ho, wo, 1, 0, 0, r};
+    return conv_launch(x, n, h, w, L, y, stream, &og);
+}
+
+hatq_status hatq_transposed_sizes(const hatq_conv_desc *d, int cls, size_t *w_elems, size_t *ch_elems) {
+    hatq_conv_desc sub;
+    TClass ty, tx;
+    hatq_status st = transposed_sub_desc(d, cls, &sub, &ty, &tx);
+    if (st != HATQ_OK) return st;
+    return hatq_prepared_sizes(&sub, w_elems, ch_elems);
+}
+
+hatq_status hatq_prepare_weights_transposed(const hatq_conv_desc *d, int out_pad, const float *w_ohwi, const float *bias,
+                                            float s_x, float s_y, int act, int hb_next, int out_f32,
+                                            hatq_prepared_transposed *out, hatq_stream stream) {
+    if (!out) return fail(HATQ_ERR_INVALID_ARG, "null output struct");
+    hatq_conv_desc sub0;
+    TClass ty, tx;
+    hatq_status st = transposed_sub_desc(d, 0, &sub0, &ty, &tx);
+    if (st != HATQ_OK) return st;
+    const int s = d->stride;
+    if (out_pad < 0 || out_pad >= s) return fail(HATQ_ERR_INVALID_ARG, "output padding must be in [0, stride)");
+    if (act == HATQ_ACT_SILU || act == HATQ_ACT_GELU)
+        return fail(HATQ_ERR_UNSUPPORTED, "transposed layers take the homogeneous transition (none / ReLU)");
+    Geometry gf;
+    if ((st = validate_prepare(d, w_ohwi, s_x, s_y, act, hb_next, out_f32, &gf)) != HATQ_OK) return st;
+    for (int c = 0; c < s * s; ++c)
+        if ((st = check_out_buffers(&out->sub[c])) != HATQ_OK) return st;
+    // the whole kernel, transformed and quantized once
+    HostLayer full(d->c_out, gf.k_pad);
+    st = prepare_core(d, w_ohwi, bias, s_x, s_y, act, hb_next, out_f32, nullptr, 0, full.w_i8.data(), full.w_f16.data(),
+                      full.b_int.data(), full.mult.data(), full.deq.data(), full.s_w.data(), &full.shift);
+    if (st != HATQ_OK) return st;
+    const int ci = d->c_in, co = d->c_out;
+    auto full_index = [&](int ky, int kx, int c) -> long long {
+        return gf.gather ? (long long)ky * gf.seg + (long long)kx * ci + c : (long long)(ky * d->kw + kx) * gf.cin_pad + c;
+    };
+    for (int cls = 0; cls < s * s; ++cls) {
+        hatq_conv_desc sub;
+        if ((st = transposed_sub_desc(d, cls, &sub, &ty, &tx)) != HATQ_OK) return st;
+        Geometry gs;
+        if ((st = geometry(&sub, hb_next, &gs)) != HATQ_OK) return st;
+        HostLayer hs(co, gs.k_pad);
+        hs.b_int = full.b_int;
+        hs.mult = full.mult;
+        hs.deq = full.deq;
+        hs.s_w = full.s_w;
+        hs.shift = full.shift;
+        for (size_t k = 0; k < hs.w_f16.size(); ++k) hs.w_f16[k] = f16_bits(0);
+        for (int o = 0; o < co; ++o)
+            for (int j = 0; j < ty.taps; ++j)
+                for (int l = 0; l < tx.taps; ++l)
+                    for (int c = 0; c < ci; ++c) {
+                        const long long src = (long long)o * gf.k_pad + full_index(ty.ky_max - s * j, tx.ky_max - s * l, c);
+                        const long long dst = (long long)o * gs.k_pad +
+                                              (gs.gather ? (long long)j * gs.seg + (long long)l * ci + c
+                                                         : (long long)(j * tx.taps + l) * gs.cin_pad + c);
+                        hs.w_i8[dst] = full.w_i8[src];
+                        hs.w_f16[dst] = full.w_f16[src];
+                    }
+        if ((st = upload_layer(sub, gs, hs, act, hb_next, out_f32, s_x, s_y, nullptr, &out->sub[cls], stream)) != HATQ_OK)
+            return st;
+        out->pad_y[cls] = ty.off;
+        out->pad_x[cls] = tx.off;
+    }
+    out->d = *d;
+    out->out_pad = out_pad;
+    out->classes = s * s;
+    return HATQ_OK;
+}
+
+hatq_status hatq_conv_transpose2d_i8(const int8_t *x, int n, int h, int w, const hatq_prepared_transposed *T, void *y,
+                                     hatq_stream stream) {
+    if (!T) return fail(HATQ_ERR_INVALID_ARG, "null layer");
+    const int s = T->d.stride;
+    if (s < 1 || s > 2 || T->classes != s * s) return fail(HATQ_ERR_INVALID_ARG, "transposed layer is not prepared");
+    if (h < 1 || w < 1 || n < 0) return fail(HATQ_ERR_INVALID_ARG, "bad input shape");
+    const int ho = (h - 1) * s - 2 * T->d.pad + T->d.kh + T->out_pad;
+    const int wo = (w - 1) * s - 2 * T->d.pad + T->d.kw + T->out_pad;
+    if (ho < 1 || wo < 1) return fail(HATQ_ERR_INVALID_ARG, "empty output");
+    for (int cls = 0; cls < s * s; ++cls) {
+        const int py = cls / s, px = cls % s;
+        const int hc = ho > py ? (ho - py + s - 1) / s : 0, wc = wo > px ? (wo - px + s - 1) / s : 0;
+        if (!hc || !wc) continue;
+        const OutGrid og{T->pad_y[cls], T->pad_x[cls], hc, wc, ho, wo, s, py, px, 0};
+        hatq_status st = conv_launch(x, n, h, w, &T->sub[cls], y, stream, &og);
+        if (st != HATQ_OK) return st;
+    }
     return HATQ_OK;
 }
 

@@ -668,7 +668,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         tma_load_2d(st + a.b_off + u * a.b_bytes, &tmB, full_bar(s), (kb0 + u) * kBlockK, n0);
                         if (!a.gather) {
                             tma_load_4d(st + a.raw_off + u * 8192, &tmA, full_bar(s), cb * kBlockK,
-                                        wo0 * a.stride + kx - a.pad, ho0 * a.stride + ky - a.pad, img);
+                                        wo0 * a.stride + kx - a.pad_x, ho0 * a.stride + ky - a.pad_y, img);
                             if (++cb == a.cin_kb) {
                                 cb = 0;
                                 if (++kx == a.kw) { kx = 0; ++ky; }
@@ -831,12 +831,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tile_coords(j, img, ho0, wo0, n0);
                 asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // previous window consumed
                 if (ok) {
-                    const int ix_lo = wo0 * a.stride - a.pad;
+                    const int ix_lo = wo0 * a.stride - a.pad_x;
                     const int row_b = a.win_w * a.c;
                     const int b_lo = max(0, -ix_lo) * a.c, b_hi = min(a.win_w, a.w - ix_lo) * a.c;
                     // per row, all of a thread's loads are issued before its stores
                     for (int r = 0; r < a.win_h; ++r) {
-                        const int iy = ho0 * a.stride - a.pad + r;
+                        const int iy = ho0 * a.stride - a.pad_y + r;
                         const bool row_in = iy >= 0 && iy < a.h;
                         const int8_t *src = a.x + (((long long)img * a.h + (row_in ? iy : 0)) * a.w + ix_lo) * a.c;
                         for (int b0 = m; b0 < row_b; b0 += 8 * kConvThreads) {
@@ -973,7 +973,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (a.out_f32) {
                     const int oy = ho0 + row / a.tw, ox = wo0 + row % a.tw;
                     if (oy < a.ho && ox < a.wo)
-                        e.gout = static_cast<float *>(a.y) + (((long long)img * a.ho + oy) * a.wo + ox) * a.co + n0;
+                        e.gout = static_cast<float *>(a.y) + (((long long)img * a.y_h + oy * a.ostride + a.ooy) * a.y_w +
+                                                              ox * a.ostride + a.oox) * a.co + n0;
                 }
                 if (G == 128) {
                     // n_t == 128, nbuf == 1: the warpgroups share the group; the shared-memory
@@ -999,9 +1000,30 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int r = jj / cpr, c = jj - r * cpr;
                     const int oy = ho0 + r / a.tw, ox = wo0 + r % a.tw;
                     if (oy < a.ho && ox < a.wo) {
-                        const long long pix = ((long long)img * a.ho + oy) * a.wo + ox;
-                        const int4 v = *reinterpret_cast<const int4 *>(stage_tile + (size_t)r * a.row_stride + c * 16);
-                        *reinterpret_cast<int4 *>(static_cast<uint8_t *>(a.y) + (pix * a.co + n0) * esz + c * 16) = v;
+                        const int gy = oy * a.ostride + a.ooy, gx = ox * a.ostride + a.oox;
+                        const uint8_t *src = stage_tile + (size_t)r * a.row_stride;
+                        if (!a.d2s) {
+                            const long long pix = ((long long)img * a.y_h + gy) * a.y_w + gx;
+                            const int4 v = *reinterpret_cast<const int4 *>(src + c * 16);
+                            *reinterpret_cast<int4 *>(static_cast<uint8_t *>(a.y) + pix * a.co + n0 + c * 16) = v;
+                        } else {
+                            // sub-pixel rearrangement: channel cd r^2 + i r + j of pixel (gy, gx) goes to
+                            // channel cd of pixel (gy r + i, gx r + j); chunk c holds 16 destination channels
+                            // of one (i, j), gathered from the tile row with stride r^2
+                            const int rr = a.d2s, r2 = rr * rr, per = cpr / r2;
+                            const int g = c / per, q = c - g * per, i = g / rr, j = g - i * rr;
+                            const uint8_t *s0 = src + (16 * q) * r2 + i * rr + j;
+                            uint32_t wd[4];
+#pragma unroll
+                            for (int k = 0; k < 4; ++k)
+                                wd[k] = (uint32_t)s0[(4 * k) * r2] | ((uint32_t)s0[(4 * k + 1) * r2] << 8) |
+                                        ((uint32_t)s0[(4 * k + 2) * r2] << 16) | ((uint32_t)s0[(4 * k + 3) * r2] << 24);
+                            const int cd = a.co / r2;
+                            const long long pix =
+                                ((long long)img * a.y_h * rr + gy * rr + i) * ((long long)a.y_w * rr) + gx * rr + j;
+                            *reinterpret_cast<int4 *>(static_cast<uint8_t *>(a.y) + pix * cd + n0 / r2 + 16 * q) =
+                                make_int4((int)wd[0], (int)wd[1], (int)wd[2], (int)wd[3]);
+                        }
                     }
                 }
                 if (nbuf == 2) asm volatile("bar.sync %0, 128;" ::"r"(2 + wg) : "memory");

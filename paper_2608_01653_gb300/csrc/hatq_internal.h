@@ -57,8 +57,12 @@ cudaError_t launch_act_dynamic(const ActQuantArgs &a, float s_in, float *s_used,
 // ---------------------------------------------------------------- conv
 struct ConvArgs {
     int n, h, w, c;
-    int ho, wo, co;
-    int kh, kw, stride, pad;
+    int ho, wo, co;                  // output pixels this launch computes (a sub-convolution's own grid)
+    int kh, kw, stride, pad_y, pad_x;   // input row / column of output (oy, ox), tap (ky, kx): oy s + ky - pad_y
+    // where output pixel (oy, ox) goes: pixel (oy ostride + ooy, ox ostride + oox) of a [n][y_h][y_w][co]
+    // tensor (transposed convolutions write one output parity class per launch); with d2s = r >= 2 the
+    // channels are rearranged depth-to-space into a [n][y_h r][y_w r][co / r^2] tensor
+    int y_h, y_w, ostride, ooy, oox, d2s;
     int tw, th, tiles_w, tiles_h;    // output tile: tw x th pixels (tw * th == 128)
     int n_t;                         // output channels per tile
     int num_kb;                      // 64-wide reduction blocks

@@ -48,6 +48,15 @@ class PreparedStruct(ctypes.Structure):
                 ("reserved", ctypes.c_int), ("mult_in", ctypes.c_longlong), ("lut", ctypes.c_int8 * 256)]
 
 
+MAX_TRANSPOSED_CLASSES = 4
+
+
+class PreparedTransposedStruct(ctypes.Structure):
+    _fields_ = [("d", ConvDesc), ("out_pad", ctypes.c_int), ("classes", ctypes.c_int),
+                ("pad_y", ctypes.c_int * MAX_TRANSPOSED_CLASSES), ("pad_x", ctypes.c_int * MAX_TRANSPOSED_CLASSES),
+                ("sub", PreparedStruct * MAX_TRANSPOSED_CLASSES)]
+
+
 _LIB = None
 _P = ctypes.c_void_p
 _I = ctypes.c_int
@@ -89,6 +98,12 @@ def load(build: bool = True) -> ctypes.CDLL:
             "hatq_prepare_weights_order_host": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _I, _I, _I,
                                                      _P, _P, _P, _P, _P, _P, ctypes.POINTER(_I)]),
             "hatq_prepare_order_transform": (_I, [_I, _F, _F, ctypes.POINTER(PreparedStruct), _P]),
+            "hatq_transposed_sizes": (_I, [ctypes.POINTER(ConvDesc), _I, ctypes.POINTER(ctypes.c_size_t),
+                                           ctypes.POINTER(ctypes.c_size_t)]),
+            "hatq_prepare_weights_transposed": (_I, [ctypes.POINTER(ConvDesc), _I, _P, _P, _F, _F, _I, _I, _I,
+                                                     ctypes.POINTER(PreparedTransposedStruct), _P]),
+            "hatq_conv_transpose2d_i8": (_I, [_P, _I, _I, _I, ctypes.POINTER(PreparedTransposedStruct), _P, _P]),
+            "hatq_conv2d_i8_subpixel": (_I, [_P, _I, _I, _I, ctypes.POINTER(PreparedStruct), _I, _P, _P]),
             "hatq_layer_noalloc": (_I, [_P, _I, _F, _I, _I, _I, ctypes.POINTER(PreparedStruct), _P, _P]),
             "hatq_version": (_I, []),
         }
@@ -313,6 +328,84 @@ def prepare_order_transform(c: int, s_in, s_out, stream=None, device="cuda") -> 
     _check(load().hatq_prepare_order_transform(int(c), float(s_in), float(s_out), ctypes.byref(L.struct),
                                                _stream(stream)))
     return L
+
+
+class PreparedTransposed:
+    """A prepared transposed convolution: one sub-layer (device buffers + C
+    struct) per output parity class, inside the C struct
+    hatq_prepared_transposed."""
+
+    def __init__(self, desc: ConvDesc, out_pad: int, device="cuda"):
+        torch = _torch()
+        self.desc = desc
+        self.out_pad = out_pad
+        self.struct = PreparedTransposedStruct()
+        self.buffers = []
+        for cls in range(desc.stride * desc.stride):
+            w = ctypes.c_size_t()
+            c = ctypes.c_size_t()
+            _check(load().hatq_transposed_sizes(ctypes.byref(desc), cls, ctypes.byref(w), ctypes.byref(c)))
+            bufs = dict(w_i8=torch.zeros(w.value, dtype=torch.int8, device=device),
+                        w_f16=torch.zeros(w.value, dtype=torch.float16, device=device),
+                        b_int=torch.zeros(c.value, dtype=torch.int32, device=device),
+                        mult=torch.zeros(c.value, dtype=torch.int32, device=device),
+                        deq=torch.zeros(c.value, dtype=torch.float32, device=device),
+                        s_w=torch.zeros(c.value, dtype=torch.float32, device=device))
+            for k, t in bufs.items():
+                setattr(self.struct.sub[cls], k, t.data_ptr())
+            self.buffers.append(bufs)
+
+    @property
+    def c_in(self):
+        return self.desc.c_in
+
+    @property
+    def out_f32(self):
+        return bool(self.struct.sub[0].out_f32)
+
+    def out_shape(self, n, h, w):
+        d = self.desc
+        return (n, (h - 1) * d.stride - 2 * d.pad + d.kh + self.out_pad,
+                (w - 1) * d.stride - 2 * d.pad + d.kw + self.out_pad, d.c_out)
+
+
+def prepare_weights_transposed(desc: ConvDesc, out_pad, w_ohwi, bias, s_x, s_y, act="none", hb_next=0,
+                               out_f32=False, stream=None, device="cuda") -> PreparedTransposed:
+    """hatq_prepare_weights_transposed: a transposed convolution (decoder side)
+    prepared as one stride-1 sub-layer per output parity class."""
+    T = PreparedTransposed(desc, out_pad, device)
+    w = np.ascontiguousarray(w_ohwi, dtype=np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    _check(load().hatq_prepare_weights_transposed(ctypes.byref(desc), int(out_pad), w.ctypes.data,
+                                                  None if b is None else b.ctypes.data, float(s_x), float(s_y),
+                                                  _ACTS.get(act, act), int(hb_next), int(bool(out_f32)),
+                                                  ctypes.byref(T.struct), _stream(stream)))
+    return T
+
+
+def conv_transpose2d_i8(x, T: PreparedTransposed, y=None, stream=None):
+    """hatq_conv_transpose2d_i8 on the INT8 operand x (NHWC)."""
+    n, h, w, c = _check_layer_io(x, IN_OPERAND, T, y)
+    torch = _torch()
+    if y is None:
+        y = torch.empty(T.out_shape(n, h, w), dtype=torch.float32 if T.out_f32 else torch.int8, device=x.device)
+    _check(load().hatq_conv_transpose2d_i8(_ptr(x), n, h, w, ctypes.byref(T.struct), _ptr(y), _stream(stream)))
+    return y
+
+
+def conv2d_i8_subpixel(x, L: "PreparedLayer", r: int, y=None, stream=None):
+    """hatq_conv2d_i8_subpixel: the convolution followed by the sub-pixel
+    (depth-to-space) rearrangement with factor r, in the copy-out."""
+    n, h, w, c = _check_layer_io(x, IN_OPERAND, L, None)
+    _, ho, wo, co = L.out_shape(n, h, w)
+    shape = (n, ho * r, wo * r, co // (r * r))
+    if y is not None:
+        _check_tensor(y, "y", "int8", shape)
+    torch = _torch()
+    if y is None:
+        y = torch.empty(shape, dtype=torch.int8, device=x.device)
+    _check(load().hatq_conv2d_i8_subpixel(_ptr(x), n, h, w, ctypes.byref(L.struct), int(r), _ptr(y), _stream(stream)))
+    return y
 
 
 @dataclass

@@ -374,3 +374,37 @@ def test_order_layers_reject_what_they_do_not_cover(lib):
     for bad in (H.ConvDesc(192, 192, 3, 3, 1, 1, H.TRANSFORM, 0, 0), H.ConvDesc(192, 100, 1, 1, 1, 0, H.TRANSFORM, 0, 0)):
         with pytest.raises(H.HatqError):
             H.prepared_sizes(bad)
+
+
+def test_transposed_struct_mirror_matches_the_c_layout(tmp_path):
+    """The ctypes mirror of hatq_prepared_transposed has the C layout."""
+    import shutil
+    import subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    fields = ["d", "out_pad", "classes", "pad_y", "pad_x", "sub"]
+    src = tmp_path / "tlayout.c"
+    inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
+    src.write_text("#include <stdio.h>\n#include <stddef.h>\n#include \"hatq.h\"\nint main(void) {\n"
+                   "  printf(\"%zu\\n\", sizeof(hatq_prepared_transposed));\n"
+                   + "".join(f"  printf(\"%zu\\n\", offsetof(hatq_prepared_transposed, {f}));\n" for f in fields)
+                   + "  return 0;\n}\n")
+    exe = tmp_path / "tlayout"
+    subprocess.run([cc, "-I", inc, str(src), "-o", str(exe)], check=True, capture_output=True)
+    out = [int(v) for v in subprocess.run([str(exe)], check=True, capture_output=True, text=True).stdout.split()]
+    assert ctypes.sizeof(H.PreparedTransposedStruct) == out[0]
+    for f, off in zip(fields, out[1:]):
+        assert getattr(H.PreparedTransposedStruct, f).offset == off, f
+
+
+@pytest.mark.parametrize("k,s,p,cls,taps", [(5, 2, 2, 0, (3, 3)), (5, 2, 2, 3, (2, 2)), (4, 2, 1, 1, (2, 2)),
+                                            (3, 2, 1, 2, (2, 1)), (3, 1, 1, 0, (3, 3))])
+def test_transposed_class_sizes(k, s, p, cls, taps):
+    """Class (py, px) of a transposed convolution is a stride-1 sub-convolution
+    with the taps ky = py + p (mod s), kx likewise."""
+    d = H.make_desc(64, 128, k, s, p, "DH", hb_in=64)
+    w, c = ctypes.c_size_t(), ctypes.c_size_t()
+    assert H.load().hatq_transposed_sizes(ctypes.byref(d), cls, ctypes.byref(w), ctypes.byref(c)) == H.OK
+    assert c.value == 128 and w.value == 128 * taps[0] * taps[1] * 64
+    assert H.load().hatq_transposed_sizes(ctypes.byref(d), s * s, ctypes.byref(w), ctypes.byref(c)) == H.ERR_INVALID_ARG
