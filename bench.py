@@ -560,7 +560,12 @@ def main():
     traffic = None
     prof = os.path.join(ROOT, "profiles", "conv_cfg4_traffic.json")
     if os.path.exists(prof):
-        traffic = json.load(open(prof)).get("dram_bytes_per_launch")
+        # the captured counters stand for the kernel source they were taken on, and for no later one
+        import hashlib
+        rec = json.load(open(prof))
+        src = os.path.join(ROOT, "paper_2608_01653_gb300", "csrc", "hatq_conv.cu")
+        if hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] == rec.get("kernel_source_sha256_16"):
+            traffic = rec.get("dram_bytes_per_launch")
     roofline = {"bound": "tensor", "achieved": achieved, "peak": tc_peak, "unit": "TFLOP/s", "frac": achieved / tc_peak,
                 "traffic": traffic, "kernel": "hatq conv_kernel (tcgen05 kind::f16, exact INT8)",
                 "launches": n_conv, "avg_launch_ms": conv_ms / max(n_conv, 1), "peak_source": tc_src,
