@@ -115,7 +115,7 @@ typedef struct {
     float s_z;            /* preactivation scale */
     float s_u;            /* activation-output scale */
     int shift_in;         /* n_in of Eq. supp_general_input_scale */
-    int reserved;
+    int in_affine;        /* 1: prepared by hatq_prepare_weights_affine (centred int16 operand, float output) */
     long long mult_in;    /* M_in of Eq. supp_general_input_scale */
     int8_t lut[256];      /* phi_int of Eq. supp_general_activation at z = -127..127 (index z + 127) */
 } hatq_prepared;
@@ -392,6 +392,40 @@ hatq_status hatq_conv_transpose2d_i8(const int8_t *x, int n, int h, int w, const
  * hold whole 16-channel groups per sub-pixel (HATQ_ERR_UNSUPPORTED otherwise). */
 hatq_status hatq_conv2d_i8_subpixel(const int8_t *x, int n, int h, int w, const hatq_prepared *L, int r, void *y,
                                     hatq_stream stream);
+
+/*
+ * Dynamic affine activation quantization (PTQ setting; Eqs. uniform_q,
+ * affine_q; supplementary, affine activation quantization). Per input tensor
+ * the operand v = T x (T the layer's normalized input-side block transform for
+ * DH, the identity for WH) takes
+ *   lo = min(min v, 0), hi = max(max v, 0), s = (hi - lo) / 255,
+ *   z = clamp(round(-lo / s), 0, 255), x_int = clamp(round(v / s) + z, 0, 255)
+ * (a zero range gives s = 1, z = 0), and the convolution runs on the centred
+ * codes x_int - z in [-255, 255], so zero padding is a centred zero. The
+ * output is dequantized: y = phi(H_out(s s_w (.) a + b_bar)).
+ *
+ * hatq_quantize_act_affine: x device fp16 NHWC [n][h][w][c] (c % 16 == 0), hb
+ * the input-side block (1 for WH); y device int16 NHWC centred codes;
+ * params device float[2] written with (s, z); workspace device >= 32 bytes
+ * (reset each call). v is computed with an fp32 butterfly, so codes can differ
+ * from an exact evaluation by one step where v / s lies at a rounding tie.
+ */
+hatq_status hatq_quantize_act_affine(const void *x, int n, int h, int w, int c, int hb, int16_t *y, float *params,
+                                     void *workspace, hatq_stream stream);
+/* A layer for affine activations: the weights, channel scales and transformed
+ * bias of hatq_prepare_weights (any s_x: the activation scale is per input),
+ * float32 output, act HATQ_ACT_NONE or HATQ_ACT_RELU, no next-layer
+ * transform, c_in % 16 == 0. The bias stays real: deq holds b_bar_c / gamma_out
+ * and in_affine is set. Buffers as for hatq_prepare_weights. */
+hatq_status hatq_prepare_weights_affine(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, int act,
+                                        hatq_prepared *out, hatq_stream stream);
+/* The convolution on centred affine codes x (device int16 NHWC [n][h][w][c_in])
+ * with s read from params[0] (device, as written by hatq_quantize_act_affine):
+ * a = sum (x_int - z) w_int exactly (fp32 chunks of 512 products below 2^24,
+ * int32 totals), y = phi(H~_out((s s_w,c / gamma_out) a + b_bar_c / gamma_out))
+ * in float32, device NHWC [n][ho][wo][c_out]. */
+hatq_status hatq_conv2d_affine(const int16_t *x, int n, int h, int w, const hatq_prepared *L, const float *params,
+                               float *y, hatq_stream stream);
 
 /* Layer-wise strategy selection (Eqs. hadamard_sensitivity,
  * layerwise_hadamard_selection) from the per-image indicators of

@@ -835,11 +835,17 @@ def conv_layer_affine(x_real, p: Prepared):
         np.asarray(x_real, dtype=np.float64)
     s, z = affine_params(v)
     centred = quantize_affine(v, s, z) - z
+    return conv_layer_affine_codes(centred, s, p), s, z
+
+
+def conv_layer_affine_codes(centred, s: float, p: Prepared):
+    """The second half of conv_layer_affine: the convolution on centred codes
+    at step s and the dequantized output y = phi(H_out(s s_w (.) a) + b_bar)."""
     acc = conv_codes_wide(centred, p.w_int, p.stride, p.pad)
     t = (s * p.s_w) * acc.astype(np.float64)
     y = transform_real(t, p.hb_out) if p.form == "WH" else t
     y = y + p.bbar if p.form == "DH" else y + transform_real(p.bbar, p.hb_out)
-    return (np.maximum(y, 0.0) if p.act == "relu" else y), s, z
+    return np.maximum(y, 0.0) if p.act == "relu" else y
 
 
 # --------------------------------------------------------------------------

@@ -373,7 +373,7 @@ hatq_status operand_desc(const hatq_conv_desc *d, int order, hatq_conv_desc *op)
 hatq_status prepare_core(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, float s_x, float s_y,
                          int act, int hb_next, int out_f32, GeneralParams *gen, int order, int8_t *w_i8_out,
                          uint16_t *w_f16_out, int32_t *b_int_out, int32_t *mult_out, float *deq_out, float *s_w_out,
-                         int *shift_out) {
+                         int *shift_out, double *bbar_out = nullptr) {
     hatq_conv_desc dop;
     hatq_status st = operand_desc(d, order, &dop);
     if (st != HATQ_OK) return st;
@@ -428,6 +428,8 @@ hatq_status prepare_core(const hatq_conv_desc *d, const float *w_ohwi, const flo
         std::vector<double> b0 = bbar;
         for (int blk = 0; blk < co / hb; ++blk) block_transform(&b0[blk * hb], &bbar[blk * hb], hb, 1);
     }
+    if (bbar_out)
+        for (int o = 0; o < co; ++o) bbar_out[o] = bbar[o];
     // 2. channel-wise symmetric weight quantization, bias codes, bounds
     std::vector<double> s_a(co), rho(co);
     std::vector<long long> abound(co);
@@ -625,7 +627,7 @@ hatq_status upload_layer(const hatq_conv_desc &dop, const Geometry &g, const Hos
     out->s_z = gen ? gen->s_z : 0.f;
     out->s_u = gen ? gen->s_u : 0.f;
     out->shift_in = gen ? gen->shift_in : 0;
-    out->reserved = 0;
+    out->in_affine = 0;
     out->mult_in = gen ? gen->mult_in : 0;
     if (gen) std::memcpy(out->lut, gen->lut, sizeof out->lut);
     else std::memset(out->lut, 0, sizeof out->lut);
@@ -799,8 +801,8 @@ struct OutGrid {
     int pad_y, pad_x, ho, wo, y_h, y_w, ostride, ooy, oox, d2s;
 };
 
-hatq_status conv_launch(const int8_t *x, int n, int h, int w, const hatq_prepared *L, void *y, hatq_stream stream,
-                        const OutGrid *og) {
+hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared *L, void *y, hatq_stream stream,
+                        const OutGrid *og, const float *affine_s = nullptr) {
     if (!L) return fail(HATQ_ERR_INVALID_ARG, "null layer");
     if (n == 0 && h >= 1 && w >= 1) return HATQ_OK;                    // empty batch: nothing to do
     if (!x || !y) return fail(HATQ_ERR_INVALID_ARG, "null argument");
@@ -821,6 +823,11 @@ hatq_status conv_launch(const int8_t *x, int n, int h, int w, const hatq_prepare
     }
     if (ho < 1 || wo < 1) return HATQ_OK;
     if ((long long)n * h * w * d->c_in >= (1LL << 40)) return fail(HATQ_ERR_UNSUPPORTED, "input too large");
+    if ((L->in_affine != 0) != (affine_s != nullptr))
+        return fail(HATQ_ERR_INVALID_ARG, L->in_affine ? "a layer prepared for affine activations runs through "
+                                                         "hatq_conv2d_affine"
+                                                       : "hatq_conv2d_affine needs a layer from "
+                                                         "hatq_prepare_weights_affine");
     if (n == 0) return HATQ_OK;
     Geometry g;
     if ((st = geometry(d, L->hb_next, &g)) != HATQ_OK) return st;
@@ -856,9 +863,11 @@ hatq_status conv_launch(const int8_t *x, int n, int h, int w, const hatq_prepare
     a.num_kb = g.k_pad / 64;
     a.cin_kb = g.cin_pad / 64;
     a.gather = g.gather;
-    a.chunk_kb = 16;
+    // exact fp32 chunks: 1024 products of |x| <= 127 (INT8 codes), 512 of |x| <= 255 (centred affine codes)
+    a.affine = L->in_affine ? 1 : 0;
+    a.chunk_kb = a.affine ? 8 : 16;
     a.b_bytes = a.n_t * 128;
-    a.raw_bytes = g.gather ? 0 : 8192;
+    a.raw_bytes = g.gather ? 0 : (a.affine ? 16384 : 8192);
     a.n_tiles_n = d->c_out / a.n_t;
     {
         const long long nt = (long long)n * a.tiles_w * a.tiles_h * a.n_tiles_n;
@@ -889,7 +898,7 @@ hatq_status conv_launch(const int8_t *x, int n, int h, int w, const hatq_prepare
     const int win_bytes = g.gather ? (a.win_h * a.win_pitch + 16 + 127) & ~127 : 0;
     const int table_bytes = g.gather ? a.num_kb * 8 * 4 : 0;
     const bool general = L->act == HATQ_ACT_SILU || L->act == HATQ_ACT_GELU;
-    const int const_bytes = ((3 * d->c_out * 4 + 127) & ~127) + (general ? 256 : 0);
+    const int const_bytes = ((4 * d->c_out * 4 + 127) & ~127) + (general ? 256 : 0);
     const int fixed = 1024 /* align */ + 8 * (3 * 8 + 9) + 16 + 128 + table_bytes + const_bytes + win_bytes;
     const int budget = 227 * 1024 - 1024 /* static */ - fixed - a.staging_bytes;
     // a stage holds `sub` 64-wide reduction blocks: [weights x sub | INT8 box x sub].
@@ -920,10 +929,14 @@ hatq_status conv_launch(const int8_t *x, int n, int h, int w, const hatq_prepare
     if (g.G == 128 && L->hb_next == 128 && a.staging_bytes < 2 * kTileRows * 64)
         return fail(HATQ_ERR_UNSUPPORTED, "output tile too small for the 128-wide transition exchange");
     if (smem_bytes > 227 * 1024 - 1024) return fail(HATQ_ERR_UNSUPPORTED, "shared memory budget exceeded (%d bytes)", smem_bytes);
-    a.x = x;
+    if (a.affine && g.gather) return fail(HATQ_ERR_UNSUPPORTED, "affine activations need c_in % 16 == 0");
+    a.x = static_cast<const int8_t *>(x);
     a.b_int = L->b_int;
     a.mult = L->mult;
     a.deq = L->deq;
+    a.s_w = L->s_w;
+    a.affine_s = affine_s;
+    a.inv_gamma = d->form == HATQ_WH ? (float)(1.0 / std::sqrt((double)d->hb_out)) : 1.0f;
     a.shift = L->shift;
     a.hb_out = d->form == HATQ_WH ? d->hb_out : 0;
     a.hb_next = L->hb_next;
@@ -931,7 +944,7 @@ hatq_status conv_launch(const int8_t *x, int n, int h, int w, const hatq_prepare
     a.general = general ? 1 : 0;
     a.shift_in = L->shift_in;
     a.mult_in = L->mult_in;
-    a.lut_off = a.const_off + ((3 * d->c_out * 4 + 127) & ~127);
+    a.lut_off = a.const_off + ((4 * d->c_out * 4 + 127) & ~127);
     std::memcpy(a.lut, L->lut, sizeof a.lut);
     a.out_f32 = L->out_f32;
     a.y = y;
@@ -943,13 +956,17 @@ hatq_status conv_launch(const int8_t *x, int n, int h, int w, const hatq_prepare
     if (!g.gather) {
         EncodeTiledFn enc = encode_fn();
         if (!enc) return fail(HATQ_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+        // INT8 codes (64-byte box rows, 64-byte swizzle) or centred int16 affine codes (128-byte rows)
+        const cuuint64_t es = a.affine ? 2 : 1;
         const cuuint64_t dims[4] = {(cuuint64_t)d->c_in, (cuuint64_t)w, (cuuint64_t)h, (cuuint64_t)n};
-        const cuuint64_t strides[3] = {(cuuint64_t)d->c_in, (cuuint64_t)w * d->c_in, (cuuint64_t)h * w * d->c_in};
+        const cuuint64_t strides[3] = {(cuuint64_t)d->c_in * es, (cuuint64_t)w * d->c_in * es,
+                                       (cuuint64_t)h * w * d->c_in * es};
         const cuuint32_t box[4] = {64, (cuuint32_t)(a.tw * d->stride), (cuuint32_t)(a.th * d->stride), 1};
         const cuuint32_t estr[4] = {1, (cuuint32_t)d->stride, (cuuint32_t)d->stride, 1};
-        CUresult r = enc(&tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 4, const_cast<int8_t *>(x), dims, strides, box, estr,
-                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
-                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        CUresult r = enc(&tmA, a.affine ? CU_TENSOR_MAP_DATA_TYPE_UINT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 4,
+                         const_cast<void *>(x), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                         a.affine ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "activation tensor map encoding failed (%d)", (int)r);
     } else {
         tmA = tmB;
@@ -1010,6 +1027,63 @@ hatq_status hatq_conv2d_i8_subpixel(const int8_t *x, int n, int h, int w, const 
         return fail(HATQ_ERR_INVALID_ARG, "input smaller than the kernel");
     const OutGrid og{d->pad, d->pad, ho, wo, ho, wo, 1, 0, 0, r};
     return conv_launch(x, n, h, w, L, y, stream, &og);
+}
+
+hatq_status hatq_prepare_weights_affine(const hatq_conv_desc *d, const float *w_ohwi, const float *bias, int act,
+                                        hatq_prepared *out, hatq_stream stream) {
+    hatq_conv_desc dop;
+    hatq_status st = operand_desc(d, 0, &dop);
+    if (st != HATQ_OK) return st;
+    if (act != HATQ_ACT_NONE && act != HATQ_ACT_RELU)
+        return fail(HATQ_ERR_UNSUPPORTED, "affine layers take no activation or ReLU");
+    if (d->c_in % 16) return fail(HATQ_ERR_UNSUPPORTED, "affine activations need c_in % 16 == 0");
+    Geometry g;
+    if ((st = validate_prepare(&dop, w_ohwi, 1.f, 1.f, act, 0, 1, &g)) != HATQ_OK) return st;
+    if ((st = check_out_buffers(out)) != HATQ_OK) return st;
+    HostLayer hl(dop.c_out, g.k_pad);
+    std::vector<double> bbar(dop.c_out);
+    st = prepare_core(d, w_ohwi, bias, 1.f, 1.f, act, 0, 1, nullptr, 0, hl.w_i8.data(), hl.w_f16.data(), hl.b_int.data(),
+                      hl.mult.data(), hl.deq.data(), hl.s_w.data(), &hl.shift, bbar.data());
+    if (st != HATQ_OK) return st;
+    // the bias stays real-valued (the activation scale is per input): beta_c = b_bar_c / gamma_out
+    const double g_out = d->form == HATQ_WH ? std::sqrt((double)d->hb_out) : 1.0;
+    for (int o = 0; o < dop.c_out; ++o) {
+        hl.b_int[o] = 0;
+        hl.mult[o] = 0;
+        hl.deq[o] = (float)(bbar[o] / g_out);
+    }
+    if ((st = upload_layer(dop, g, hl, act, 0, 1, 1.f, 0.f, nullptr, out, stream)) != HATQ_OK) return st;
+    out->in_affine = 1;
+    out->s_x = 0.f;
+    return HATQ_OK;
+}
+
+hatq_status hatq_quantize_act_affine(const void *x, int n, int h, int w, int c, int hb, int16_t *y, float *params,
+                                     void *workspace, hatq_stream stream) {
+    if (n == 0 && h >= 0 && w >= 0 && c >= 0) return HATQ_OK;
+    if (!x || !y || !params || !workspace) return fail(HATQ_ERR_INVALID_ARG, "null argument");
+    if (!aligned16(x) || !aligned16(y) || !aligned16(workspace))
+        return fail(HATQ_ERR_INVALID_ARG, "input, output and workspace must be 16-byte aligned");
+    if (n < 0 || h < 0 || w < 0 || c < 16 || c % 16) return fail(HATQ_ERR_INVALID_ARG, "shape must be n,h,w >= 0, c % 16 == 0");
+    if (!pow2(hb) || hb > 256 || c % hb) return fail(HATQ_ERR_INVALID_ARG, "hb must be a power of two <= 256 dividing c");
+    const long long total = (long long)n * h * w * c;
+    if (total == 0) return HATQ_OK;
+    hatq::AffineQuantArgs a{};
+    a.x = x;
+    a.y = y;
+    a.total = total;
+    a.hb = hb;
+    a.p = static_cast<hatq::AffineParams *>(workspace);
+    a.params_out = params;
+    cudaError_t e = hatq::launch_act_affine(a, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "affine quantization launch");
+    return HATQ_OK;
+}
+
+hatq_status hatq_conv2d_affine(const int16_t *x, int n, int h, int w, const hatq_prepared *L, const float *params,
+                               float *y, hatq_stream stream) {
+    if (!params) return fail(HATQ_ERR_INVALID_ARG, "null scale");
+    return conv_launch(x, n, h, w, L, y, stream, nullptr, params);
 }
 
 hatq_status hatq_transposed_sizes(const hatq_conv_desc *d, int cls, size_t *w_elems, size_t *ch_elems) {

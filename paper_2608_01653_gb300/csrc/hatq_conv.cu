@@ -185,6 +185,17 @@ __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t
     asm("sub.f16x2 %0, %1, %2;" : "=r"(hi) : "r"(b), "r"(0x64806480u));
 }
 
+// two int16 codes c0 (low half) and c1 in [-255, 255] -> one fp16x2 word,
+// exactly: offset binary c + 32768 minus 32512 gives c + 256 in [1, 511] per
+// half (no borrow between halves), 0x6400 | (c + 256) is 1024 + 256 + c, and
+// subtracting 1280 leaves c.
+__device__ __forceinline__ uint32_t i16x2_to_f16x2(uint32_t w) {
+    const uint32_t t = ((w ^ 0x80008000u) - 0x7F007F00u) | 0x64006400u;
+    uint32_t r;
+    asm("sub.f16x2 %0, %1, %2;" : "=r"(r) : "r"(t), "r"(0x65006500u));
+    return r;
+}
+
 // ------------------------------------------------------------------ epilogue math
 
 __device__ __forceinline__ int requant8(long long v, int n) {
@@ -256,6 +267,7 @@ struct EpiCtx {
     const int *b_int;    // this tile's bias codes, multipliers and dequant factors (shared memory)
     const int *mult;
     const float *deq;
+    const float *biasf;  // float bias added after the scale (dynamic affine input), else zeros
     uint32_t t_acc;      // TMEM address of this warp's lanes, column 0 of the accumulator
     bool int_acc;        // the accumulator holds exact int32 totals (else exact fp32 integers)
     uint8_t *row;        // this thread's row of the shared-memory output tile (INT8 output)
@@ -297,13 +309,14 @@ __device__ __forceinline__ void scale_i64(const EpiCtx &e, int col, const int (&
 }
 __device__ __forceinline__ void scale_f32(const EpiCtx &e, int col, const int (&v)[16], float *t) {
     const float4 *dp = reinterpret_cast<const float4 *>(e.deq + col);
+    const float4 *bp = reinterpret_cast<const float4 *>(e.biasf + col);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        const float4 d = dp[i];
-        t[4 * i] = d.x * (float)v[4 * i];
-        t[4 * i + 1] = d.y * (float)v[4 * i + 1];
-        t[4 * i + 2] = d.z * (float)v[4 * i + 2];
-        t[4 * i + 3] = d.w * (float)v[4 * i + 3];
+        const float4 d = dp[i], b = bp[i];
+        t[4 * i] = d.x * (float)v[4 * i] + b.x;
+        t[4 * i + 1] = d.y * (float)v[4 * i + 1] + b.y;
+        t[4 * i + 2] = d.z * (float)v[4 * i + 2] + b.z;
+        t[4 * i + 3] = d.w * (float)v[4 * i + 3] + b.w;
     }
 }
 
@@ -609,10 +622,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     // bias codes, multipliers and dequant factors of all output channels,
     // staged once per CTA (128-byte aligned, read with 16-byte vector loads)
     int *cb = reinterpret_cast<int *>(bar_area + a.const_off);
+    const float s_aff = a.affine ? *a.affine_s : 0.f;
     for (int c = threadIdx.x; c < a.co; c += kThreads) {
         cb[c] = a.b_int[c];
         cb[a.co + c] = a.mult[c];
-        reinterpret_cast<float *>(cb)[2 * a.co + c] = a.deq[c];
+        reinterpret_cast<float *>(cb)[2 * a.co + c] = a.affine ? s_aff * a.s_w[c] * a.inv_gamma : a.deq[c];
+        reinterpret_cast<float *>(cb)[3 * a.co + c] = a.affine ? a.deq[c] : 0.f;
     }
     int8_t *lut_s = reinterpret_cast<int8_t *>(bar_area + a.lut_off);
     if (a.general)
@@ -667,7 +682,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         if (u >= nsub) break;
                         tma_load_2d(st + a.b_off + u * a.b_bytes, &tmB, full_bar(s), (kb0 + u) * kBlockK, n0);
                         if (!a.gather) {
-                            tma_load_4d(st + a.raw_off + u * 8192, &tmA, full_bar(s), cb * kBlockK,
+                            tma_load_4d(st + a.raw_off + u * a.raw_bytes, &tmA, full_bar(s), cb * kBlockK,
                                         wo0 * a.stride + kx - a.pad_x, ho0 * a.stride + ky - a.pad_y, img);
                             if (++cb == a.cin_kb) {
                                 cb = 0;
@@ -775,6 +790,19 @@ __global__ void __launch_bounds__(kThreads, 1)
             // row m of a 64-wide INT8 box (64 bytes, 16-byte chunks permuted by the
             // 64-byte swizzle) -> 32 columns of fp16 pairs
             auto convert_row = [&](const uint8_t *raw, uint32_t (&h)[32]) {
+                if (a.affine) {
+                    // row m of a 64-wide int16 box (128 bytes, 16-byte chunks permuted by the 128-byte swizzle)
+                    const int sw = m & 7;
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) {
+                        const uint4 v = *reinterpret_cast<const uint4 *>(raw + ((q ^ sw) << 4));
+                        h[4 * q + 0] = i16x2_to_f16x2(v.x);
+                        h[4 * q + 1] = i16x2_to_f16x2(v.y);
+                        h[4 * q + 2] = i16x2_to_f16x2(v.z);
+                        h[4 * q + 3] = i16x2_to_f16x2(v.w);
+                    }
+                    return;
+                }
                 const int sw = (m >> 1) & 3;
                 uint4 v[4];
 #pragma unroll
@@ -787,12 +815,13 @@ __global__ void __launch_bounds__(kThreads, 1)
                     i8x4_to_f16x4(v[q].w, h[8 * q + 6], h[8 * q + 7]);
                 }
             };
+            const int row_in = a.affine ? 128 : 64;     // bytes of one operand row of a 64-wide block
             for (int j = 0; j < my_tiles && ok; ++j) {
                 for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB) {
                     const int nsub = min(SUB, a.num_kb - kb0);
                     ok = __all_sync(0xffffffffu, mbar_wait(full_bar(s), ph, abort_flag, a.err));
                     if (!ok) break;
-                    const uint8_t *raw = smem + (size_t)s * a.stage_bytes + a.raw_off + m * 64;
+                    const uint8_t *raw = smem + (size_t)s * a.stage_bytes + a.raw_off + m * row_in;
                     const uint32_t t_slot = t_lane + (uint32_t)(slot * SUB * 32);
                     uint32_t h[32];
                     convert_row(raw, h);              // the first block is converted before the slot frees up
@@ -802,7 +831,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll 1
                     for (int u = 1; u < SUB; ++u) {
                         if (u >= nsub) break;
-                        convert_row(raw + u * 8192, h);
+                        convert_row(raw + u * a.raw_bytes, h);
                         tmem_st32(t_slot + (uint32_t)(u * 32), h);
                     }
                     tmem_wait_st();
@@ -965,6 +994,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 e.b_int = cb + n0;
                 e.mult = cb + a.co + n0;
                 e.deq = reinterpret_cast<const float *>(cb + 2 * a.co) + n0;
+                e.biasf = reinterpret_cast<const float *>(cb + 3 * a.co) + n0;
                 e.t_acc = t_acc;
                 e.int_acc = nbuf == 1;
                 e.lut = lut_s;

@@ -219,6 +219,108 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
     }
 }
 
+// ------------------------------------------------------------------ dynamic affine (PTQ) activations
+// Eqs. uniform_q, affine_q with the range extended to include zero:
+// lo = min(min v, 0), hi = max(max v, 0), s = (hi - lo) / 255,
+// z = clamp(round(-lo / s), 0, 255), x_int = clamp(round(v / s) + z, 0, 255);
+// the layer consumes the centred codes x_int - z (int16, in [-255, 255]).
+// v = T x is the fp32 butterfly of the FP16 input (T the normalized block
+// transform of a DH layer; the identity for hb = 1).
+
+// order-preserving unsigned key of a float (larger float, larger key)
+__device__ __forceinline__ unsigned int float_key(float f) {
+    const unsigned int b = __float_as_uint(f);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+__device__ __forceinline__ float key_float(unsigned int k) {
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7FFFFFFFu) : ~k);
+}
+
+// MODE 0: range pass (max v, max -v). MODE 1: quantize to centred int16 codes.
+template <int MODE>
+__global__ void __launch_bounds__(kThreads) act_affine_kernel(AffineQuantArgs a) {
+    const int lane = threadIdx.x & 31;
+    const long long warp = ((long long)blockIdx.x * kThreads + threadIdx.x) >> 5;
+    const long long nwarps = ((long long)gridDim.x * kThreads) >> 5;
+    const long long tiles = (a.total + 511) >> 9;
+    const float norm = 1.0f / sqrtf((float)a.hb);     // exact for the power-of-four blocks
+    float vmax = -3.0e38f, vmin = 3.0e38f;
+    float inv_s = 0.f, z = 0.f;
+    if (MODE == 1) {
+        inv_s = a.p->inv_s;
+        z = a.p->z;
+    }
+    for (long long t = warp; t < tiles; t += nwarps) {
+        const long long e0 = (t << 9) + lane * 16;
+        const bool valid = e0 < a.total;
+        int4 v0 = make_int4(0, 0, 0, 0), v1 = make_int4(0, 0, 0, 0);
+        if (valid) {
+            const int4 *p = reinterpret_cast<const int4 *>(static_cast<const __half *>(a.x) + e0);
+            v0 = __ldg(p);
+            v1 = __ldg(p + 1);
+        }
+        float f[16];
+        const uint32_t w[8] = {(uint32_t)v0.x, (uint32_t)v0.y, (uint32_t)v0.z, (uint32_t)v0.w,
+                               (uint32_t)v1.x, (uint32_t)v1.y, (uint32_t)v1.z, (uint32_t)v1.w};
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const float2 v = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
+            f[2 * i] = v.x;
+            f[2 * i + 1] = v.y;
+        }
+        butterfly_f32(f, a.hb, lane);
+#pragma unroll
+        for (int i = 0; i < 16; ++i) f[i] *= norm;
+        if (!valid) continue;
+        if (MODE == 0) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                vmax = fmaxf(vmax, f[i]);
+                vmin = fminf(vmin, f[i]);
+            }
+        } else {
+            uint32_t o[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const float q0 = fminf(fmaxf(rintf(f[2 * i] * inv_s) + z, 0.f), 255.f) - z;
+                const float q1 = fminf(fmaxf(rintf(f[2 * i + 1] * inv_s) + z, 0.f), 255.f) - z;
+                o[i] = ((uint32_t)(uint16_t)(int16_t)(int)q0) | ((uint32_t)(uint16_t)(int16_t)(int)q1 << 16);
+            }
+            int4 *dst = reinterpret_cast<int4 *>(a.y + e0);
+            dst[0] = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
+            dst[1] = make_int4((int)o[4], (int)o[5], (int)o[6], (int)o[7]);
+        }
+    }
+    if (MODE == 0) {
+        unsigned int kmax = float_key(vmax), kneg = float_key(-vmin);
+        kmax = __reduce_max_sync(0xffffffffu, kmax);
+        kneg = __reduce_max_sync(0xffffffffu, kneg);
+        if (lane == 0) {
+            atomicMax(&a.p->max_key, kmax);
+            atomicMax(&a.p->negmin_key, kneg);
+        }
+    }
+}
+
+// s, z from the range (fp64 arithmetic on the fp32 extremes); a zero range gives (1, 0)
+__global__ void act_affine_params_kernel(AffineParams *p, float *params_out) {
+    if (threadIdx.x != 0 || blockIdx.x != 0) return;
+    const double hi = fmax((double)key_float(p->max_key), 0.0);
+    const double lo = fmin(-(double)key_float(p->negmin_key), 0.0);
+    double s = 1.0, z = 0.0;
+    if (hi - lo > 0.0) {
+        s = (hi - lo) / 255.0;
+        z = fmin(fmax(rint(-lo / s), 0.0), 255.0);
+    }
+    p->s = (float)s;
+    p->inv_s = (float)(1.0 / s);
+    p->z = (float)z;
+    if (params_out) {
+        params_out[0] = (float)s;
+        params_out[1] = (float)z;
+    }
+}
+
 // round(num / den) half to even for num, den > 0.
 __device__ long long div_rne(unsigned long long num, unsigned long long den) {
     unsigned long long q = num / den, r = num % den;
@@ -291,6 +393,18 @@ cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s) {
     const int grid = grid_for(a.total);
     if (a.f16) act_quant_kernel<true, 0><<<grid, kThreads, 0, s>>>(a);
     else act_quant_kernel<false, 0><<<grid, kThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_act_affine(const AffineQuantArgs &a, cudaStream_t s) {
+    cudaError_t e = cudaMemsetAsync(a.p, 0, sizeof(AffineParams), s);
+    if (e != cudaSuccess) return e;
+    const int grid = grid_for(a.total);
+    act_affine_kernel<0><<<grid, kThreads, 0, s>>>(a);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    act_affine_params_kernel<<<1, 32, 0, s>>>(a.p, a.params_out);
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    act_affine_kernel<1><<<grid, kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -41,6 +41,26 @@ struct DynParams {
     unsigned long long reserved;
 };
 
+// Device-side state of the dynamic affine quantizer (Eqs. uniform_q, affine_q;
+// lives in the caller's workspace): order-preserving keys of max v and of
+// -min v (both taken with atomicMax from zero), then the parameters.
+struct AffineParams {
+    unsigned int max_key, negmin_key;
+    float s, inv_s;      // step and its reciprocal (fp32, for the quantize pass)
+    float z;             // zero point, an integer in [0, 255]
+    int pad_[3];
+};
+
+struct AffineQuantArgs {
+    const void *x;        // fp16 NHWC
+    int16_t *y;           // centred codes x_int - z, NHWC
+    long long total;      // elements, multiple of 16
+    int hb;               // block of the input-side transform (1: none)
+    AffineParams *p;
+    float *params_out;    // device [2]: s, z (float)
+};
+cudaError_t launch_act_affine(const AffineQuantArgs &a, cudaStream_t s);
+
 // ---------------------------------------------------------------- profiling
 struct ProfileArgs {
     const int8_t *x;       // NHWC codes, n images of per_image elements
@@ -91,6 +111,13 @@ struct ConvArgs {
     int *err;
     // general transition (Sec. general nonlinearities): shift = n_out, mult = M_out,
     // then the table and the input-side pair (mult_in, shift_in)
+    // dynamic affine activations (Eq. affine_q): the operand holds centred int16 codes (128-byte box
+    // rows), the float epilogue takes s from *affine_s: t = (s s_w,c / gamma_out) a + beta_c with
+    // beta_c = b_bar_c / gamma_out in `deq`
+    int affine;
+    float inv_gamma;
+    const float *affine_s;
+    const float *s_w;
     int general, shift_in;
     int lut_off;                     // offset of the table copy from the barrier area
     long long mult_in;

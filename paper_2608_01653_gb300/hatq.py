@@ -45,7 +45,7 @@ class PreparedStruct(ctypes.Structure):
                 ("mult", ctypes.c_void_p), ("deq", ctypes.c_void_p), ("s_w", ctypes.c_void_p),
                 ("opaque", ctypes.c_uint64 * 16),
                 ("s_z", ctypes.c_float), ("s_u", ctypes.c_float), ("shift_in", ctypes.c_int),
-                ("reserved", ctypes.c_int), ("mult_in", ctypes.c_longlong), ("lut", ctypes.c_int8 * 256)]
+                ("in_affine", ctypes.c_int), ("mult_in", ctypes.c_longlong), ("lut", ctypes.c_int8 * 256)]
 
 
 MAX_TRANSPOSED_CLASSES = 4
@@ -98,6 +98,10 @@ def load(build: bool = True) -> ctypes.CDLL:
             "hatq_prepare_weights_order_host": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _F, _F, _I, _I, _I,
                                                      _P, _P, _P, _P, _P, _P, ctypes.POINTER(_I)]),
             "hatq_prepare_order_transform": (_I, [_I, _F, _F, ctypes.POINTER(PreparedStruct), _P]),
+            "hatq_prepare_weights_affine": (_I, [ctypes.POINTER(ConvDesc), _P, _P, _I, ctypes.POINTER(PreparedStruct),
+                                                 _P]),
+            "hatq_quantize_act_affine": (_I, [_P, _I, _I, _I, _I, _I, _P, _P, _P, _P]),
+            "hatq_conv2d_affine": (_I, [_P, _I, _I, _I, ctypes.POINTER(PreparedStruct), _P, _P, _P]),
             "hatq_transposed_sizes": (_I, [ctypes.POINTER(ConvDesc), _I, ctypes.POINTER(ctypes.c_size_t),
                                            ctypes.POINTER(ctypes.c_size_t)]),
             "hatq_prepare_weights_transposed": (_I, [ctypes.POINTER(ConvDesc), _I, _P, _P, _F, _F, _I, _I, _I,
@@ -328,6 +332,55 @@ def prepare_order_transform(c: int, s_in, s_out, stream=None, device="cuda") -> 
     _check(load().hatq_prepare_order_transform(int(c), float(s_in), float(s_out), ctypes.byref(L.struct),
                                                _stream(stream)))
     return L
+
+
+def prepare_weights_affine(desc: ConvDesc, w_ohwi, bias, act="none", stream=None, device="cuda") -> "PreparedLayer":
+    """hatq_prepare_weights_affine: a layer for dynamic affine activations
+    (centred int16 operand, per-input scale, float32 output)."""
+    L = PreparedLayer(desc, device)
+    w = np.ascontiguousarray(w_ohwi, dtype=np.float32)
+    b = None if bias is None else np.ascontiguousarray(bias, dtype=np.float32)
+    _check(load().hatq_prepare_weights_affine(ctypes.byref(desc), w.ctypes.data, None if b is None else b.ctypes.data,
+                                              _ACTS.get(act, act), ctypes.byref(L.struct), _stream(stream)))
+    return L
+
+
+def quantize_act_affine(x, hb, y=None, params=None, workspace=None, stream=None):
+    """hatq_quantize_act_affine on a CUDA fp16 NHWC tensor: returns (centred
+    int16 codes, params = device float[2] holding s and z)."""
+    if getattr(x, "dim", lambda: 0)() != 4:
+        raise ValueError("x must be a 4-D NHWC tensor")
+    _check_tensor(x, "x", "float16")
+    n, h, w, c = x.shape
+    if y is not None:
+        _check_tensor(y, "y", "int16", (n, h, w, c))
+    _check_cuda(("x", x), ("y", y))
+    torch = _torch()
+    if y is None:
+        y = torch.empty((n, h, w, c), dtype=torch.int16, device=x.device)
+    if params is None:
+        params = torch.empty(2, dtype=torch.float32, device=x.device)
+    if workspace is None:
+        workspace = torch.empty(64, dtype=torch.uint8, device=x.device)
+    _check(load().hatq_quantize_act_affine(_ptr(x), n, h, w, c, int(hb), _ptr(y), _ptr(params), _ptr(workspace),
+                                           _stream(stream)))
+    return y, params
+
+
+def conv2d_affine(x, L: "PreparedLayer", params, y=None, stream=None):
+    """hatq_conv2d_affine: the convolution on centred int16 codes at step params[0]."""
+    if getattr(x, "dim", lambda: 0)() != 4 or x.shape[-1] != L.c_in:
+        raise ValueError("x must be a 4-D NHWC tensor with the layer's input channels")
+    _check_tensor(x, "x", "int16")
+    n, h, w, c = x.shape
+    if y is not None:
+        _check_tensor(y, "y", "float32", L.out_shape(n, h, w))
+    _check_cuda(("x", x), ("y", y), ("params", params))
+    torch = _torch()
+    if y is None:
+        y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32, device=x.device)
+    _check(load().hatq_conv2d_affine(_ptr(x), n, h, w, ctypes.byref(L.struct), _ptr(params), _ptr(y), _stream(stream)))
+    return y
 
 
 class PreparedTransposed:

@@ -284,7 +284,7 @@ def test_prepared_struct_mirror_matches_the_c_layout(tmp_path):
     if cc is None:
         pytest.skip("no C compiler")
     fields = ["d", "act", "hb_next", "out_f32", "shift", "k_pad", "gather", "s_x", "s_y", "w_i8", "w_f16", "b_int",
-              "mult", "deq", "s_w", "opaque", "s_z", "s_u", "shift_in", "reserved", "mult_in", "lut"]
+              "mult", "deq", "s_w", "opaque", "s_z", "s_u", "shift_in", "in_affine", "mult_in", "lut"]
     src = tmp_path / "layout.c"
     inc = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include")
     src.write_text("#include <stdio.h>\n#include <stddef.h>\n#include \"hatq.h\"\nint main(void) {\n"
