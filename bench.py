@@ -53,12 +53,13 @@ def parse():
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="cfg4",
-                   choices=["cfg4", "cfg2", "cfg1", "fwht", "profile", "int8mm", "orders", "decoder"],
+                   choices=["cfg4", "cfg2", "cfg1", "fwht", "profile", "int8mm", "orders", "decoder", "affine"],
                    help="fwht: the INT8 transform+requantize pass alone on the config-4 ga2 input; "
                         "profile: the range-expansion profiling pass on the same tensor; "
                         "int8mm: torch._int_mm 8192^3, the library INT8 GEMM as a reference point; "
                         "orders: the paper's order-192 transform layer and ga2 in that basis at batch 8; "
-                        "decoder: a synthesis-side transposed 5x5 s2 layer and a sub-pixel layer at batch 8")
+                        "decoder: a synthesis-side transposed 5x5 s2 layer and a sub-pixel layer at batch 8; "
+                        "affine: ga2 with dynamic affine (PTQ) activations at batch 8")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--layer", default="", help="time one layer of the config-4 chains (e.g. ga2, h1, s0a)")
@@ -382,6 +383,39 @@ def run_decoder_mode(args):
         "peak_bf16_burst": tc}), flush=True)
 
 
+def run_affine_mode(args):
+    """ga2 (5x5 s2, 192 -> 192, DH 64) with dynamic affine activations at
+    batch 8 on the 1080 x 1920 fp16 input: the range + quantize passes
+    (fp16 in, centred int16 out) and the convolution on the centred codes."""
+    import torch
+    from paper_2608_01653_gb300 import hatq as H
+    H.load()
+    peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
+    tc, hbm = peaks.get("bf16_tflops", FALLBACK_BF16_TFLOPS), peaks.get("hbm_gbs", FALLBACK_HBM_GBS)
+    n, h, w = 8, 1080, 1920
+    g = torch.Generator(device="cuda")
+    g.manual_seed(17)
+    x = (torch.randn((n, h, w, 192), device="cuda", generator=g) + 0.5).to(torch.float16)
+    codes = torch.empty((n, h, w, 192), dtype=torch.int16, device="cuda")
+    params = torch.empty(2, dtype=torch.float32, device="cuda")
+    ws = torch.empty(64, dtype=torch.uint8, device="cuda")
+    L = C.layer("ga2", 192, 192, 5, 2, 2, "DH", "relu", hb_in=64)
+    P = H.prepare_weights_affine(H.desc_from_spec(L), I.weights(192, 5, 5, 192, 2001), I.bias(192, 2051), "relu")
+    y = torch.empty(P.out_shape(n, h, w), dtype=torch.float32, device="cuda")
+    q_ms = time_events(lambda: H.quantize_act_affine(x, 64, y=codes, params=params, workspace=ws), args.steps,
+                       args.warmup)
+    c_ms = time_events(lambda: H.conv2d_affine(codes, P, params, y=y), args.steps, args.warmup)
+    H.sync_status()
+    q_bytes = x.numel() * (2 + 2 + 2)                         # fp16 read twice (range, quantize) + int16 write
+    ho, wo = L.out_hw(h, w)
+    c_flops = 2 * n * ho * wo * 192 * 25 * 192
+    print(json.dumps({"mode": "affine", "batch": n, "in_hw": [h, w],
+                      "quantize": {"ms": q_ms, "gbs": q_bytes / (q_ms / 1000) / 1e9,
+                                   "frac": q_bytes / (hbm * 1e9) * 1000 / q_ms},
+                      "conv": {"ms": c_ms, "tflops": c_flops / (c_ms / 1000) / 1e12,
+                               "frac": c_flops / (tc * 1e12) * 1000 / c_ms}}), flush=True)
+
+
 def run_int8mm_mode(args):
     """torch._int_mm (the library INT8 GEMM, int32 output) on 8192^3, CUDA
     events: the measured INT8 tensor-core reference point of this GPU."""
@@ -422,8 +456,8 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
-    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile", "int8mm", "orders", "decoder")
-                                  else args.workload)
+    cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile", "int8mm", "orders", "decoder",
+                                                              "affine") else args.workload)
     if args.impl == "reference":
         run_reference(args, cfg, scales)
         return
@@ -444,6 +478,9 @@ def main():
         return
     if args.workload == "decoder":
         run_decoder_mode(args)
+        return
+    if args.workload == "affine":
+        run_affine_mode(args)
         return
 
     import torch
