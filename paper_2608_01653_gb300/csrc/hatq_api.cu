@@ -847,6 +847,7 @@ hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared 
     a.oox = og ? og->oox : 0;
     a.d2s = og ? og->d2s : 0;
     choose_mtile(ho, wo, d->stride, &a.tw, &a.th);
+    a.tw_log2 = __builtin_ctz((unsigned)a.tw);
     a.tiles_w = (wo + a.tw - 1) / a.tw;
     a.tiles_h = (ho + a.th - 1) / a.th;
     if ((long long)n * a.tiles_w * a.tiles_h >= (1LL << 31)) return fail(HATQ_ERR_UNSUPPORTED, "grid too large");

@@ -1025,11 +1025,12 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const int tid = nbuf == 2 ? et : et + 128 * wg;
                 if (nbuf == 2) asm volatile("bar.sync %0, 128;" ::"r"(2 + wg) : "memory");
                 else asm volatile("bar.sync 4, 256;" ::: "memory");
+                // a half-warp per tile row (at most 14 chunks of 16 bytes), so no division per chunk
                 const int cpr = row_bytes >> 4;
-                for (int jj = tid; ok && !a.out_f32 && jj < kTileM * cpr; jj += nthr) {
-                    const int r = jj / cpr, c = jj - r * cpr;
-                    const int oy = ho0 + r / a.tw, ox = wo0 + r % a.tw;
-                    if (oy < a.ho && ox < a.wo) {
+                const int c = lane & 15;
+                for (int r = (tid >> 5) * 2 + (lane >> 4); ok && !a.out_f32 && r < kTileM; r += nthr >> 4) {
+                    const int oy = ho0 + (r >> a.tw_log2), ox = wo0 + (r & (a.tw - 1));
+                    if (c < cpr && oy < a.ho && ox < a.wo) {
                         const int gy = oy * a.ostride + a.ooy, gx = ox * a.ostride + a.oox;
                         const uint8_t *src = stage_tile + (size_t)r * a.row_stride;
                         if (!a.d2s) {

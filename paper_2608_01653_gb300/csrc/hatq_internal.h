@@ -83,7 +83,8 @@ struct ConvArgs {
     // tensor (transposed convolutions write one output parity class per launch); with d2s = r >= 2 the
     // channels are rearranged depth-to-space into a [n][y_h r][y_w r][co / r^2] tensor
     int y_h, y_w, ostride, ooy, oox, d2s;
-    int tw, th, tiles_w, tiles_h;    // output tile: tw x th pixels (tw * th == 128)
+    int tw, th, tiles_w, tiles_h;    // output tile: tw x th pixels (tw * th == 128, tw a power of two)
+    int tw_log2;
     int n_t;                         // output channels per tile
     int num_kb;                      // 64-wide reduction blocks
     int cin_kb;                      // reduction blocks per kernel tap (tiled loader)
