@@ -40,6 +40,23 @@ CALIB = os.path.join(ROOT, "tests", "golden", "calibration.json")
 PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_BF16_TFLOPS = 1900.0
 FALLBACK_HBM_GBS = 6800.0
+# Integer issue capacity of a GB300 for integer-only code: one warp instruction per clock per SM
+# sub-partition split between the half-rate ALU and FMA-heavy pipes, 152 SMs x 4 x 32 lanes x 2.07 GHz
+INT_OPS_PEAK = 152 * 4 * 32 * 2.07e9
+
+
+def epilogue_int_ops(L, hb_next):
+    """Integer operations per output value of the exact requantize epilogue:
+    conversion, bias, 64-bit multiply (3), the ReLU on 64 bits (3), the
+    round-half-even shift with clamp (7), packing (1), and two 32-bit
+    operations per value for each stage of each int64 Sylvester transform."""
+    import math
+    hb_out = L.hb_out if L.form == "WH" else 0
+    ops = 11 + (3 if L.act == "relu" else 0)
+    for hb in (hb_out, hb_next):
+        if hb:
+            ops += 2 * int(math.log2(hb))
+    return ops
 CPU_SAMPLE_HW = (1024, 1536)      # bounded oracle sample: one 1536x1024 crop of image 0 (~10-15 s)
 CPU_SAMPLE_LATENT = (64, 96)
 REF_SAMPLE_HW = (512, 768)        # per step of --impl reference (~3 s), so K steps end within minutes
@@ -585,11 +602,14 @@ def main():
         flops = 2 * L.macs(n, h, w)
         nbytes = n * h * w * L.c_in + n * ho * wo * L.c_out + L.c_out * L.k * L.k * L.c_in
         lms = sum(times) / len(times)
-        t_tc, t_hbm = flops / (tc_peak * 1e12), nbytes / (hbm_peak * 1e9)
-        bound = "tensor" if t_tc >= t_hbm else "hbm"
+        int_ops = n * ho * wo * L.c_out * epilogue_int_ops(L, chains[ci]["chain"].plan[i])
+        t_tc, t_hbm, t_int = flops / (tc_peak * 1e12), nbytes / (hbm_peak * 1e9), int_ops / INT_OPS_PEAK
+        bound = max((t_tc, "tensor"), (t_hbm, "hbm"), (t_int, "alu"))[1]
         layers.append({"layer": L.name, "chain": ch.name, "ms": lms, "bound": bound,
                        "tflops": flops / (lms / 1000) / 1e12, "gbs": nbytes / (lms / 1000) / 1e9,
-                       "flops": flops, "bytes": nbytes, "frac": max(t_tc, t_hbm) * 1000 / lms})
+                       "int_tops": int_ops / (lms / 1000) / 1e12,
+                       "flops": flops, "bytes": nbytes, "int_ops": int_ops,
+                       "frac": max(t_tc, t_hbm, t_int) * 1000 / lms})
     conv_ms = sum(x["ms"] for x in layers)
     conv_flops = sum(x["flops"] for x in layers)
     n_conv = len(layers)
@@ -603,6 +623,9 @@ def main():
         src = os.path.join(ROOT, "paper_2608_01653_gb300", "csrc", "hatq_conv.cu")
         if hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] == rec.get("kernel_source_sha256_16"):
             traffic = rec.get("dram_bytes_per_launch")
+    roofline_peaks = {"tensor_tflops": tc_peak, "hbm_gbs": hbm_peak, "int_tops": INT_OPS_PEAK / 1e12,
+                      "int_source": "derived: 152 SMs x 4 sub-partitions x 32 lanes x 2.07 GHz (half-rate ALU + "
+                                    "FMA-heavy integer pipes)"}
     roofline = {"bound": "tensor", "achieved": achieved, "peak": tc_peak, "unit": "TFLOP/s", "frac": achieved / tc_peak,
                 "traffic": traffic, "kernel": "hatq conv_kernel (tcgen05 kind::f16, exact INT8)",
                 "launches": n_conv, "avg_launch_ms": conv_ms / max(n_conv, 1), "peak_source": tc_src,
@@ -708,7 +731,8 @@ def main():
         "effective_tops": world * 2 * macs_step / (ms / 1000.0) / 1e12,
         "config": {"workload": workload_name(cfg), "global_batch": world * images_step,
                    "parallelism": f"replicas x{world}", "l2": "inputs larger than L2 (199 MB image batch)"},
-        "roofline": roofline, "roofline_layers": layers, "roofline_fwht": roofline_fwht,
+        "roofline": roofline, "roofline_layers": layers, "roofline_peaks": roofline_peaks,
+        "roofline_fwht": roofline_fwht,
         "cpu_baseline": cpu, "e2e": e2e, "clocks": clocks,
         "gpu_launches": launches_step * args.steps,
     }
