@@ -305,6 +305,24 @@ void choose_mtile(int ho, int wo, int stride, int *tw, int *th) {
     }
 }
 
+// Bytes of one row of a small-channel layer's TMA window box: the window's
+// win_w * c bytes starting anywhere inside a 16-byte granule, rounded up to 16.
+int window_box_bytes(int tw, int stride, int kw, int c) { return (((tw - 1) * stride + kw) * c + 15 + 15) & ~15; }
+
+// Tile shape of a small-channel layer whose input window is loaded as one TMA
+// box per tile (box row <= 256 bytes and rows <= 256), or false when none fits
+// (the window is then staged by the converter warps).
+bool choose_window_tile(int ho, int wo, int stride, int kh, int kw, int c, int *tw, int *th) {
+    long long best = -1;
+    for (int t = 128; t >= 8; t >>= 1) {
+        const int h = 128 / t;
+        if (window_box_bytes(t, stride, kw, c) > 256 || (h - 1) * stride + kh > 256) continue;
+        const long long area = (long long)((wo + t - 1) / t) * t * (long long)((ho + h - 1) / h) * h;
+        if (best < 0 || area < best) { best = area; *tw = t; *th = h; }
+    }
+    return best >= 0;
+}
+
 hatq_status validate_prepare(const hatq_conv_desc *d, const float *w_ohwi, float s_x, float s_y, int act,
                                     int hb_next, int out_f32, Geometry *g) {
     hatq_status st = check_desc(d);
@@ -846,7 +864,11 @@ hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared 
     a.ooy = og ? og->ooy : 0;
     a.oox = og ? og->oox : 0;
     a.d2s = og ? og->d2s : 0;
-    choose_mtile(ho, wo, d->stride, &a.tw, &a.th);
+    // the small-channel loader takes its window by TMA when the input rows are 16-byte multiples
+    // (the tensor map's stride rule) and a tile shape's window fits one box
+    a.win_tma = g.gather && ((long long)w * d->c_in) % 16 == 0 &&
+                choose_window_tile(ho, wo, d->stride, d->kh, d->kw, d->c_in, &a.tw, &a.th);
+    if (!a.win_tma) choose_mtile(ho, wo, d->stride, &a.tw, &a.th);
     a.tw_log2 = __builtin_ctz((unsigned)a.tw);
     a.tiles_w = (wo + a.tw - 1) / a.tw;
     a.tiles_h = (ho + a.th - 1) / a.th;
@@ -894,13 +916,15 @@ hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared 
     a.staging_bytes = L->out_f32 ? 0 : a.nbuf * kTileRows * a.row_stride;   // float32 output is stored directly
     a.win_h = (a.th - 1) * d->stride + d->kh;
     a.win_w = (a.tw - 1) * d->stride + d->kw;
-    a.win_pitch = (a.win_w * d->c_in + 15) & ~15;
+    a.win_pitch = a.win_tma ? window_box_bytes(a.tw, d->stride, d->kw, d->c_in) : (a.win_w * d->c_in + 15) & ~15;
+    a.win_tma_bytes = a.win_tma ? a.win_pitch * a.win_h : 0;
+    a.win_buf = (a.win_h * a.win_pitch + 16 + 127) & ~127;  // + 16: the gather reads up to 11 bytes past a segment
     // + 16 bytes: the gather reads up to 11 bytes past a row segment
-    const int win_bytes = g.gather ? (a.win_h * a.win_pitch + 16 + 127) & ~127 : 0;
+    const int win_bytes = g.gather ? a.win_buf * (a.win_tma ? 2 : 1) : 0;
     const int table_bytes = g.gather ? a.num_kb * 8 * 4 : 0;
     const bool general = L->act == HATQ_ACT_SILU || L->act == HATQ_ACT_GELU;
     const int const_bytes = ((4 * d->c_out * 4 + 127) & ~127) + (general ? 256 : 0);
-    const int fixed = 1024 /* align */ + 8 * (3 * 8 + 9) + 16 + 128 + table_bytes + const_bytes + win_bytes;
+    const int fixed = 1024 /* align */ + 8 * (3 * 8 + 13) + 16 + 128 + table_bytes + const_bytes + win_bytes;
     const int budget = 227 * 1024 - 1024 /* static */ - fixed - a.staging_bytes;
     // a stage holds `sub` 64-wide reduction blocks: [weights x sub | INT8 box x sub].
     // The cost of a stage is dominated by its barrier hand-offs, not its bytes,
@@ -922,7 +946,7 @@ hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared 
     if (a.stages > 8) a.stages = 8;
     if (g.gather && a.stages > 4) a.stages = 4;
     if (a.stages < 2) return fail(HATQ_ERR_UNSUPPORTED, "tile does not fit in shared memory");
-    const int bar_bytes = 8 * (3 * a.stages + 9) + 16;
+    const int bar_bytes = 8 * (3 * a.stages + 13) + 16;
     a.const_off = (bar_bytes + table_bytes + 127) & ~127;
     a.win_off = a.const_off + const_bytes;
     const int smem_bytes = a.stages * a.stage_bytes + a.staging_bytes + 1024 + a.win_off + win_bytes;
@@ -969,6 +993,18 @@ hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared 
                          a.affine ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
                          CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "activation tensor map encoding failed (%d)", (int)r);
+    } else if (a.win_tma) {
+        // the input as a [n][h][w c] byte tensor; one box = one tile's window rows
+        EncodeTiledFn enc = encode_fn();
+        if (!enc) return fail(HATQ_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+        const cuuint64_t dims[3] = {(cuuint64_t)w * d->c_in, (cuuint64_t)h, (cuuint64_t)n};
+        const cuuint64_t strides[2] = {(cuuint64_t)w * d->c_in, (cuuint64_t)h * w * d->c_in};
+        const cuuint32_t box[3] = {(cuuint32_t)a.win_pitch, (cuuint32_t)a.win_h, 1};
+        const cuuint32_t estr[3] = {1, 1, 1};
+        CUresult r = enc(&tmA, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<void *>(x), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "input window tensor map encoding failed (%d)", (int)r);
     } else {
         tmA = tmB;
     }

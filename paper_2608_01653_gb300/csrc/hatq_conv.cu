@@ -107,6 +107,12 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *tm,
         "l"(tm), "r"(bar), "r"(x), "r"(y)
         : "memory");
 }
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *tm, uint32_t bar, int c0, int c1, int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+        "l"(tm), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
 __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *tm, uint32_t bar, int c0, int c1, int c2, int c3) {
     asm volatile(
         "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
@@ -577,8 +583,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto acc_empty = [&](int b) { return bar0 + 8u * (3 * S + 2 + b); };
     auto a_free = [&](int q) { return bar0 + 8u * (3 * S + 4 + q); };
     const uint32_t mma_done = bar0 + 8u * (3 * S + 8);
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_area + 8 * (3 * S + 9));
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_area + 8 * (3 * S + 9) + 4);
+    // small-channel layers with a TMA-loaded input window: two window buffers
+    auto win_full = [&](int b) { return bar0 + 8u * (3 * S + 9 + b); };
+    auto win_empty = [&](int b) { return bar0 + 8u * (3 * S + 11 + b); };
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_area + 8 * (3 * S + 13));
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_area + 8 * (3 * S + 13) + 4);
 
     // A failure already recorded by this launch (or an earlier, unread one)
     // ends every CTA that has not started, so a fault cannot serialize waits.
@@ -610,6 +619,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         for (int q = 0; q < 4; ++q) mbar_init(a_free(q), 1);
         mbar_init(mma_done, 1);
+        for (int b = 0; b < 2; ++b) {
+            mbar_init(win_full(b), 1);
+            mbar_init(win_empty(b), kConvThreads);
+        }
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -665,12 +678,24 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t tx_bytes = (uint32_t)(a.b_bytes + (a.gather ? 0 : a.raw_bytes));
             int issued_ph[8];
             for (int q = 0; q < 8; ++q) issued_ph[q] = -1;
+            int win_ph[2] = {-1, -1};
             bool ok = true;
             int s = 0;
             uint32_t ph = 0;
             for (int j = 0; j < my_tiles && ok; ++j) {
                 int img, ho0, wo0, n0;
                 tile_coords(j, img, ho0, wo0, n0);
+                if (a.win_tma) {
+                    // the tile's input window: one 3-D box of the [n][h][w c] byte tensor, its first byte
+                    // column rounded down to 16 (out-of-image parts, also negative ones, are zero-filled)
+                    const int b = j & 1;
+                    if (j >= 2 && !mbar_wait(win_empty(b), ((j >> 1) - 1) & 1, abort_flag, a.err)) { ok = false; break; }
+                    mbar_expect_tx(win_full(b), (uint32_t)a.win_tma_bytes);
+                    const int xb = (wo0 * a.stride - a.pad_x) * a.c;
+                    tma_load_3d(smem_addr(bar_area + a.win_off + b * a.win_buf), &tmA, win_full(b), xb & ~15,
+                                ho0 * a.stride - a.pad_y, img);
+                    win_ph[b] = (j >> 1) & 1;
+                }
                 int cb = 0, kx = 0, ky = 0;          // 64-channel block, kernel column and row of block kb
                 for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB) {
                     const int nsub = min(SUB, a.num_kb - kb0);
@@ -696,6 +721,12 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (!ok) {
                 // let our own copies land before the CTA unwinds
+                for (int b = 0; b < 2; ++b)
+                    if (win_ph[b] >= 0) {
+                        const long long t0 = clock64();
+                        while (!mbar_try_wait(win_full(b), (uint32_t)win_ph[b]) && clock64() - t0 < kWaitLimitCycles) {
+                        }
+                    }
                 for (int q = 0; q < S && q < 8; ++q)
                     if (issued_ph[q] >= 0) {
                         const long long t0 = clock64();
@@ -846,20 +877,33 @@ __global__ void __launch_bounds__(kThreads, 1)
             // memory; kernel row ky of output pixel m is then one contiguous
             // kw*c-byte segment of window row py*s+ky, read as 8-entry pieces
             // through a per-CTA table (window offset of each piece, -1 = zero).
-            int *tab = reinterpret_cast<int *>(bar_area + 8 * (3 * S + 9) + 16);
+            int *tab = reinterpret_cast<int *>(bar_area + 8 * (3 * S + 13) + 16);
             uint8_t *win = bar_area + a.win_off;
             for (int q = m; q < a.num_kb * 8; q += kConvThreads) {
                 const int k0 = q * 8, ky = k0 / a.seg;
                 tab[q] = ky < a.kh ? ky * a.win_pitch + (k0 - ky * a.seg) : -1;
             }
             const int rbase = (m / a.tw) * a.stride * a.win_pitch + (m % a.tw) * a.stride * a.c;
-            // Every converter thread runs the same tile loop (also after an
-            // abort, doing no work) so all four warps reach each named barrier.
+            // Without a TMA window, every converter thread runs the same tile loop
+            // (also after an abort, doing no work) so all four warps reach each named
+            // barrier. With one (win_tma) the producer loads the window one tile
+            // ahead into one of two buffers and no named barrier is used.
             for (int j = 0; j < my_tiles; ++j) {
                 int img, ho0, wo0, n0;
                 tile_coords(j, img, ho0, wo0, n0);
-                asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // previous window consumed
-                if (ok) {
+                const uint8_t *wv = win;                  // this tile's window
+                int woff = 0;                             // its first byte inside the buffer
+                if (a.win_tma) {
+                    if (!ok) break;
+                    const int b = j & 1;
+                    ok = __all_sync(0xffffffffu, mbar_wait(win_full(b), (j >> 1) & 1, abort_flag, a.err));
+                    if (!ok) break;
+                    wv = win + b * a.win_buf;
+                    const int xb = (wo0 * a.stride - a.pad_x) * a.c;
+                    woff = xb - (xb & ~15);
+                }
+                if (!a.win_tma) asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // previous window consumed
+                if (ok && !a.win_tma) {
                     const int ix_lo = wo0 * a.stride - a.pad_x;
                     const int row_b = a.win_w * a.c;
                     const int b_lo = max(0, -ix_lo) * a.c, b_hi = min(a.win_w, a.w - ix_lo) * a.c;
@@ -883,7 +927,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                         }
                     }
                 }
-                asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // window complete
+                if (!a.win_tma) asm volatile("bar.sync 1, %0;" ::"r"(kConvThreads) : "memory");   // window complete
                 for (int kb = 0; kb < a.num_kb && ok; ++kb) {
                     // the operand comes from the window: it is built first, then the
                     // stage (which keeps conv[s] in step with the MMA issuer) and the
@@ -894,8 +938,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                         const int off = tab[kb * 8 + q];
                         uint32_t w0 = 0u, w1 = 0u;
                         if (off >= 0) {
-                            const int o = rbase + off;
-                            const uint32_t *p = reinterpret_cast<const uint32_t *>(win + (o & ~3));
+                            const int o = rbase + woff + off;
+                            const uint32_t *p = reinterpret_cast<const uint32_t *>(wv + (o & ~3));
                             const uint32_t x0 = p[0], x1 = p[1], x2 = p[2];
                             w0 = __funnelshift_r(x0, x1, (uint32_t)(o & 3) * 8u);
                             w1 = __funnelshift_r(x1, x2, (uint32_t)(o & 3) * 8u);
@@ -913,6 +957,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mbar_arrive(conv_bar(s));
                     advance();
                 }
+                if (a.win_tma && ok) mbar_arrive(win_empty(j & 1));   // this thread's reads of the window are done
             }
         }
     } else {

@@ -103,6 +103,8 @@ struct ConvArgs {
     int const_off;                   // offsets from the barrier area: epilogue constants,
     int win_off, win_h, win_w;       // small-channel input window and its size
     int win_pitch;                   // bytes per window row
+    int win_tma;                     // 1: the producer loads the window by TMA (two buffers, win_buf bytes apart)
+    int win_buf, win_tma_bytes;      //    buffer stride and bytes of one window box
     const int8_t *x;
     const int32_t *b_int;
     const int32_t *mult;

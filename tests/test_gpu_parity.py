@@ -159,6 +159,10 @@ LAYER_CASES = [
     ("dh1x1_next128_nodrain", C.layer("a", 64, 128, 1, 1, 0, "DH", "relu", hb_in=64), (1, 12, 12), 128),
     ("wh3x3_c640_128_next128", C.layer("a", 320, 640, 3, 1, 1, "WH", "relu", hb_out=128), (1, 7, 10), 128),
     ("wh5x5s2_c3_next128", C.layer("a", 3, 128, 5, 2, 2, "WH", "relu", hb_out=128), (1, 30, 44), 128),
+    # small-channel layers whose input rows are 16-byte multiples: the window comes by TMA
+    ("wh5x5s2_c3_tma_window", C.layer("a", 3, 192, 5, 2, 2, "WH", "relu", hb_out=64), (2, 41, 64), 64),
+    ("wh3x3_c4_tma_window", C.layer("a", 4, 64, 3, 1, 1, "WH", "relu", hb_out=64), (1, 21, 36), 0),
+    ("wh7x7_c8_tma_window", C.layer("a", 8, 64, 7, 1, 3, "WH", "none", hb_out=32), (2, 19, 34), 32),
 ]
 
 
