@@ -20,7 +20,9 @@ Readings the paper leaves open (the same list is kept with the design notes):
      the largest shared n in [0, 62] such that every M_c = rint(rho_c 2^n) is
      below 2^31 and max_c(M_c A_c) * g_out * g_next < 2^62, with A_c the
      worst-case |accumulator| of channel c and g the gains (block sizes) of the
-     unnormalized transforms; fewer than 16 bits in max_c M_c is an error.
+     unnormalized transforms; fewer than 16 bits in max_c M_c is an error. The
+     INT8-entry activation requantizer (a 32-bit computation) takes the bound
+     M 127 hb < 2^30 instead of 2^62 and a 15-bit precision floor.
   R4 symmetric INT8 range [-127, 127]; a zero range gives scale 1.
   R5 bias enters the int32 accumulator before M (.) and before H_out.
   R6 fixed summation order for real-valued transforms: for output j,
@@ -303,11 +305,15 @@ def rshift_rne(v, n: int) -> np.ndarray:
     return q + up.astype(np.int64)
 
 
-def fixed_point(rho, a_bound, gain: int = 1):
+def fixed_point(rho, a_bound, gain: int = 1, prod_bits: int = 62, min_bits: int = 16):
     """Multiplier/shift pair of Eqs. (fixed_point_scale, integer_fixed_point_scale)
     under reading R3. rho: per-channel real ratios (> 0); a_bound: per-channel
     bound on |input| of the multiplication; gain: product of the unnormalized
-    transform gains applied after M (.). Returns (M int64 array, n)."""
+    transform gains applied after M (.); prod_bits: the products M a gain stay
+    below 2^prod_bits (62 for the 64-bit epilogue, 30 for the 32-bit activation
+    requantizer); min_bits: the least multiplier precision (16, and 15 for
+    the activation requantizer, whose 32-bit bound leaves 15 bits at hb = 256).
+    Returns (M int64 array, n)."""
     rho = np.asarray(rho, dtype=np.float64)
     a_bound = [int(a) for a in np.asarray(a_bound).ravel()]
     if np.any(rho < 0) or not np.all(np.isfinite(rho)):
@@ -317,10 +323,10 @@ def fixed_point(rho, a_bound, gain: int = 1):
         if max(M) >= 2 ** 31:
             continue
         worst = max(m * a for m, a in zip(M, a_bound)) * int(gain)
-        if worst >= 2 ** 62:
+        if worst >= 2 ** prod_bits:
             continue
-        if max(M) < 2 ** 15:
-            raise OverflowError("fewer than 16 bits of multiplier precision")
+        if max(M) < 2 ** (min_bits - 1):
+            raise OverflowError(f"fewer than {min_bits} bits of multiplier precision")
         return np.array(M, dtype=np.int64), n
     raise OverflowError("no shift satisfies the multiplier and overflow bounds")
 
@@ -335,15 +341,16 @@ def round_half_even_fraction(f: Fraction) -> int:
 
 def dynamic_multiplier(maxy: int, hb: int):
     """(M, n) for the dynamic INT8-entry quantizer: rho = 127 / max|y| as an
-    exact rational, M = round(rho 2^n) half to even, n by reading R3."""
+    exact rational, M = round(rho 2^n) half to even, n by reading R3 with the
+    activation requantizer's 32-bit product bound M 127 hb < 2^30."""
     if maxy <= 0:
         return 0, 0
     for n in range(62, -1, -1):
         M = round_half_even_fraction(Fraction(QMAX << n, maxy))
-        if M >= 2 ** 31 or M * QMAX * hb >= 2 ** 62:
+        if M >= 2 ** 31 or M * QMAX * hb >= 2 ** 30:
             continue
-        if M < 2 ** 15:
-            raise OverflowError("fewer than 16 bits of multiplier precision")
+        if M < 2 ** 14:
+            raise OverflowError("fewer than 15 bits of multiplier precision")
         return M, n
     raise OverflowError("no shift satisfies the bounds")
 
@@ -484,9 +491,10 @@ def quantize_act_f16(x, hb: int, s_x: float) -> np.ndarray:
 
 
 def act_multiplier(hb: int, s_in: float, s_x: float):
-    """(M_q, n_q) with M_q / 2^n_q ~ s_in / (sqrt(hb) s_x), bound |y| <= 127 hb."""
+    """(M_q, n_q) with M_q / 2^n_q ~ s_in / (sqrt(hb) s_x), bound |y| <= 127 hb,
+    products M_q |y| below 2^30 (reading R3, 32-bit activation requantizer)."""
     rho = float(np.float32(s_in)) / (math.sqrt(hb) * float(np.float32(s_x)))
-    M, n = fixed_point([rho], [QMAX * hb], 1)
+    M, n = fixed_point([rho], [QMAX * hb], 1, prod_bits=30, min_bits=15)
     return int(M[0]), n
 
 
@@ -788,13 +796,16 @@ AFFINE_QMIN, AFFINE_QMAX = 0, 255          # unsigned 8-bit grid of Eq. affine_q
 def affine_params(x):
     """(s, z) of Eq. affine_q from the tensor's range, zero kept representable:
     x_min' = min(x_min, 0), x_max' = max(x_max, 0), s = (x_max' - x_min') / 255,
-    z = clamp(round(0 - x_min' / s), 0, 255); a zero range gives (1, 0)."""
+    z = clamp(round(0 - x_min' / s), 0, 255); a zero range gives (1, 0), and so
+    does a range too small for a nonzero step (s underflows to 0)."""
     x = np.asarray(x, dtype=np.float64)
     lo = min(float(x.min()), 0.0) if x.size else 0.0
     hi = max(float(x.max()), 0.0) if x.size else 0.0
     if hi - lo <= 0.0:
         return 1.0, 0
     s = (hi - lo) / (AFFINE_QMAX - AFFINE_QMIN)
+    if not s > 0.0:
+        return 1.0, 0
     z = int(min(max(round(AFFINE_QMIN - lo / s), AFFINE_QMIN), AFFINE_QMAX))
     return s, z
 
