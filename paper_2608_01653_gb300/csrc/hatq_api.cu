@@ -248,9 +248,11 @@ hatq_status geometry(const hatq_conv_desc *d, int hb_next, Geometry *g) {
 // ------------------------------------------------------------ fixed point (M, n)
 
 // Largest n in [0, 62] with all M_c = rint(rho_c 2^n) < 2^31 and
-// max_c(M_c A_c) * gain < 2^62; fewer than 16 bits in max M is an error.
+// max_c(M_c A_c) * gain < 2^prod_bits; fewer than min_bits bits in max M is an
+// error. The 64-bit epilogue takes (62, 16); the INT8-entry activation
+// requantizer, a 32-bit computation, (30, 15).
 hatq_status fixed_point(const std::vector<double> &rho, const std::vector<long long> &abound, long long gain,
-                        std::vector<int32_t> &M, int &shift) {
+                        std::vector<int32_t> &M, int &shift, int prod_bits = 62, int min_bits = 16) {
     for (double r : rho)
         if (!(r >= 0.0) || !std::isfinite(r)) return fail(HATQ_ERR_INVALID_ARG, "scale ratio must be finite and >= 0");
     M.assign(rho.size(), 0);
@@ -268,8 +270,9 @@ hatq_status fixed_point(const std::vector<double> &rho, const std::vector<long l
             if (w > worst) worst = w;
         }
         if (!ok) continue;
-        if (worst * (unsigned __int128)gain >= ((unsigned __int128)1 << 62)) continue;
-        if (mmax < (1LL << 15)) return fail(HATQ_ERR_OVERFLOW, "fewer than 16 bits of multiplier precision");
+        if (worst * (unsigned __int128)gain >= ((unsigned __int128)1 << prod_bits)) continue;
+        if (mmax < (1LL << (min_bits - 1)))
+            return fail(HATQ_ERR_OVERFLOW, "fewer than %d bits of multiplier precision", min_bits);
         for (size_t c = 0; c < rho.size(); ++c) M[c] = (int32_t)m[c];
         shift = n;
         return HATQ_OK;
@@ -797,7 +800,7 @@ hatq_status hatq_quantize_act(const void *x, int x_kind, float s_in, int n, int 
             const double rho = (double)s_in / (std::sqrt((double)hb) * (double)s_out);
             std::vector<int32_t> M;
             int shift = 0;
-            hatq_status st = fixed_point({rho}, {127LL * hb}, 1, M, shift);
+            hatq_status st = fixed_point({rho}, {127LL * hb}, 1, M, shift, 30, 15);
             if (st != HATQ_OK) return st;
             a.mult = M[0];
             a.shift = shift;

@@ -110,6 +110,11 @@ __device__ __forceinline__ int requant_hi(long long P, int s, long long k) {
     const long long u = P + k + (long long)bit;
     return clamp127((int)(u >> 32) >> s);
 }
+// round(P / 2^n) half to even for 1 <= n <= 30 in 32-bit arithmetic (the
+// multiplier rule keeps |P| < 2^30, so P + 2^(n-1) does not overflow), clamped.
+__device__ __forceinline__ int requant32(int P, int n, int k) {
+    return clamp127((P + k + ((P >> n) & 1)) >> n);
+}
 __device__ __forceinline__ uint32_t pack4p(int a, int b, int c, int d) {
     return __byte_perm(__byte_perm((uint32_t)a, (uint32_t)b, 0x0040), __byte_perm((uint32_t)c, (uint32_t)d, 0x0040), 0x5410);
 }
@@ -133,9 +138,10 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
     }
     uint32_t local_max = 0;
     float local_maxf = 0.f;
-    // Software pipelining: the loads of this warp's next tile are in flight
-    // while the current tile is transformed and stored.
+    // Software pipelining: the loads of this warp's next two tiles are in
+    // flight while the current tile is transformed and stored.
     int4 cur0 = make_int4(0, 0, 0, 0), cur1 = make_int4(0, 0, 0, 0);
+    int4 mid0 = make_int4(0, 0, 0, 0), mid1 = make_int4(0, 0, 0, 0);
     auto load_tile = [&](long long t, int4 &v0, int4 &v1) {
         const long long e0 = (t << 9) + lane * 16;
         v0 = make_int4(0, 0, 0, 0);
@@ -151,9 +157,10 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
         }
     };
     load_tile(warp, cur0, cur1);
+    load_tile(warp + nwarps, mid0, mid1);
     for (long long t = warp; t < tiles; t += nwarps) {
         int4 nxt0, nxt1;
-        load_tile(t + nwarps, nxt0, nxt1);
+        load_tile(t + 2 * nwarps, nxt0, nxt1);
         const long long e0 = (t << 9) + lane * 16;
         const bool valid = e0 < a.total;
         if (!F16) {
@@ -166,7 +173,14 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
             } else if (valid) {
                 uint32_t o[4];
                 const int m32 = (int)mult;            // M_q < 2^31
-                if (shift >= 32) {
+                if (shift >= 1 && shift <= 30) {
+                    // M_q 127 hb < 2^30: the products fit 32 bits
+                    const int k = (1 << (shift - 1)) - 1;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        o[i] = pack4p(requant32(m32 * v[4 * i], shift, k), requant32(m32 * v[4 * i + 1], shift, k),
+                                      requant32(m32 * v[4 * i + 2], shift, k), requant32(m32 * v[4 * i + 3], shift, k));
+                } else if (shift >= 32) {
                     const int sh = shift - 32;
                     const long long k = (1LL << (shift - 1)) - 1;
 #pragma unroll
@@ -209,8 +223,10 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
                 *reinterpret_cast<int4 *>(a.y + e0) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
             }
         }
-        cur0 = nxt0;
-        cur1 = nxt1;
+        cur0 = mid0;
+        cur1 = mid1;
+        mid0 = nxt0;
+        mid1 = nxt1;
     }
     if (MODE == 2) {
         uint32_t m = F16 ? __float_as_uint(local_maxf) : local_max;   // nonnegative floats order as integers
@@ -330,9 +346,10 @@ __device__ long long div_rne(unsigned long long num, unsigned long long den) {
 
 // Dynamic parameters from the max-abs: INT8 entry uses the exact rational
 // rho = 127 / max|v| (the 1/sqrt(hb) and s_in cancel), M = round(rho 2^n) with
-// the largest n such that M < 2^31 and M 127 hb < 2^62; the scan starts at
-// n = 55 (127 * 2^55 < 2^63), and every n > 39 fails M < 2^31 for the
-// max |v| <= 127 * 256 of this operator, so the result equals a scan from 62.
+// the largest n such that M < 2^31 and M 127 hb < 2^30 (the requantizer's
+// 32-bit product bound; at least 15 bits in M); the scan starts at n = 55
+// (127 * 2^55 < 2^63), and every n > 39 fails M < 2^31 for the max
+// |v| <= 127 * 256 of this operator, so the result equals a scan from 62.
 __global__ void act_dyn_params_kernel(DynParams *p, int f16, int hb, float s_in, float *s_used, int *err) {
     if (threadIdx.x != 0 || blockIdx.x != 0) return;
     const unsigned int mb = p->maxbits;
@@ -355,11 +372,11 @@ __global__ void act_dyn_params_kernel(DynParams *p, int f16, int hb, float s_in,
         const long long m = div_rne(127ull << n, (unsigned long long)mb);
         if (m >= (1LL << 31)) continue;
         const unsigned long long worst = (unsigned long long)m * 127ull * (unsigned long long)hb;
-        if (worst >= (1ull << 62)) continue;
+        if (worst >= (1ull << 30)) continue;        // the requantizer's 32-bit product bound
         found = n; M = m;
         break;
     }
-    if (found < 0 || M < (1LL << 15)) {
+    if (found < 0 || M < (1LL << 14)) {
         atomicExch(err, kErrBounds);
         found = 0; M = 0;
     }
@@ -380,45 +397,47 @@ int num_sms() {
     return sms;
 }
 
-int grid_for(long long total) {
+// One wave: the blocks of kernel `k` that are resident at once (the grid-stride
+// loop then gives every warp the same number of tiles).
+template <typename K>
+int grid_for(long long total, K k) {
     const long long tiles = (total + 511) / 512;
     const long long want = (tiles + 7) / 8;           // 8 warps per block
-    const long long cap = (long long)num_sms() * 8;   // 8 resident blocks of 256 threads per SM
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kThreads, 0) != cudaSuccess || per_sm < 1) per_sm = 4;
+    const long long cap = (long long)num_sms() * per_sm;
     return (int)(want < 1 ? 1 : (want < cap ? want : cap));
 }
 
 }  // namespace
 
 cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s) {
-    const int grid = grid_for(a.total);
-    if (a.f16) act_quant_kernel<true, 0><<<grid, kThreads, 0, s>>>(a);
-    else act_quant_kernel<false, 0><<<grid, kThreads, 0, s>>>(a);
+    if (a.f16) act_quant_kernel<true, 0><<<grid_for(a.total, act_quant_kernel<true, 0>), kThreads, 0, s>>>(a);
+    else act_quant_kernel<false, 0><<<grid_for(a.total, act_quant_kernel<false, 0>), kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 
 cudaError_t launch_act_affine(const AffineQuantArgs &a, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(a.p, 0, sizeof(AffineParams), s);
     if (e != cudaSuccess) return e;
-    const int grid = grid_for(a.total);
-    act_affine_kernel<0><<<grid, kThreads, 0, s>>>(a);
+    act_affine_kernel<0><<<grid_for(a.total, act_affine_kernel<0>), kThreads, 0, s>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     act_affine_params_kernel<<<1, 32, 0, s>>>(a.p, a.params_out);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    act_affine_kernel<1><<<grid, kThreads, 0, s>>>(a);
+    act_affine_kernel<1><<<grid_for(a.total, act_affine_kernel<1>), kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 
 cudaError_t launch_act_dynamic(const ActQuantArgs &a, float s_in, float *s_used, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(a.dyn, 0, sizeof(DynParams), s);
     if (e != cudaSuccess) return e;
-    const int grid = grid_for(a.total);
-    if (a.f16) act_quant_kernel<true, 2><<<grid, kThreads, 0, s>>>(a);
-    else act_quant_kernel<false, 2><<<grid, kThreads, 0, s>>>(a);
+    if (a.f16) act_quant_kernel<true, 2><<<grid_for(a.total, act_quant_kernel<true, 2>), kThreads, 0, s>>>(a);
+    else act_quant_kernel<false, 2><<<grid_for(a.total, act_quant_kernel<false, 2>), kThreads, 0, s>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     act_dyn_params_kernel<<<1, 32, 0, s>>>(a.dyn, a.f16, a.hb, s_in, s_used, a.err);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    if (a.f16) act_quant_kernel<true, 1><<<grid, kThreads, 0, s>>>(a);
-    else act_quant_kernel<false, 1><<<grid, kThreads, 0, s>>>(a);
+    if (a.f16) act_quant_kernel<true, 1><<<grid_for(a.total, act_quant_kernel<true, 1>), kThreads, 0, s>>>(a);
+    else act_quant_kernel<false, 1><<<grid_for(a.total, act_quant_kernel<false, 1>), kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

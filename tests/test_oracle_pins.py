@@ -202,6 +202,22 @@ def test_fixed_point_precision_floor():
         O.fixed_point([1e-9], [2 ** 30], 2 ** 28)
 
 
+@pytest.mark.parametrize("hb,rho", [(64, 0.5), (64, 0.013), (256, 0.9), (1, 0.37), (16, 3.0)])
+def test_activation_multiplier_32bit_bound_and_maximality(hb, rho):
+    """Reading R3 for the activation requantizer: the largest n with
+    M < 2^31 and M 127 hb < 2^30, so M |y| + 2^(n-1) fits a signed 32-bit word;
+    n + 1 breaks the bound; M / 2^n within half a unit of rho 2^n."""
+    s_x = 1.0 / (math.sqrt(hb) * rho)
+    M, n = O.act_multiplier(hb, 1.0, s_x)
+    r = 1.0 / (math.sqrt(hb) * float(np.float32(s_x)))
+    assert M * 127 * hb < 2 ** 30 and M < 2 ** 31 and M >= 2 ** 14
+    assert abs(M - r * 2.0 ** n) <= 0.5
+    M2 = int(np.rint(math.ldexp(r, n + 1)))
+    assert M2 * 127 * hb >= 2 ** 30 or M2 >= 2 ** 31
+    y = np.array([127 * hb, -127 * hb, 0, 1, -1])
+    assert np.all(np.abs(M * y) + (1 << max(n - 1, 0)) < 2 ** 31)
+
+
 def test_dynamic_multiplier_exact():
     for maxy in (1, 3, 127, 1000, 8191, 127 * 64):
         M, n = O.dynamic_multiplier(maxy, 64)
