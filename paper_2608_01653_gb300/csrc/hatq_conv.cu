@@ -221,18 +221,28 @@ __device__ __forceinline__ int requant8(long long v, int n) {
     return q < -127 ? -127 : (q > 127 ? 127 : q);
 }
 
-// The same rounding for 32 <= n <= 62 in 32-bit pieces: with k = 2^(n-1) - 1
-// and s = n - 32, v + k + bit_n(v) stays below 2^63 and its arithmetic shift
-// by n is the high word shifted by s.
-__device__ __forceinline__ int requant8_hi(long long v, int s, unsigned long long k) {
-    const uint32_t bit = ((uint32_t)((unsigned long long)v >> 32) >> s) & 1u;
-    const long long u = v + (long long)k + (long long)bit;
-    const int q = (int)(u >> 32) >> s;
-    return min(max(q, -127), 127);
+// The same rounding for 33 <= n <= 62 on the 32-bit halves of v (s = n - 32,
+// kh = 2^(s-1) - 1): v + 2^(n-1) - 1 + bit_n(v) has the high word
+// hi + kh + c, where c is the carry out of the low word, lo + (2^32 - 1) + bit,
+// i.e. c = [lo or bit nonzero]; its shift by n is that high word shifted by s.
+__device__ __forceinline__ int requant8_hi(long long v, int s, int kh) {
+    const uint32_t lo = (uint32_t)v;
+    const int hi = (int)((unsigned long long)v >> 32);
+    const uint32_t bit = (uint32_t)(hi >> s) & 1u;
+    const int c = (int)min(lo | bit, 1u);
+    return min(max((hi + kh + c) >> s, -127), 127);
 }
-// requant8 with the 32-bit-piece path for shifts >= 32 (n is uniform).
+// n = 32: v + 2^31 - 1 + bit_32(v) carries out of the low word iff lo + bit > 2^31.
+__device__ __forceinline__ int requant8_32(long long v) {
+    const uint32_t lo = (uint32_t)v;
+    const int hi = (int)((unsigned long long)v >> 32);
+    const int c = (lo > 0x80000000u || (lo == 0x80000000u && (hi & 1))) ? 1 : 0;
+    return min(max(hi + c, -127), 127);
+}
+// requant8 with the 32-bit-piece paths for shifts >= 32 (n is uniform).
 __device__ __forceinline__ int requant8_any(long long v, int n) {
-    return n >= 32 ? requant8_hi(v, n - 32, (1ull << (n - 1)) - 1) : requant8(v, n);
+    if (n > 32) return requant8_hi(v, n - 32, (1 << (n - 33)) - 1);
+    return n == 32 ? requant8_32(v) : requant8(v, n);
 }
 
 // Low bytes of four codes in [-127, 127] packed into one word.
@@ -330,17 +340,30 @@ __device__ __forceinline__ void scale_f32(const EpiCtx &e, int col, const int (&
 // thread's row of the shared-memory output tile (copied out coalesced later).
 template <int G>
 __device__ __forceinline__ void store_codes(const ConvArgs &a, uint8_t *row, int col, const long long (&t)[G]) {
-    if (a.shift >= 32) {
+    if (a.shift > 32) {
         const int sh = a.shift - 32;
-        const unsigned long long k = (1ull << (a.shift - 1)) - 1;
+        const int kh = (1 << (sh - 1)) - 1;
 #pragma unroll
         for (int i = 0; i < G / 16; ++i) {
             uint32_t w[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const int b = 16 * i + 4 * j;
-                w[j] = pack4(requant8_hi(t[b], sh, k), requant8_hi(t[b + 1], sh, k), requant8_hi(t[b + 2], sh, k),
-                             requant8_hi(t[b + 3], sh, k));
+                w[j] = pack4(requant8_hi(t[b], sh, kh), requant8_hi(t[b + 1], sh, kh), requant8_hi(t[b + 2], sh, kh),
+                             requant8_hi(t[b + 3], sh, kh));
+            }
+            reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
+        }
+        return;
+    }
+    if (a.shift == 32) {
+#pragma unroll
+        for (int i = 0; i < G / 16; ++i) {
+            uint32_t w[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int b = 16 * i + 4 * j;
+                w[j] = pack4(requant8_32(t[b]), requant8_32(t[b + 1]), requant8_32(t[b + 2]), requant8_32(t[b + 3]));
             }
             reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
         }
