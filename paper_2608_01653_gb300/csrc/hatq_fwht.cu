@@ -337,6 +337,232 @@ __global__ void act_affine_params_kernel(AffineParams *p, float *params_out) {
     }
 }
 
+// INT8 entry, static scale, blocks of at most 64: a lane owns 64 consecutive
+// elements (four 16-byte loads; the warp's loads cover 2 KB contiguously), so
+// every butterfly stage runs inside the lane without shuffles. SMALL: the
+// requantization fits 32-bit words (shift <= 30 under the multiplier rule).
+template <int HB, bool SMALL>
+__global__ void __launch_bounds__(kThreads) act_quant_i8_wide_kernel(ActQuantArgs a) {
+    const int lane = threadIdx.x & 31;
+    const long long warp = ((long long)blockIdx.x * kThreads + threadIdx.x) >> 5;
+    const long long nwarps = ((long long)gridDim.x * kThreads) >> 5;
+    const long long tiles = (a.total + 2047) >> 11;
+    const int m32 = (int)a.mult;
+    const int shift = a.shift;
+    const int k32 = shift >= 1 ? (1 << (shift - 1)) - 1 : 0;
+    const int sh = shift - 32;
+    const long long k64 = shift >= 1 ? (1LL << (shift - 1)) - 1 : 0;
+    auto load = [&](long long t, int4 (&r)[4]) {
+        const long long e0 = (t << 11) + lane * 64;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            r[q] = make_int4(0, 0, 0, 0);
+            if (t < tiles && e0 + 16 * q < a.total)
+                r[q] = __ldg(reinterpret_cast<const int4 *>(static_cast<const int8_t *>(a.x) + e0 + 16 * q));
+        }
+    };
+    int4 cur[4], nxt[4];
+    load(warp, cur);
+    for (long long t = warp; t < tiles; t += nwarps) {
+        load(t + nwarps, nxt);
+        const long long e0 = (t << 11) + lane * 64;
+        int v[64];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            int u[16];
+            unpack_i8x16_i32(cur[q], u);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[16 * q + i] = u[i];
+        }
+#pragma unroll
+        for (int h = 1; h < HB; h <<= 1) {
+#pragma unroll
+            for (int i = 0; i < 64; ++i) {
+                if (i & h) continue;
+                const int x = v[i], y = v[i + h];
+                v[i] = x + y;
+                v[i + h] = x - y;
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            if (e0 + 16 * q >= a.total) break;
+            uint32_t o[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                int c[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const int x = v[16 * q + 4 * i + j];
+                    if (SMALL) c[j] = shift ? requant32(m32 * x, shift, k32) : clamp127(m32 * x);
+                    else c[j] = shift >= 32 ? requant_hi((long long)m32 * x, sh, k64) : requant((long long)m32 * x, shift);
+                }
+                o[i] = pack4p(c[0], c[1], c[2], c[3]);
+            }
+            *reinterpret_cast<int4 *>(a.y + e0 + 16 * q) = make_int4((int)o[0], (int)o[1], (int)o[2], (int)o[3]);
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) cur[q] = nxt[q];
+    }
+}
+
+// Two 16-bit lanes per 32-bit word. A lane owns 128 consecutive elements and
+// word j carries elements j (low half) and 64 + j (high half) as the integer
+// lo + 65536 hi. Integer addition is linear, so one 32-bit add or subtract is
+// a butterfly on both halves, and blocks of at most 64 never mix the halves.
+// The bytes enter biased by 128 (v ^ 0x80); the first stage removes that bias
+// and adds kBlo to the low half of every output, so at the end the low half
+// is nonnegative and the word's bit pattern is the pair (lo, hi) of signed
+// 16-bit values (|y| <= 127 * 64 < 2^15).
+struct SwarParams {
+    uint32_t clo;        // s16x2 lower clamp bound -vmax of y, plus the biases
+    uint32_t clow, chigh; // requantization addends of the low and high halves
+    uint32_t mult;
+    int shift;
+};
+
+__device__ __forceinline__ uint32_t max_s16x2(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("max.s16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+// bytes (q0, q1, q2, q3) of a word, each q saturated to [-128, 127]
+__device__ __forceinline__ uint32_t pack4s(int q0, int q1, int q2, int q3) {
+    uint32_t hi, d;
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(hi) : "r"(q3), "r"(q2), "r"(0u));
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(q1), "r"(q0), "r"(hi));
+    return d;
+}
+
+// TIES: rounding ties M y = 2^(n-1) (mod 2^n) can occur, so the half-to-even
+// correction is applied; otherwise round half up is the same function.
+template <int HB, bool TIES>
+__device__ __forceinline__ int swar_requant(uint32_t a, uint32_t c, uint32_t m, int n) {
+    const int p = (int)(m * a + c);                 // M y + 2^(n-1) (- 1 with TIES), exact mod 2^32
+    if (TIES) return (p + ((p >> n) & 1)) >> n;
+    return p >> n;
+}
+
+// Per-warp staging of the packed kernel: a 4 KB tile is 32 rows of 128 bytes,
+// row l belonging to lane l; the 16-byte chunk q of row r sits at position
+// q ^ (r & 7), so the coalesced copies (chunk 32 i + lane) and the row-wise
+// reads and writes of a lane both touch 32 distinct banks per 8 lanes.
+constexpr int kSwarWarps = 4;
+constexpr int kSwarStages = 3;
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ int swz(int row, int chunk) { return row * 128 + ((chunk ^ (row & 7)) << 4); }
+
+template <int HB, bool TIES>
+__global__ void __launch_bounds__(kSwarWarps * 32) act_quant_i8_swar_kernel(ActQuantArgs a, SwarParams sp) {
+    constexpr uint32_t kBlo = HB >= 2 ? 128u * HB : 0u;
+    constexpr uint32_t kBias2 = 256u * 65537u;      // the two halves' input bias after one stage
+    __shared__ __align__(128) uint8_t stage[kSwarWarps][kSwarStages][4096];
+    const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+    const long long warp = (long long)blockIdx.x * kSwarWarps + wib;
+    const long long nwarps = (long long)gridDim.x * kSwarWarps;
+    const long long tiles = (a.total + 4095) >> 12;
+    const int8_t *xg = static_cast<const int8_t *>(a.x);
+    // Copy tile t into a stage with zero fill past the end; one commit group
+    // per call, empty when t is past the last tile.
+    auto issue = [&](long long t, int slot) {
+        if (t < tiles) {
+            const long long e0 = t << 12;
+            uint8_t *buf = stage[wib][slot];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int c = 32 * i + lane;
+                const bool ok = e0 + 16 * c < a.total;
+                const int8_t *src = ok ? xg + e0 + 16 * c : xg;
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(buf + swz(c >> 3, c & 7))),
+                             "l"(src), "r"(ok ? 16 : 0)
+                             : "memory");
+            }
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+#pragma unroll
+    for (int k = 0; k < kSwarStages; ++k) issue(warp + k * nwarps, k);
+    int slot = 0;
+    for (long long t = warp; t < tiles; t += nwarps) {
+        asm volatile("cp.async.wait_group %0;" ::"n"(kSwarStages - 1) : "memory");
+        __syncwarp();
+        uint8_t *buf = stage[wib][slot];
+        uint32_t x[64];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int4 ra = *reinterpret_cast<const int4 *>(buf + swz(lane, q));
+            const int4 rb = *reinterpret_cast<const int4 *>(buf + swz(lane, q + 4));
+            const uint32_t wa[4] = {(uint32_t)ra.x, (uint32_t)ra.y, (uint32_t)ra.z, (uint32_t)ra.w};
+            const uint32_t wb[4] = {(uint32_t)rb.x, (uint32_t)rb.y, (uint32_t)rb.z, (uint32_t)rb.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint32_t ae = (wa[i] ^ 0x80808080u) & 0x00FF00FFu, ao = (wa[i] ^ 0x80808080u) & 0xFF00FF00u;
+                const uint32_t be = (wb[i] ^ 0x80808080u) & 0x00FF00FFu, bo = (wb[i] ^ 0x80808080u) & 0xFF00FF00u;
+                const int j = 16 * q + 4 * i;
+                x[j] = prmt(ae, be, 0x5410u);
+                x[j + 1] = prmt(ao, bo, 0x4501u);
+                x[j + 2] = prmt(ae, be, 0x7632u);
+                x[j + 3] = prmt(ao, bo, 0x6723u);
+            }
+        }
+        __syncwarp();                                  // the stage is free for this tile's codes
+#pragma unroll
+        for (int h = 1; h < HB; h <<= 1) {
+#pragma unroll
+            for (int i = 0; i < 64; ++i) {
+                if (i & h) continue;
+                const uint32_t u = x[i], v = x[i + h];
+                if (h == 1) {
+                    // (u + v) carries the bias 2 * 128 of both halves, (u - v)
+                    // none; kBlo on the first pair of a block is kBlo on its
+                    // first input, which the transform spreads to every output
+                    const uint32_t c = (i % HB) == 0 ? kBlo : 0u;
+                    x[i] = u + v - kBias2 + c;
+                    x[i + 1] = u - v + c;
+                } else {
+                    x[i] = u + v;
+                    x[i + h] = u - v;
+                }
+            }
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint32_t oa[4], ob[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                int ql[4], qh[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    // y >= -vmax keeps the code >= -127; above, the saturating
+                    // pack turns every code >= 128 into 127
+                    const uint32_t w = max_s16x2(x[16 * q + 4 * i + k], sp.clo);
+                    ql[k] = swar_requant<HB, TIES>(w & 0xFFFFu, sp.clow, sp.mult, sp.shift);
+                    qh[k] = swar_requant<HB, TIES>((uint32_t)((int)w >> 16), sp.chigh, sp.mult, sp.shift);
+                }
+                oa[i] = pack4s(ql[0], ql[1], ql[2], ql[3]);
+                ob[i] = pack4s(qh[0], qh[1], qh[2], qh[3]);
+            }
+            *reinterpret_cast<int4 *>(buf + swz(lane, q)) = make_int4((int)oa[0], (int)oa[1], (int)oa[2], (int)oa[3]);
+            *reinterpret_cast<int4 *>(buf + swz(lane, q + 4)) = make_int4((int)ob[0], (int)ob[1], (int)ob[2], (int)ob[3]);
+        }
+        __syncwarp();
+        const long long e0 = t << 12;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int c = 32 * i + lane;
+            if (e0 + 16 * c < a.total)
+                *reinterpret_cast<int4 *>(a.y + e0 + 16 * c) = *reinterpret_cast<const int4 *>(buf + swz(c >> 3, c & 7));
+        }
+        __syncwarp();                                  // every lane has read the stage back
+        issue(t + kSwarStages * nwarps, slot);
+        slot = slot + 1 == kSwarStages ? 0 : slot + 1;
+    }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
 // round(num / den) half to even for num, den > 0.
 __device__ long long div_rne(unsigned long long num, unsigned long long den) {
     unsigned long long q = num / den, r = num % den;
@@ -411,10 +637,106 @@ int grid_for(long long total, K k) {
 
 }  // namespace
 
-cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s) {
-    if (a.f16) act_quant_kernel<true, 0><<<grid_for(a.total, act_quant_kernel<true, 0>), kThreads, 0, s>>>(a);
-    else act_quant_kernel<false, 0><<<grid_for(a.total, act_quant_kernel<false, 0>), kThreads, 0, s>>>(a);
+template <int HB>
+cudaError_t launch_wide(const ActQuantArgs &a, cudaStream_t s) {
+    // grid_for counts 512-element warp tiles; a wide tile is 2048 elements
+    if (a.shift <= 30) {
+        auto k = act_quant_i8_wide_kernel<HB, true>;
+        k<<<grid_for((a.total + 3) / 4, k), kThreads, 0, s>>>(a);
+    } else {
+        auto k = act_quant_i8_wide_kernel<HB, false>;
+        k<<<grid_for((a.total + 3) / 4, k), kThreads, 0, s>>>(a);
+    }
     return cudaGetLastError();
+}
+
+// round(M y / 2^n) half to even, 64-bit host arithmetic (the kernels' function).
+long long host_rne(long long p, int n) {
+    if (n <= 0) return p;
+    return (p + ((1LL << (n - 1)) - 1) + ((p >> n) & 1)) >> n;
+}
+
+template <int HB>
+cudaError_t launch_swar(const ActQuantArgs &a, cudaStream_t s) {
+    const long long m = a.mult;
+    const int n = a.shift;
+    // |y| <= vmax keeps round(M y / 2^n) within [-127, 127]; with M <= 2^n the
+    // codes step by at most one, so clamping y below at -vmax gives code -127
+    // exactly where the clamp of the code would (codes above 127 saturate in
+    // the pack).
+    long long lo = 0, hi = 127LL * HB;
+    if (host_rne(m * hi, n) > 127) {
+        while (lo < hi) {
+            const long long mid = (lo + hi + 1) / 2;
+            if (host_rne(m * mid, n) <= 127) lo = mid;
+            else hi = mid - 1;
+        }
+    }
+    const long long vmax = hi;
+    // A tie M y = 2^(n-1) (mod 2^n) needs |y| >= 2^(n-1-t), t the trailing zeros of M.
+    int t = 0;
+    while (t < n && ((m >> t) & 1) == 0) ++t;
+    const bool ties = t < n && (1LL << (n - 1 - t)) <= vmax;
+    const uint32_t blo = HB >= 2 ? 128u * HB : 128u, bhi = HB >= 2 ? 0u : 128u;
+    auto pair = [](long long lo16, long long hi16) {
+        return (uint32_t)(lo16 & 0xFFFF) | ((uint32_t)(hi16 & 0xFFFF) << 16);
+    };
+    SwarParams sp;
+    sp.clo = pair(-vmax + blo, -vmax + bhi);
+    const uint32_t half = (1u << (n - 1)) - (ties ? 1u : 0u);
+    sp.mult = (uint32_t)m;
+    sp.clow = half - (uint32_t)m * blo;
+    sp.chigh = half - (uint32_t)m * bhi;
+    sp.shift = n;
+    auto grid = [&](auto k) {
+        const long long want = ((a.total + 4095) / 4096 + kSwarWarps - 1) / kSwarWarps;
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kSwarWarps * 32, 0) != cudaSuccess || per_sm < 1)
+            per_sm = 4;
+        const long long cap = (long long)num_sms() * per_sm;
+        return (int)(want < cap ? want : cap);
+    };
+    if (ties) {
+        auto k = act_quant_i8_swar_kernel<HB, true>;
+        k<<<grid(k), kSwarWarps * 32, 0, s>>>(a, sp);
+    } else {
+        auto k = act_quant_i8_swar_kernel<HB, false>;
+        k<<<grid(k), kSwarWarps * 32, 0, s>>>(a, sp);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s) {
+    // packed pairs: INT8 entry, blocks of at most 64, 32-bit requantization
+    // (1 <= n <= 30) and M <= 2^n (codes step by at most one)
+    if (!a.f16 && a.hb <= 64 && a.shift >= 1 && a.shift <= 30 && a.mult <= (1LL << a.shift)) {
+        switch (a.hb) {
+            case 1: return launch_swar<1>(a, s);
+            case 2: return launch_swar<2>(a, s);
+            case 4: return launch_swar<4>(a, s);
+            case 8: return launch_swar<8>(a, s);
+            case 16: return launch_swar<16>(a, s);
+            case 32: return launch_swar<32>(a, s);
+            case 64: return launch_swar<64>(a, s);
+            default: break;
+        }
+    }
+    if (a.f16) {
+        act_quant_kernel<true, 0><<<grid_for(a.total, act_quant_kernel<true, 0>), kThreads, 0, s>>>(a);
+        return cudaGetLastError();
+    }
+    switch (a.hb) {
+        case 1: return launch_wide<1>(a, s);
+        case 2: return launch_wide<2>(a, s);
+        case 4: return launch_wide<4>(a, s);
+        case 8: return launch_wide<8>(a, s);
+        case 16: return launch_wide<16>(a, s);
+        case 32: return launch_wide<32>(a, s);
+        case 64: return launch_wide<64>(a, s);
+        default:
+            act_quant_kernel<false, 0><<<grid_for(a.total, act_quant_kernel<false, 0>), kThreads, 0, s>>>(a);
+            return cudaGetLastError();
+    }
 }
 
 cudaError_t launch_act_affine(const AffineQuantArgs &a, cudaStream_t s) {

@@ -63,6 +63,28 @@ def test_quantize_i8_static_bit_exact(H, shape, hb):
     assert np.array_equal(host(y), ref)
 
 
+# (shape, hb, s_in, rho = s_in / (sqrt(hb) s_x)): rho <= 1 takes the packed
+# 16-bit-pair kernel; rho = 1/4 at hb = 64 gives M = 2^(n-2), where rounding
+# ties occur; rho = 1 gives M = 2^n; odd totals leave a lane half-empty.
+PACKED = [((2, 37, 41, 192), 64, 0.05, 0.3), ((1, 4, 6, 64), 64, 0.5, 0.25), ((1, 5, 5, 64), 64, 0.5, 1.0),
+          ((1, 1, 3, 48), 16, 0.05, 0.7), ((1, 1, 5, 16), 16, 0.05, 0.9), ((1, 3, 7, 96), 32, 0.05, 0.05),
+          ((1, 2, 9, 48), 1, 0.05, 0.9), ((1, 6, 7, 64), 2, 0.05, 0.5), ((3, 3, 5, 32), 8, 0.05, 0.4),
+          ((1, 7, 3, 128), 4, 0.05, 0.6)]
+
+
+@pytest.mark.parametrize("shape,hb,s_in,rho", PACKED)
+def test_quantize_i8_packed_pairs_bit_exact(H, shape, hb, s_in, rho):
+    x = I.activations_i8(shape, seed=400 + hb, s_in=s_in)
+    x.reshape(-1)[: min(64, x.size)] = 127                 # coherent blocks: |y| = 127 hb, saturating codes
+    s_x = float(np.float32(s_in / (np.sqrt(hb) * rho)))
+    y = H.quantize_act(dev(x), H.IN_I8, s_in, hb, s_x)
+    H.sync_status()
+    ref = O.quantize_act_i8(x, hb, s_in, s_x)
+    assert np.array_equal(host(y), ref)
+    if rho * hb >= 1:                                       # the coherent block's code rho 127 hb saturates
+        assert (np.abs(ref.astype(int)) == 127).any()
+
+
 @pytest.mark.parametrize("shape,hb", [((1, 16, 16, 128), 128), ((2, 5, 7, 192), 64), ((1, 3, 3, 256), 256),
                                       ((1, 4, 5, 32), 16)])
 def test_quantize_f16_static_within_tolerance(H, shape, hb):
