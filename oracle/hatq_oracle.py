@@ -44,6 +44,15 @@ Readings the paper leaves open (the same list is kept with the design notes):
   R11 dynamic affine activations: unsigned 8-bit codes (q_min 0, q_max 255),
      a zero range gives (s, z) = (1, 0), the input-side operand (T x for DH)
      is quantized and padding is a centred zero.
+  R21 phi_int for GDN / IGDN (Eq. supp_general_activation) in integers:
+     G_ij = rint(gamma_ij s_z^2 2^e), B_i = max(1, rint(beta_i 2^e)) with the
+     largest e such that max G <= 511 and max_i (B_i + 127^2 sum_j G_ij) < 2^31;
+     D_i = B_i + sum_j G_ij z_j^2 (exact). GDN: X_i = R |z_i| / sqrt(D_i) with
+     R^2 = (s_z / s_u)^2 2^e; IGDN: X_i = R |z_i| sqrt(D_i) with
+     R^2 = (s_z / s_u)^2 2^-e. R^2 ~ P / 2^t (largest t keeping the tests below
+     in 63 bits, P >= 2^15). |u_i| = min(127, round(X_i)) with ties away from
+     zero, decided exactly: the largest k with (2k - 1)^2 D_i 2^t <= 4 P z_i^2
+     (GDN) or (2k - 1)^2 2^t <= 4 P z_i^2 D_i (IGDN); u_i takes the sign of z_i.
 
 parity unpinned: the rounding convention R2 and the (M, n) rule R3 are
 conventions of this implementation (the paper fixes neither); the oracle pins
@@ -416,13 +425,13 @@ def activation_lut(kind: str, s_z: float, s_u: float) -> np.ndarray:
 def prepare_layer(w_ohwi, b, form: str, hb_in: int, hb_out: int, s_x: float,
                   s_y: float, act: str, hb_next: int, out_f32: bool,
                   stride: int, pad: int, s_z: float = None, s_u: float = None,
-                  order_in: int = 0) -> Prepared:
+                  order_in: int = 0, gdn_beta=None, gdn_gamma=None) -> Prepared:
     """Offline preparation of one layer (Sec. deployment realization).
     s_x: scale of the INT8 operand this layer consumes; s_y: scale of the
     INT8 operand the next layer consumes (or of this layer's output).
-    A non-homogeneous act ('silu', 'gelu') takes the two-step transition of
-    Sec. general nonlinearities with preactivation scale s_z and activation
-    scale s_u. order_in > 0 (DH only): the input side takes the paper's
+    A non-homogeneous act ('silu', 'gelu'; 'gdn', 'igdn' with gdn_beta,
+    gdn_gamma) takes the two-step transition of Sec. general nonlinearities
+    with preactivation scale s_z and activation scale s_u. order_in > 0 (DH only): the input side takes the paper's
     single order m = order_in instead of blocks, W' = W (I (x) P_C H_m)
     (Eqs. supp_padded_transforms, supp_padded_dh); the layer then consumes an
     operand of m channels."""
@@ -460,6 +469,7 @@ def prepare_layer(w_ohwi, b, form: str, hb_in: int, hb_out: int, s_x: float,
         # Eq. supp_general_output_scale: s_A,c / (gamma_out s_z) ~ M_out / 2^n_out, M before H_out
         prep.M, prep.n = fixed_point(s_a / (g_out * s_z), a_bound, hb_out if form == "WH" else 1)
         prep.lut = activation_lut(act, s_z, s_u) if act in GENERAL_ACTS else None
+        prep.gdn = gdn_params(gdn_beta, gdn_gamma, s_z, s_u, act == "igdn") if act in VECTOR_ACTS else None
         # Eq. supp_general_input_scale: s_u / (gamma_in,next s_x,next) ~ M_in / 2^n_in
         M_in, n_in = fixed_point([s_u / (g_in * s_y)], [QMAX], hb_next if hb_next else 1)
         prep.M_in, prep.n_in = int(M_in[0]), n_in
@@ -662,19 +672,117 @@ def gdn(v, beta, gamma, inverse: bool = False) -> np.ndarray:
     return v * norm if inverse else v / norm
 
 
-def epilogue_general_vector(acc, p: Prepared, phi_vec) -> np.ndarray:
-    """The transition of Sec. general nonlinearities for a channel-coupled
-    activation (GDN / IGDN): z as in epilogue_general, then per pixel
-    u = clamp(round(phi(s_z z) / s_u)) with phi on the whole channel vector
-    (fp64, rounded half to even), then the input-side rescale."""
+class GdnParams:
+    """Integer parameters of phi_int for GDN / IGDN (reading R21)."""
+
+    def __init__(self, **kw):
+        self.__dict__.update(kw)
+
+
+GDN_G_MAX = 511                 # 9-bit G: G z^2 limb products stay exact in fp32 sums
+GDN_D_LIMIT = 2 ** 31
+GDN_P_MIN = 2 ** 15
+
+
+def gdn_params(beta, gamma, s_z: float, s_u: float, inverse: bool = False) -> GdnParams:
+    """phi_int of Eq. (supp_general_activation) for y_i = v_i / sqrt(beta_i +
+    sum_j gamma_ij v_j^2) (IGDN: times the root) with v = s_z z, read as R21:
+    the normalization pool in integers D_i = B_i + sum_j G_ij z_j^2 and the
+    rounding of R |z| / sqrt(D) (IGDN: R |z| sqrt(D)) decided by squares."""
+    beta = np.asarray(beta, dtype=np.float64).ravel()
+    gamma = np.asarray(gamma, dtype=np.float64)
+    c = beta.size
+    if gamma.shape != (c, c):
+        raise ValueError("gamma must be C x C")
+    if not (np.all(np.isfinite(beta)) and np.all(np.isfinite(gamma))):
+        raise ValueError("beta and gamma must be finite")
+    if np.any(beta <= 0) or np.any(gamma < 0):
+        raise ValueError("GDN needs beta > 0 and gamma >= 0")
+    s_z = float(np.float32(s_z))
+    s_u = float(np.float32(s_u))
+    if not (s_z > 0 and s_u > 0):
+        raise ValueError("scales must be positive")
+    gs = gamma * s_z * s_z
+    for e in range(62, -126, -1):
+        if gs.max(initial=0.0) * 2.0 ** e >= GDN_G_MAX + 0.5 or beta.max() * 2.0 ** e >= GDN_D_LIMIT:
+            continue
+        G = np.rint(gs * 2.0 ** e).astype(np.int64)
+        B = np.maximum(1, np.rint(beta * 2.0 ** e)).astype(np.int64)
+        d_max = int(np.max(B + QMAX * QMAX * G.sum(axis=1)))
+        if d_max < GDN_D_LIMIT:
+            break
+    else:
+        raise OverflowError("no scaling keeps the GDN pool in range")
+    r2 = (s_z / s_u) ** 2 * (2.0 ** -e if inverse else 2.0 ** e)
+    for t in range(62, -1, -1):
+        P = int(np.rint(math.ldexp(r2, t)))
+        if inverse:
+            ok = (2 * QMAX - 1) ** 2 * 2 ** t < 2 ** 63 and 4 * P * QMAX * QMAX * d_max < 2 ** 63
+        else:
+            ok = (2 * QMAX - 1) ** 2 * d_max * 2 ** t < 2 ** 63 and 4 * P * QMAX * QMAX < 2 ** 63
+        if ok:
+            break
+    else:
+        raise OverflowError("no fixed-point R^2 fits the 63-bit tests")
+    if P < GDN_P_MIN:
+        raise OverflowError("fewer than 16 bits in the fixed-point R^2")
+    return GdnParams(G=G, B=B, e=e, P=P, t=t, inverse=bool(inverse), d_max=d_max, c=c)
+
+
+def gdn_pool(z, g: GdnParams) -> np.ndarray:
+    """D_i = B_i + sum_j G_ij z_j^2 over the last axis (exact int64)."""
+    z2 = np.asarray(z, dtype=np.int64) ** 2
+    return g.B + z2 @ g.G.T
+
+
+def isqrt_floor(q) -> np.ndarray:
+    """floor(sqrt(q)) elementwise for 0 <= q < 2^52, exact (float estimate
+    corrected by integer comparisons)."""
+    q = np.asarray(q, dtype=np.int64)
+    s = np.floor(np.sqrt(q.astype(np.float64))).astype(np.int64)
+    s = np.where(s * s > q, s - 1, s)
+    s = np.where((s + 1) * (s + 1) <= q, s + 1, s)
+    return s
+
+
+def gdn_int(z, g: GdnParams) -> np.ndarray:
+    """u = phi_int(z) for GDN / IGDN (R21): |u| is the largest k <= 127 with
+    (2k - 1)^2 Den <= Num, i.e. k <= (isqrt(floor(Num / Den)) + 1) / 2, where
+    GDN: Num = 4 P z^2, Den = D 2^t; IGDN: Num = 4 P z^2 D, Den = 2^t."""
+    z = np.asarray(z, dtype=np.int64)
+    D = gdn_pool(z, g)
+    z2 = z * z
+    if g.inverse:
+        q = (4 * g.P * z2 * D) >> g.t
+    else:
+        q = (4 * g.P * z2) // (D << g.t)
+    q = np.minimum(q, (2 * QMAX + 1) ** 2)        # any S >= 253 gives |u| = 127
+    k = np.minimum(QMAX, (isqrt_floor(q) + 1) // 2)
+    return np.sign(z) * k
+
+
+def input_transition(u, p: Prepared) -> np.ndarray:
+    """Eq. (supp_general_input_transition): x_next = clamp(round(H~_in,next
+    (M_in u) / 2^n_in), -127, 127)."""
+    w = p.M_in * np.asarray(u, dtype=np.int64)
+    w = transform_int(w, p.hb_next) if p.hb_next else w
+    return np.clip(rshift_rne(w, p.n_in), -QMAX, QMAX).astype(np.int8)
+
+
+def preactivation(acc, p: Prepared) -> np.ndarray:
+    """Eq. (supp_general_preactivation): z = clamp(round(H~_out (M_out (.) a)
+    / 2^n_out), -127, 127) with a = acc + b_int."""
     a = np.asarray(acc, dtype=np.int64) + p.b_int
     t = p.M * a
     v = transform_int(t, p.hb_out) if p.hb_out else t
-    z = np.clip(rshift_rne(v, p.n), -QMAX, QMAX)
-    u = np.clip(np.rint(phi_vec(p.s_z * z.astype(np.float64)) / p.s_u), -QMAX, QMAX).astype(np.int64)
-    w = p.M_in * u
-    w = transform_int(w, p.hb_next) if p.hb_next else w
-    return np.clip(rshift_rne(w, p.n_in), -QMAX, QMAX).astype(np.int8)
+    return np.clip(rshift_rne(v, p.n), -QMAX, QMAX)
+
+
+def epilogue_general_vector(acc, p: Prepared) -> np.ndarray:
+    """The transition of Sec. general nonlinearities for a channel-coupled
+    activation (GDN / IGDN): z by Eq. supp_general_preactivation, u = phi_int(z)
+    on each pixel's channel vector (R21), then the input-side rescale."""
+    return input_transition(gdn_int(preactivation(acc, p), p.gdn), p)
 
 
 def epilogue_f32(acc, p: Prepared) -> np.ndarray:

@@ -16,7 +16,7 @@ _orig = {k: getattr(O, k) for k in ("sylvester", "transform_real", "transform_in
                                     "act_multiplier", "range_expansion_codes", "select_form",
                                     "epilogue_general", "phi", "paley1", "padded_transforms",
                                     "_jacobsthal", "conv_transpose_codes", "conv_transpose_real",
-                                    "depth_to_space", "affine_params", "conv_layer_affine", "gdn",
+                                    "depth_to_space", "affine_params", "conv_layer_affine", "gdn", "gdn_pool", "gdn_int",
                                     "transform_order_real", "transform_order_int", "quantize_act_order_i8",
                                     "hadamard_of_order")}
 
@@ -206,6 +206,21 @@ def _igdn_divides(v, beta, gamma, inverse=False):
     return _orig["gdn"](v, beta, gamma, False)
 
 
+def _gdn_pool_unsquared(z, g):
+    return g.B + np.abs(np.asarray(z, dtype=np.int64)) @ g.G.T
+
+
+def _gdn_pool_transposed(z, g):
+    return g.B + (np.asarray(z, dtype=np.int64) ** 2) @ g.G
+
+
+def _gdn_int_floor(z, g):
+    z = np.asarray(z, dtype=np.int64)
+    D = O.gdn_pool(z, g)
+    q = (4 * g.P * z * z * D) >> g.t if g.inverse else (4 * g.P * z * z) // (D << g.t)
+    return np.sign(z) * np.minimum(127, O.isqrt_floor(np.minimum(q, 255 ** 2)) // 2)
+
+
 def _order_real_by_sqrt_c(x, m):
     c = np.shape(x)[-1]
     return _orig["transform_order_real"](x, m) * math.sqrt(m) / math.sqrt(c)
@@ -238,6 +253,9 @@ MUTATIONS = {
     "order_quantizer_sqrt_c": ("quantize_act_order_i8", _order_quant_sqrt_c),
     "gdn_norm_unsquared": ("gdn", _gdn_unsquared),
     "igdn_divides": ("gdn", _igdn_divides),
+    "gdn_pool_unsquared": ("gdn_pool", _gdn_pool_unsquared),
+    "gdn_pool_transposed": ("gdn_pool", _gdn_pool_transposed),
+    "gdn_int_floor": ("gdn_int", _gdn_int_floor),
     "affine_zero_point_sign": ("affine_params", _affine_z_sign),
     "affine_zero_not_in_range": ("affine_params", _affine_no_zero_in_range),
     "affine_padding_raw_code": ("conv_layer_affine", _affine_raw_padding),

@@ -850,14 +850,105 @@ def test_gdn_transition_tracks_real_model(inverse):
     b = I.bias(c, seed=132)
     beta = 1.0 + rng.random(c)
     gamma = np.abs(rng.standard_normal((c, c))) * 0.01
-    phi_vec = lambda v: O.gdn(v, beta, gamma, inverse)
     y = O.conv_real(x_real, w, b, 1, 1)
-    u = phi_vec(y)
+    u = O.gdn(y, beta, gamma, inverse)
     s_x = O.symmetric_scale(O.transform_real(x_real, 64))
     s_z, s_u = O.symmetric_scale(y), O.symmetric_scale(u)
     p = O.prepare_layer(w, b, "DH", 64, 0, s_x, s_u, "igdn" if inverse else "gdn", 0, False, 1, 1,
-                        s_z=s_z, s_u=s_u)
+                        s_z=s_z, s_u=s_u, gdn_beta=beta, gdn_gamma=gamma)
     op = O.quantize_act_f16(x_real.astype(np.float16), 64, s_x)
     acc = O.conv_codes(op, p.w_int, 1, 1)
-    got = O.epilogue_general_vector(acc, p, phi_vec).astype(np.float64) * p.s_y
+    got = O.epilogue_general_vector(acc, p).astype(np.float64) * p.s_y
     assert O.sqnr_db(u, got) > 24.0
+
+
+def _round_half_away(x):
+    return np.sign(x) * np.floor(np.abs(x) + 0.5)
+
+
+def _gdn_case(c, seed, inverse, gamma_scale=0.01):
+    rng = np.random.default_rng(seed)
+    beta = 0.5 + rng.random(c)
+    gamma = np.abs(rng.standard_normal((c, c))) * gamma_scale
+    z = rng.integers(-127, 128, (400, c))
+    z[0] = 127
+    z[1] = 0
+    z[2, : c // 2] = -127
+    s_z = 0.04
+    y = O.gdn(s_z * z.astype(np.float64), beta, gamma, inverse)
+    s_u = float(np.float32(np.abs(y).max() / 120.0))
+    return beta, gamma, z, s_z, s_u, y
+
+
+@pytest.mark.parametrize("inverse", [False, True])
+@pytest.mark.parametrize("c", [16, 64, 192])
+def test_gdn_int_rounds_the_real_gdn(inverse, c):
+    """R21: phi_int(z) is round(phi(s_z z) / s_u) up to the 9-bit pool
+    coefficients and the fixed-point R^2: never more than one code away from
+    the fp64 model, equal on at least 97% of the codes, and the pool
+    parameters respect their bounds."""
+    beta, gamma, z, s_z, s_u, y = _gdn_case(c, 40 + c, inverse)
+    g = O.gdn_params(beta, gamma, s_z, s_u, inverse)
+    assert g.G.max() <= 511 and g.d_max < 2 ** 31 and g.P >= 2 ** 15
+    assert g.G.max() >= 256                                     # e is the largest admissible
+    u = O.gdn_int(z, g)
+    ref = np.clip(_round_half_away(y / s_u), -127, 127)
+    d = np.abs(u - ref)
+    assert d.max() <= 1 and np.mean(d > 0) < 0.03
+    assert np.abs(u).max() >= 118
+
+
+def test_gdn_int_is_the_largest_admissible_code():
+    """Brute force on three channels: |u| is the largest k in [0, 127] with
+    (2k - 1)^2 D 2^t <= 4 P z^2 (GDN) / (2k - 1)^2 2^t <= 4 P z^2 D (IGDN),
+    found by trying every k with Python integers; D itself by the definition
+    B_i + sum_j G_ij z_j^2 written out term by term."""
+    rng = np.random.default_rng(3)
+    beta = np.array([0.7, 1.3, 0.2])
+    gamma = np.array([[0.1, 0.02, 0.0], [0.03, 0.2, 0.05], [0.0, 0.01, 0.3]])
+    for inverse in (False, True):
+        g = O.gdn_params(beta, gamma, 0.05, 0.012 if not inverse else 0.05, inverse)
+        z = rng.integers(-127, 128, (60, 3))
+        u = O.gdn_int(z, g)
+        for r in range(z.shape[0]):
+            for i in range(3):
+                D = int(g.B[i]) + sum(int(g.G[i, j]) * int(z[r, j]) ** 2 for j in range(3))
+                zi = int(z[r, i])
+                best = 0
+                for k in range(1, 128):
+                    lhs = (2 * k - 1) ** 2 * (2 ** g.t if inverse else D * 2 ** g.t)
+                    rhs = 4 * g.P * zi * zi * (D if inverse else 1)
+                    if lhs <= rhs:
+                        best = k
+                assert int(u[r, i]) == (best if zi >= 0 else -best)
+
+
+def test_gdn_int_gamma_zero_and_symmetries():
+    """gamma = 0: the pool is beta alone, u = round(s_z z / (s_u sqrt(beta)))
+    within one code; phi_int is odd in z; permuting the channels of z, beta
+    and gamma permutes u; IGDN of the GDN codes returns z within 2 codes
+    when gamma = 0 (the two roots cancel)."""
+    c = 8
+    beta = np.linspace(0.5, 2.0, c)
+    z = np.random.default_rng(5).integers(-127, 128, (200, c))
+    g0 = O.gdn_params(beta, np.zeros((c, c)), 0.05, 0.05 / np.sqrt(0.5), False)
+    u = O.gdn_int(z, g0)
+    ref = _round_half_away(0.05 * z / (0.05 / np.sqrt(0.5) * np.sqrt(beta)))
+    assert np.abs(u - np.clip(ref, -127, 127)).max() <= 1
+    assert np.array_equal(O.gdn_int(-z, g0), -u)
+    inv = O.gdn_params(beta, np.zeros((c, c)), 0.05 / np.sqrt(0.5), 0.05, True)
+    assert np.abs(O.gdn_int(u, inv) - z).max() <= 2
+    beta2, gamma2, z2, s_z, s_u, _ = _gdn_case(c, 7, False, 0.05)
+    g = O.gdn_params(beta2, gamma2, s_z, s_u)
+    perm = np.random.default_rng(8).permutation(c)
+    gp = O.gdn_params(beta2[perm], gamma2[np.ix_(perm, perm)], s_z, s_u)
+    assert np.array_equal(O.gdn_int(z2[:, perm], gp), O.gdn_int(z2, g)[:, perm])
+
+
+def test_gdn_params_reject_invalid():
+    with pytest.raises(ValueError):
+        O.gdn_params([1.0, 0.0], np.zeros((2, 2)), 0.1, 0.1)
+    with pytest.raises(ValueError):
+        O.gdn_params([1.0, 1.0], -np.ones((2, 2)), 0.1, 0.1)
+    with pytest.raises(ValueError):
+        O.gdn_params([1.0, 1.0], np.zeros((3, 3)), 0.1, 0.1)
