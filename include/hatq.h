@@ -441,6 +441,67 @@ hatq_status hatq_conv2d_affine(const int16_t *x, int n, int h, int w, const hatq
  * Host only, synchronous; HATQ_ERR_INVALID_ARG for a bad argument. */
 hatq_status hatq_select_form(const uint8_t *expands, int n, int tau_num, int tau_den, int *form, int *expanded);
 
+/*
+ * GDN / IGDN transition (Sec. general nonlinearities, Eqs.
+ * supp_general_activation, supp_general_input_scale,
+ * supp_general_input_transition) for the channel-coupled activations
+ * y_i = v_i / sqrt(beta_i + sum_j gamma_ij v_j^2) (IGDN: times the root),
+ * v = s_z z. The layer before emits the integer preactivation z of
+ * Eq. supp_general_preactivation: prepare it with hatq_prepare_weights,
+ * act HATQ_ACT_NONE, hb_next 0 and output scale s_y = s_z. phi_int in
+ * integers:
+ *   G_ij = rint(gamma_ij s_z^2 2^e), B_i = max(1, rint(beta_i 2^e)), e the
+ *     largest integer with max G <= 511 and max_i (B_i + 127^2 sum_j G_ij) < 2^31;
+ *   D_i = B_i + sum_j G_ij z_j^2 (per pixel, exact);
+ *   R^2 = (s_z / s_u)^2 2^e (GDN) or 2^-e (IGDN), P = rint(R^2 2^t) with the
+ *     largest t in [0, 62] keeping every comparison below in 63 bits; P >= 2^15;
+ *   |u_i| = the largest k <= 127 with (2k - 1)^2 D_i 2^t <= 4 P z_i^2 (GDN),
+ *     (2k - 1)^2 2^t <= 4 P z_i^2 D_i (IGDN): round(R |z_i| / sqrt(D_i)) (IGDN:
+ *     R |z_i| sqrt(D_i)) with ties away from zero, clamped to 127; u_i takes
+ *     the sign of z_i;
+ *   x = clamp(round(H~_next (M_in u) / 2^n_in), -127, 127) with
+ *     s_u / (gamma_in,next s_y) ~ M_in / 2^n_in by the (M, n) rule of
+ *     hatq_prepare_weights (bound 127).
+ * Real arithmetic in fp64; rint rounds half to even.
+ */
+typedef struct {
+    int c;                /* channels: 64, 128, 192 or 256 */
+    int inverse;          /* 0 GDN, 1 IGDN */
+    int hb_next;          /* block of the next layer's DH transform (0: none; else a power of two <= 64) */
+    int e;                /* pool scale exponent */
+    int t;                /* R^2 ~ P / 2^t */
+    int shift_in;         /* n_in */
+    long long P;
+    long long mult_in;    /* M_in */
+    float s_z, s_u, s_y;
+    uint16_t *g_f16;      /* device [c][c] G as IEEE fp16 (exact integers <= 511); set by the caller */
+    int32_t *b_pool;      /* device [c] B_i; set by the caller */
+    uint64_t opaque[16];  /* the library's tensor-memory-access descriptor of g_f16 */
+} hatq_prepared_gdn;
+
+/* The arithmetic of hatq_prepare_gdn into HOST outputs: g [c][c] int32,
+ * b [c] int32, and the scalars. beta [c] (> 0) and gamma [c][c] (>= 0,
+ * row-major, gamma[i * c + j] = gamma_ij) are host float64. Errors:
+ * HATQ_ERR_INVALID_ARG (bad argument), HATQ_ERR_UNSUPPORTED (c or hb_next
+ * outside the list above), HATQ_ERR_OVERFLOW (no e, t or (M_in, n_in)
+ * satisfies the bounds, or P < 2^15). */
+hatq_status hatq_prepare_gdn_host(int c, const double *beta, const double *gamma, float s_z, float s_u, int inverse,
+                                  float s_y, int hb_next, int32_t *g_out, int32_t *b_out, int *e_out, long long *p_out,
+                                  int *t_out, long long *mult_in_out, int *shift_in_out);
+
+/* hatq_prepare_gdn_host, then the upload of G (as fp16) and B to the caller's
+ * device buffers out->g_f16 (c * c elements) and out->b_pool (c), both 16-byte
+ * aligned, and the struct's other fields. Synchronizes `stream`. */
+hatq_status hatq_prepare_gdn(int c, const double *beta, const double *gamma, float s_z, float s_u, int inverse,
+                             float s_y, int hb_next, hatq_prepared_gdn *out, hatq_stream stream);
+
+/* The GDN / IGDN transition on device tensors: z [n][h][w][c] INT8
+ * preactivation codes, y [n][h][w][c] the next layer's INT8 operand (both
+ * 16-byte aligned, not overlapping). The pool runs on the tensor cores (the
+ * squared codes in two exact fp16 limbs times G, fp32 sums below 2^24).
+ * Stream-ordered; device errors surface through hatq_sync_status(). */
+hatq_status hatq_gdn(const int8_t *z, int n, int h, int w, const hatq_prepared_gdn *g, int8_t *y, hatq_stream stream);
+
 /* Failure-detection self test (the paper has no counterpart): launches one
  * thread that waits, through the same bounded mbarrier wait the convolution
  * pipeline uses, on a barrier nothing arrives at. The wait expires after

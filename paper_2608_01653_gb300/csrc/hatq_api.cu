@@ -1048,6 +1048,89 @@ hatq_status transposed_sub_desc(const hatq_conv_desc *d, int cls, hatq_conv_desc
     return HATQ_OK;
 }
 
+// phi_int parameters of GDN / IGDN (the rules of hatq_prepare_gdn_host).
+struct GdnHost {
+    std::vector<int32_t> G, B;
+    int e = 0, t = 0, shift_in = 0;
+    long long P = 0, d_max = 0, mult_in = 0;
+};
+
+hatq_status gdn_host(int c, const double *beta, const double *gamma, float s_z, float s_u, int inverse, float s_y,
+                     int hb_next, GdnHost &h) {
+    if (!beta || !gamma) return fail(HATQ_ERR_INVALID_ARG, "null beta or gamma");
+    if (c != 64 && c != 128 && c != 192 && c != 256) return fail(HATQ_ERR_UNSUPPORTED, "GDN channels must be 64, 128, 192 or 256");
+    if (hb_next != 0 && (!pow2(hb_next) || hb_next > 64))
+        return fail(HATQ_ERR_UNSUPPORTED, "hb_next must be 0 or a power of two <= 64");
+    if (!(s_z > 0.f) || !(s_u > 0.f) || !(s_y > 0.f) || !std::isfinite(s_z) || !std::isfinite(s_u) || !std::isfinite(s_y))
+        return fail(HATQ_ERR_INVALID_ARG, "scales must be positive and finite");
+    const size_t cc = (size_t)c * c;
+    const double sz = (double)s_z, su = (double)s_u, sy = (double)s_y;
+    std::vector<double> gs(cc);
+    double gmax = 0.0, bmax = 0.0;
+    for (int i = 0; i < c; ++i) {
+        if (!(beta[i] > 0.0) || !std::isfinite(beta[i])) return fail(HATQ_ERR_INVALID_ARG, "beta must be positive and finite");
+        bmax = std::max(bmax, beta[i]);
+    }
+    for (size_t i = 0; i < cc; ++i) {
+        if (!(gamma[i] >= 0.0) || !std::isfinite(gamma[i])) return fail(HATQ_ERR_INVALID_ARG, "gamma must be >= 0 and finite");
+        gs[i] = gamma[i] * sz * sz;
+        gmax = std::max(gmax, gs[i]);
+    }
+    h.G.assign(cc, 0);
+    h.B.assign(c, 0);
+    bool found = false;
+    for (int e = 62; e >= -125 && !found; --e) {
+        const double sc = std::ldexp(1.0, e);
+        if (gmax * sc >= 511.5 || bmax * sc >= 2147483648.0) continue;
+        long long dmax = 0;
+        for (int i = 0; i < c; ++i) {
+            const double b = std::nearbyint(beta[i] * sc);
+            h.B[i] = (int32_t)(b < 1.0 ? 1.0 : b);
+            long long sum = 0;
+            for (int j = 0; j < c; ++j) {
+                h.G[(size_t)i * c + j] = (int32_t)std::nearbyint(gs[(size_t)i * c + j] * sc);
+                sum += h.G[(size_t)i * c + j];
+            }
+            dmax = std::max(dmax, (long long)h.B[i] + 16129LL * sum);
+        }
+        if (dmax < (1LL << 31)) {
+            h.e = e;
+            h.d_max = dmax;
+            found = true;
+        }
+    }
+    if (!found) return fail(HATQ_ERR_OVERFLOW, "no scaling keeps the GDN pool in range");
+    const double q = sz / su;
+    const double r2 = q * q * std::ldexp(1.0, inverse ? -h.e : h.e);
+    typedef unsigned __int128 u128;
+    const u128 lim = (u128)1 << 63;
+    found = false;
+    for (int t = 62; t >= 0 && !found; --t) {
+        const double pv = std::nearbyint(std::ldexp(r2, t));
+        if (pv >= 4611686018427387904.0) continue;          // 4 P 127^2 would pass 2^63
+        const long long P = (long long)pv;
+        bool ok;
+        if (inverse)
+            ok = (u128)64009 << t < lim && (u128)4 * (u128)P * 16129u * (u128)h.d_max < lim;
+        else
+            ok = ((u128)64009 * (u128)h.d_max) << t < lim && (u128)4 * (u128)P * 16129u < lim;
+        if (ok) {
+            h.P = P;
+            h.t = t;
+            found = true;
+        }
+    }
+    if (!found) return fail(HATQ_ERR_OVERFLOW, "no fixed-point R^2 fits the 63-bit tests");
+    if (h.P < (1LL << 15)) return fail(HATQ_ERR_OVERFLOW, "fewer than 16 bits in the fixed-point R^2");
+    // Eq. supp_general_input_scale: s_u / (gamma_in,next s_y)
+    const double g_in = hb_next ? std::sqrt((double)hb_next) : 1.0;
+    std::vector<int32_t> m_in;
+    hatq_status st = fixed_point({su / (g_in * sy)}, {127LL}, hb_next ? hb_next : 1, m_in, h.shift_in);
+    if (st != HATQ_OK) return st;
+    h.mult_in = m_in[0];
+    return HATQ_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -1279,6 +1362,131 @@ hatq_status hatq_select_form(const uint8_t *expands, int n, int tau_num, int tau
     // p_l = count / n > tau_num / tau_den, cross-multiplied (no rounding)
     *form = count * (long long)tau_den > (long long)n * tau_num ? HATQ_WH : HATQ_DH;
     if (expanded) *expanded = (int)count;
+    return HATQ_OK;
+}
+
+hatq_status hatq_prepare_gdn_host(int c, const double *beta, const double *gamma, float s_z, float s_u, int inverse,
+                                  float s_y, int hb_next, int32_t *g_out, int32_t *b_out, int *e_out, long long *p_out,
+                                  int *t_out, long long *mult_in_out, int *shift_in_out) {
+    if (!g_out || !b_out || !e_out || !p_out || !t_out || !mult_in_out || !shift_in_out)
+        return fail(HATQ_ERR_INVALID_ARG, "null output");
+    GdnHost h;
+    hatq_status st = gdn_host(c, beta, gamma, s_z, s_u, inverse, s_y, hb_next, h);
+    if (st != HATQ_OK) return st;
+    std::memcpy(g_out, h.G.data(), (size_t)c * c * 4);
+    std::memcpy(b_out, h.B.data(), (size_t)c * 4);
+    *e_out = h.e;
+    *p_out = h.P;
+    *t_out = h.t;
+    *mult_in_out = h.mult_in;
+    *shift_in_out = h.shift_in;
+    return HATQ_OK;
+}
+
+hatq_status hatq_prepare_gdn(int c, const double *beta, const double *gamma, float s_z, float s_u, int inverse,
+                             float s_y, int hb_next, hatq_prepared_gdn *out, hatq_stream stream) {
+    if (!out) return fail(HATQ_ERR_INVALID_ARG, "null output struct");
+    if (!out->g_f16 || !out->b_pool) return fail(HATQ_ERR_INVALID_ARG, "g_f16 and b_pool must be set before preparation");
+    if (!aligned16(out->g_f16) || !aligned16(out->b_pool)) return fail(HATQ_ERR_INVALID_ARG, "device buffers must be 16-byte aligned");
+    GdnHost h;
+    hatq_status st = gdn_host(c, beta, gamma, s_z, s_u, inverse, s_y, hb_next, h);
+    if (st != HATQ_OK) return st;
+    std::vector<uint16_t> g16((size_t)c * c);
+    for (size_t i = 0; i < g16.size(); ++i) g16[i] = f16_bits(h.G[i]);
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e;
+    if ((e = cudaMemcpyAsync(out->g_f16, g16.data(), g16.size() * 2, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaMemcpyAsync(out->b_pool, h.B.data(), (size_t)c * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess ||
+        (e = cudaStreamSynchronize(s)) != cudaSuccess)
+        return cuda_fail(e, "upload of GDN parameters");
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return fail(HATQ_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    // G: [c][c] fp16 (K innermost), 64 x c box, 128-byte swizzle
+    CUtensorMap tm;
+    const cuuint64_t dims[2] = {(cuuint64_t)c, (cuuint64_t)c};
+    const cuuint64_t strides[1] = {(cuuint64_t)c * 2};
+    const cuuint32_t box[2] = {64, (cuuint32_t)c};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(&tm, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, out->g_f16, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "pool tensor map encoding failed (%d)", (int)r);
+    std::memcpy(out->opaque, &tm, sizeof tm);
+    out->c = c;
+    out->inverse = inverse ? 1 : 0;
+    out->hb_next = hb_next;
+    out->e = h.e;
+    out->t = h.t;
+    out->shift_in = h.shift_in;
+    out->P = h.P;
+    out->mult_in = h.mult_in;
+    out->s_z = s_z;
+    out->s_u = s_u;
+    out->s_y = s_y;
+    return HATQ_OK;
+}
+
+hatq_status hatq_gdn(const int8_t *z, int n, int h, int w, const hatq_prepared_gdn *g, int8_t *y, hatq_stream stream) {
+    if (!g) return fail(HATQ_ERR_INVALID_ARG, "null prepared GDN");
+    if (n < 0 || h < 0 || w < 0) return fail(HATQ_ERR_INVALID_ARG, "negative shape");
+    const int c = g->c;
+    if (c != 64 && c != 128 && c != 192 && c != 256) return fail(HATQ_ERR_INVALID_ARG, "the struct was not prepared");
+    const long long pixels = (long long)n * h * w;
+    if (pixels == 0) return HATQ_OK;
+    if (!z || !y) return fail(HATQ_ERR_INVALID_ARG, "null tensor");
+    if (!aligned16(z) || !aligned16(y)) return fail(HATQ_ERR_INVALID_ARG, "z and y must be 16-byte aligned");
+    if (pixels > (1LL << 31) - 256) return fail(HATQ_ERR_UNSUPPORTED, "at most 2^31 - 256 pixels per call");
+    const int8_t *zl = z, *zh = z + pixels * c, *yl = y, *yh = y + pixels * c;
+    if (zl < yh && yl < zh) return fail(HATQ_ERR_INVALID_ARG, "z and y overlap");
+    int dev = 0, smem_max = 0;
+    cudaError_t e;
+    if ((e = cudaGetDevice(&dev)) != cudaSuccess ||
+        (e = cudaDeviceGetAttribute(&smem_max, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev)) != cudaSuccess)
+        return cuda_fail(e, "device query");
+    hatq::GdnArgs a{};
+    a.z = z;
+    a.y = y;
+    a.pixels = pixels;
+    a.c = c;
+    a.inverse = g->inverse;
+    a.hb_next = g->hb_next;
+    a.t = g->t;
+    a.shift_in = g->shift_in;
+    a.P = (unsigned long long)g->P;
+    a.r2f = (float)std::ldexp((double)g->P, -g->t);
+    a.mult_in = g->mult_in;
+    a.b_pool = g->b_pool;
+    a.err = err_word();
+    if (!a.err) return fail(HATQ_ERR_CUDA, "no CUDA device");
+    a.num_tiles = (int)((pixels + 127) / 128);
+    // shared memory: G, nz z tiles, the u rows, B, barriers (plus the 1024-byte alignment slack)
+    const int g_bytes = c * c * 2, z_bytes = 128 * c, u_bytes = 128 * (c + 16);
+    auto layout = [&](int nz) {
+        a.nz = nz;
+        a.z_off = g_bytes;
+        a.u_off = a.z_off + nz * z_bytes;
+        a.b_off = (a.u_off + u_bytes + 127) & ~127;
+        a.bar_off = (a.b_off + 4 * c + 63) & ~63;
+        return a.bar_off + 64 + 1024;
+    };
+    int smem = layout(2);
+    if (smem > smem_max) smem = layout(1);
+    if (smem > smem_max) return fail(HATQ_ERR_UNSUPPORTED, "the GDN tile does not fit shared memory");
+    a.tmem_cols = 2 * c <= 128 ? 128 : (2 * c <= 256 ? 256 : 512);
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return fail(HATQ_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    CUtensorMap tmZ, tmG;
+    std::memcpy(&tmG, g->opaque, sizeof tmG);
+    const cuuint64_t dims[2] = {(cuuint64_t)c, (cuuint64_t)pixels};
+    const cuuint64_t strides[1] = {(cuuint64_t)c};
+    const cuuint32_t box[2] = {64, 128};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(&tmZ, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t *>(z), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "preactivation tensor map encoding failed (%d)", (int)r);
+    if ((e = hatq::launch_gdn(tmZ, tmG, a, smem, reinterpret_cast<cudaStream_t>(stream))) != cudaSuccess)
+        return cuda_fail(e, "GDN launch");
     return HATQ_OK;
 }
 

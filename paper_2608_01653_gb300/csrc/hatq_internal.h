@@ -130,4 +130,23 @@ struct ConvArgs {
 cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const ConvArgs &a,
                         int smem_bytes, cudaStream_t s);
 
+// GDN / IGDN transition kernel (hatq_gdn.cu).
+struct GdnArgs {
+    const int8_t *z;                 // [pixels][c] preactivation codes (read through the tensor map)
+    int8_t *y;                       // [pixels][c] next-layer codes
+    long long pixels;
+    int c, inverse, hb_next, t, shift_in;
+    unsigned long long P;            // R^2 ~ P / 2^t
+    float r2f;                       // P / 2^t (estimate only)
+    long long mult_in;               // M_in
+    const int32_t *b_pool;           // [c] B_i
+    int *err;
+    int num_tiles, nz;               // 128-pixel tiles, z tile buffers (1 or 2)
+    int z_off, u_off, b_off, bar_off;  // shared-memory offsets from the 1024-aligned base
+    int tmem_cols;
+};
+
+cudaError_t launch_gdn(const CUtensorMap &tmZ, const CUtensorMap &tmG, const GdnArgs &a, int smem_bytes,
+                       cudaStream_t s);
+
 }  // namespace hatq

@@ -57,6 +57,14 @@ class PreparedTransposedStruct(ctypes.Structure):
                 ("sub", PreparedStruct * MAX_TRANSPOSED_CLASSES)]
 
 
+class PreparedGdnStruct(ctypes.Structure):
+    _fields_ = [("c", ctypes.c_int), ("inverse", ctypes.c_int), ("hb_next", ctypes.c_int), ("e", ctypes.c_int),
+                ("t", ctypes.c_int), ("shift_in", ctypes.c_int), ("P", ctypes.c_longlong),
+                ("mult_in", ctypes.c_longlong), ("s_z", ctypes.c_float), ("s_u", ctypes.c_float),
+                ("s_y", ctypes.c_float), ("g_f16", ctypes.c_void_p), ("b_pool", ctypes.c_void_p),
+                ("opaque", ctypes.c_uint64 * 16)]
+
+
 _LIB = None
 _P = ctypes.c_void_p
 _I = ctypes.c_int
@@ -109,6 +117,11 @@ def load(build: bool = True) -> ctypes.CDLL:
             "hatq_conv_transpose2d_i8": (_I, [_P, _I, _I, _I, ctypes.POINTER(PreparedTransposedStruct), _P, _P]),
             "hatq_conv2d_i8_subpixel": (_I, [_P, _I, _I, _I, ctypes.POINTER(PreparedStruct), _I, _P, _P]),
             "hatq_layer_noalloc": (_I, [_P, _I, _F, _I, _I, _I, ctypes.POINTER(PreparedStruct), _P, _P]),
+            "hatq_prepare_gdn_host": (_I, [_I, _P, _P, _F, _F, _I, _F, _I, _P, _P, ctypes.POINTER(_I),
+                                           ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(_I),
+                                           ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(_I)]),
+            "hatq_prepare_gdn": (_I, [_I, _P, _P, _F, _F, _I, _F, _I, ctypes.POINTER(PreparedGdnStruct), _P]),
+            "hatq_gdn": (_I, [_P, _I, _I, _I, ctypes.POINTER(PreparedGdnStruct), _P, _P]),
             "hatq_version": (_I, []),
         }
         for name, (res, args) in sig.items():
@@ -443,6 +456,82 @@ def conv_transpose2d_i8(x, T: PreparedTransposed, y=None, stream=None):
     if y is None:
         y = torch.empty(T.out_shape(n, h, w), dtype=torch.float32 if T.out_f32 else torch.int8, device=x.device)
     _check(load().hatq_conv_transpose2d_i8(_ptr(x), n, h, w, ctypes.byref(T.struct), _ptr(y), _stream(stream)))
+    return y
+
+
+@dataclass
+class HostGdn:
+    """hatq_prepare_gdn_host outputs."""
+    G: np.ndarray
+    B: np.ndarray
+    e: int
+    P: int
+    t: int
+    mult_in: int
+    shift_in: int
+
+
+def _gdn_args(c, beta, gamma):
+    beta = np.ascontiguousarray(beta, dtype=np.float64).ravel()
+    gamma = np.ascontiguousarray(gamma, dtype=np.float64)
+    if beta.size != c or gamma.shape != (c, c):
+        raise ValueError(f"beta must have {c} entries and gamma be {c} x {c}")
+    return beta, gamma
+
+
+def prepare_gdn_host(c, beta, gamma, s_z, s_u, inverse, s_y, hb_next=0) -> HostGdn:
+    """hatq_prepare_gdn_host: the integer GDN / IGDN parameters on the host."""
+    beta, gamma = _gdn_args(c, beta, gamma)
+    G = np.zeros((c, c), dtype=np.int32)
+    B = np.zeros(c, dtype=np.int32)
+    e, t, n_in = _I(), _I(), _I()
+    P, m_in = ctypes.c_longlong(), ctypes.c_longlong()
+    _check(load().hatq_prepare_gdn_host(int(c), beta.ctypes.data, gamma.ctypes.data, float(s_z), float(s_u),
+                                        int(bool(inverse)), float(s_y), int(hb_next), G.ctypes.data, B.ctypes.data,
+                                        ctypes.byref(e), ctypes.byref(P), ctypes.byref(t), ctypes.byref(m_in),
+                                        ctypes.byref(n_in)))
+    return HostGdn(G, B, e.value, P.value, t.value, m_in.value, n_in.value)
+
+
+class PreparedGdn:
+    """A prepared GDN / IGDN transition: device G (fp16) and B, and the C
+    struct hatq_prepared_gdn."""
+
+    def __init__(self, c, device="cuda"):
+        torch = _torch()
+        self.c = c
+        self.g_f16 = torch.zeros(c * c, dtype=torch.float16, device=device)
+        self.b_pool = torch.zeros(c, dtype=torch.int32, device=device)
+        self.struct = PreparedGdnStruct()
+        self.struct.g_f16 = self.g_f16.data_ptr()
+        self.struct.b_pool = self.b_pool.data_ptr()
+
+
+def prepare_gdn(c, beta, gamma, s_z, s_u, inverse, s_y, hb_next=0, stream=None, device="cuda") -> PreparedGdn:
+    """hatq_prepare_gdn: phi_int of GDN (inverse False) or IGDN for c channels
+    and the next layer's input transition (block hb_next, scale s_y)."""
+    beta, gamma = _gdn_args(c, beta, gamma)
+    g = PreparedGdn(c, device)
+    _check(load().hatq_prepare_gdn(int(c), beta.ctypes.data, gamma.ctypes.data, float(s_z), float(s_u),
+                                   int(bool(inverse)), float(s_y), int(hb_next), ctypes.byref(g.struct),
+                                   _stream(stream)))
+    return g
+
+
+def gdn(z, g: PreparedGdn, y=None, stream=None):
+    """hatq_gdn on the preactivation codes z (NHWC int8, c channels): the
+    next layer's INT8 operand."""
+    _check_tensor(z, "z", "int8")
+    if z.dim() != 4 or z.shape[-1] != g.c:
+        raise ValueError(f"z must be NHWC with {g.c} channels")
+    if y is not None:
+        _check_tensor(y, "y", "int8", tuple(z.shape))
+    _check_cuda(("z", z), ("y", y))
+    torch = _torch()
+    if y is None:
+        y = torch.empty_like(z)
+    n, h, w, _ = z.shape
+    _check(load().hatq_gdn(_ptr(z), n, h, w, ctypes.byref(g.struct), _ptr(y), _stream(stream)))
     return y
 
 

@@ -408,3 +408,60 @@ def test_transposed_class_sizes(k, s, p, cls, taps):
     assert H.load().hatq_transposed_sizes(ctypes.byref(d), cls, ctypes.byref(w), ctypes.byref(c)) == H.OK
     assert c.value == 128 and w.value == 128 * taps[0] * taps[1] * 64
     assert H.load().hatq_transposed_sizes(ctypes.byref(d), s * s, ctypes.byref(w), ctypes.byref(c)) == H.ERR_INVALID_ARG
+
+
+# ------------------------------------------------ GDN / IGDN (integer phi_int, reading R21)
+
+def _gdn_inputs(c, seed, scale=0.01):
+    rng = np.random.default_rng(seed)
+    beta = 0.5 + rng.random(c)
+    gamma = np.abs(rng.standard_normal((c, c))) * scale
+    return beta, gamma
+
+
+@pytest.mark.parametrize("c,inverse,hb_next", [(64, False, 0), (128, True, 64), (192, False, 16), (256, True, 1),
+                                               (192, True, 32)])
+def test_prepare_gdn_host_matches_oracle(lib, c, inverse, hb_next):
+    """The library's pool coefficients, pool bias, scale exponent, fixed-point
+    R^2 and input-side (M_in, n_in) equal the oracle's (R21 and R3)."""
+    beta, gamma = _gdn_inputs(c, c + int(inverse))
+    s_z, s_u, s_y = 0.043, 0.021 if not inverse else 0.09, 0.05
+    h = H.prepare_gdn_host(c, beta, gamma, s_z, s_u, inverse, s_y, hb_next)
+    g = O.gdn_params(beta, gamma, s_z, s_u, inverse)
+    assert np.array_equal(h.G, g.G) and np.array_equal(h.B, g.B)
+    assert (h.e, h.P, h.t) == (g.e, g.P, g.t)
+    g_in = np.sqrt(hb_next) if hb_next else 1.0
+    M, n = O.fixed_point([float(np.float32(s_u)) / (g_in * float(np.float32(s_y)))], [127], hb_next if hb_next else 1)
+    assert (h.mult_in, h.shift_in) == (int(M[0]), n)
+
+
+def test_gdn_preactivation_layer_is_a_plain_layer():
+    """The GPU runs GDN as a plain layer (act none, output scale s_z) followed
+    by hatq_gdn: its (M, n) equal the general transition's (M_out, n_out)."""
+    w, b = I.weights(64, 3, 3, 64, seed=5), I.bias(64, seed=6)
+    beta, gamma = _gdn_inputs(64, 1)
+    pg = O.prepare_layer(w, b, "DH", 64, 0, 0.02, 0.05, "gdn", 0, False, 1, 1, s_z=0.03, s_u=0.04,
+                         gdn_beta=beta, gdn_gamma=gamma)
+    pp = O.prepare_layer(w, b, "DH", 64, 0, 0.02, 0.03, "none", 0, False, 1, 1)
+    assert np.array_equal(pg.M, pp.M) and pg.n == pp.n
+
+
+def test_prepare_gdn_rejects_on_the_host(lib):
+    beta, gamma = _gdn_inputs(64, 2)
+    with pytest.raises(H.HatqError) as e:
+        H.prepare_gdn_host(96, np.ones(96), np.zeros((96, 96)), 0.1, 0.1, False, 0.1)
+    assert e.value.status == H.ERR_UNSUPPORTED
+    with pytest.raises(H.HatqError) as e:
+        H.prepare_gdn_host(64, beta, gamma, 0.1, 0.1, False, 0.1, hb_next=128)
+    assert e.value.status == H.ERR_UNSUPPORTED
+    bad = beta.copy()
+    bad[3] = 0.0
+    with pytest.raises(H.HatqError) as e:
+        H.prepare_gdn_host(64, bad, gamma, 0.1, 0.1, False, 0.1)
+    assert e.value.status == H.ERR_INVALID_ARG
+    with pytest.raises(H.HatqError) as e:
+        H.prepare_gdn_host(64, beta, -gamma - 1.0, 0.1, 0.1, False, 0.1)
+    assert e.value.status == H.ERR_INVALID_ARG
+    with pytest.raises(ValueError):
+        H.prepare_gdn_host(64, beta[:10], gamma, 0.1, 0.1, False, 0.1)
+    assert lib.hatq_gdn(None, 1, 1, 1, None, None, None) == H.ERR_INVALID_ARG
