@@ -1453,7 +1453,7 @@ hatq_status hatq_gdn(const int8_t *z, int n, int h, int w, const hatq_prepared_g
     a.t = g->t;
     a.shift_in = g->shift_in;
     a.P = (unsigned long long)g->P;
-    a.r2f = (float)std::ldexp((double)g->P, -g->t);
+    a.sr = (float)std::sqrt(std::ldexp((double)g->P, -g->t));
     a.mult_in = g->mult_in;
     a.b_pool = g->b_pool;
     a.err = err_word();
@@ -1466,13 +1466,14 @@ hatq_status hatq_gdn(const int8_t *z, int n, int h, int w, const hatq_prepared_g
         a.z_off = g_bytes;
         a.u_off = a.z_off + nz * z_bytes;
         a.b_off = (a.u_off + u_bytes + 127) & ~127;
-        a.bar_off = (a.b_off + 4 * c + 63) & ~63;
+        a.lut_off = a.b_off + 8 * c;
+        a.bar_off = (a.lut_off + 255 * (g->hb_next > 1 ? g->hb_next : 1) + 1 + 63) & ~63;
         return a.bar_off + 64 + 1024;
     };
     int smem = layout(2);
     if (smem > smem_max) smem = layout(1);
     if (smem > smem_max) return fail(HATQ_ERR_UNSUPPORTED, "the GDN tile does not fit shared memory");
-    a.tmem_cols = 2 * c <= 128 ? 128 : (2 * c <= 256 ? 256 : 512);
+    a.tmem_cols = 512;                   // A limbs (c columns) and two 128-column accumulator buffers
     EncodeTiledFn enc = encode_fn();
     if (!enc) return fail(HATQ_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
     CUtensorMap tmZ, tmG;

@@ -20,19 +20,23 @@
 // below 2^24, so the two fp32 accumulators D_h, D_l in tensor memory hold
 // exact integers and D = 128 D_h + D_l + B.
 //
-// Persistent kernel, 256 threads (8 warps). Warp w owns TMEM lane quadrant
-// w & 3 (pixels 32 (w & 3) .. + 31 of the tile) and half w >> 2 of the work
-// on those pixels. Per tile:
+// Persistent kernel, one CTA per SM, 512 threads (16 warps). Warp w owns TMEM
+// lane quadrant w & 3 (pixels 32 (w & 3) .. + 31 of the tile) and quarter
+// w >> 2 of the work on those pixels. Per tile:
 //   TMA    z tile (c / 64 boxes of 64 x 128 bytes, 64-byte swizzle), two
-//          buffers when shared memory allows, issued one tile ahead;
-//   limbs  half 0 writes limb h, half 1 limb l into TMEM (A operand);
-//   MMA    for each half of the output channels (N = c / 2): D_h, D_l by
-//          c / 16 K-steps each, G (B operand) resident in shared memory;
-//   pool   each thread finishes c / 4 channels of its pixel: D, then u
-//          (float estimate of k, corrected by exact 64-bit comparisons),
-//          into a shared-memory row;
-//   out    64-channel groups of u: Sylvester transform (int32, exact),
-//          M_in multiply and one round-shift, 16-byte stores.
+//          buffers when shared memory allows, issued ahead of use;
+//   limbs  each quarter writes both limbs of its quarter of K into TMEM
+//          (the A operand, two fp16 per column);
+//   MMA    c / 64 passes of 64 output channels, D_h and D_l by c / 16
+//          K-steps each into accumulator buffer p & 1, so the MMAs of pass
+//          p + 1 run while the threads finish pass p; G (the B operand) stays
+//          in shared memory;
+//   pool   each thread finishes 16 channels of its pixel per pass: the float
+//          estimate of the code, exact 64-bit comparisons near a rounding
+//          boundary, u into a shared-memory row;
+//   out    (pixel, 64-channel group) items over all threads: Sylvester block
+//          of u (int32, exact), then a table of clamp(round(M_in v / 2^n_in))
+//          over |v| <= 127 hb built once per CTA, 16-byte stores.
 // Every wait is bounded; the CTA leaves its loop together after a failure.
 #include <cuda_fp16.h>
 
@@ -44,7 +48,7 @@ namespace {
 
 using namespace tc;
 
-constexpr int kGdnThreads = 256;
+constexpr int kGdnThreads = 512;
 
 // two values v0 (low half), v1 in [0, 1023] -> one fp16x2 word, exactly:
 // 0x6400 | v is the fp16 pattern of 1024 + v
@@ -55,43 +59,57 @@ __device__ __forceinline__ uint32_t u10x2_to_f16x2(uint32_t v0, uint32_t v1) {
     return r;
 }
 
-__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
-            taddr),
-        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
-        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
-        : "memory");
+__device__ __forceinline__ uint32_t prmt(uint32_t x, uint32_t y, uint32_t sel) {
+    uint32_t d;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(x), "r"(y), "r"(sel));
+    return d;
 }
 
-// an fp32 accumulator holding an exact integer in [0, 2^24) -> its value
-__device__ __forceinline__ uint32_t acc_int(uint32_t bits) { return __float2uint_rz(__uint_as_float(bits)); }
+__device__ __forceinline__ void tmem_st8(uint32_t taddr, const uint32_t (&r)[8]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8};" ::"r"(taddr), "r"(r[0]),
+                 "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7])
+                 : "memory");
+}
 
-// |u| for one channel: the largest k <= 127 with (2k - 1)^2 den <= num
-// (GDN: den = D 2^t, num = 4 P a^2; IGDN: den = 2^t, num = 4 P a^2 D).
-// The float estimate is exact to well under one code; the loops make the
-// result exact whatever the estimate.
-__device__ __forceinline__ int gdn_code(int zi, uint32_t D, const GdnArgs &a) {
-    if (zi == 0) return 0;
-    const uint32_t ab = (uint32_t)abs(zi);
+// |u| for one channel, exactly: the largest k <= 127 with (2k - 1)^2 den <= num
+// (GDN: den = D 2^t, num = 4 P a^2; IGDN: den = 2^t, num = 4 P a^2 D), i.e.
+// round(X) with ties up for X = a sqrt(P / (2^t D)) (IGDN: a sqrt(P D / 2^t)),
+// searched from the estimate k0 (the loops make it exact whatever k0 is).
+__device__ __noinline__ int gdn_code_exact(uint32_t ab, uint32_t D, int k0, const GdnArgs &a) {
     unsigned long long num = 4ull * a.P * (unsigned long long)(ab * ab);
     unsigned long long den;
-    float x;
     if (a.inverse) {
         num *= D;
         den = 1ull << a.t;
-        x = (float)ab * sqrtf(a.r2f * (float)D);
     } else {
         den = (unsigned long long)D << a.t;
-        x = (float)ab * sqrtf(a.r2f / (float)D);
     }
-    int k = (int)fminf(x + 0.5f, 127.f);
     auto cond = [&](int kk) {
         const unsigned long long o = (unsigned long long)(2 * kk - 1);
         return o * o * den <= num;
     };
+    int k = k0 < 0 ? 0 : (k0 > 127 ? 127 : k0);
     while (k < 127 && cond(k + 1)) ++k;
     while (k > 0 && !cond(k)) --k;
+    return k;
+}
+
+// The code u of one channel from its pool (fp32 limb sums dh, dl of the
+// tensor cores, exact integers) and its preactivation zi. The float estimate
+// X = |z| sr rsqrt(D) (IGDN: |z| sr sqrt(D)), sr = sqrt(P / 2^t), has a
+// relative error below 2^-21 (rsqrt within 2 ulp, five roundings of 2^-24),
+// so below 2^-14 for X < 128: it decides every code whose X lies more than
+// 2^-10 from a half-integer and below 126.5; the rest take the exact path.
+__device__ __forceinline__ int gdn_code(int zi, float dh, float dl, float bf, const int32_t *bi, const GdnArgs &a) {
+    const float zf = __int_as_float(0x4B000000 | (uint32_t)(zi + 128)) - 8388736.0f;   // exact
+    const float df = fmaf(128.0f, dh, dl + bf);
+    const float r = rsqrtf(df);
+    const float x = a.inverse ? zf * a.sr * (df * r) : zf * a.sr * r;                   // signed X
+    const float t = x + 12582912.0f;
+    const float kf = t - 12582912.0f;
+    if (fabsf(x - kf) < 0.4990234375f && fabsf(x) < 126.5f) return __float_as_int(t) - 0x4B400000;
+    const uint32_t D = (__float2uint_rz(dh) << 7) + __float2uint_rz(dl) + (uint32_t)*bi;
+    const int k = gdn_code_exact((uint32_t)abs(zi), D, (int)(fabsf(x) + 0.5f), a);
     return zi < 0 ? -k : k;
 }
 
@@ -109,9 +127,10 @@ __global__ void __launch_bounds__(kGdnThreads, 1)
     uint8_t *bar_area = smem + a.bar_off;
     const uint32_t bar0 = smem_addr(bar_area);
     auto zfull = [&](int b) { return bar0 + 8u * b; };
-    const uint32_t gbar = bar0 + 16u, mma_bar = bar0 + 24u;
-    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_area + 32);
-    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_area + 36);
+    const uint32_t gbar = bar0 + 16u;
+    auto mma_bar = [&](int b) { return bar0 + 24u + 8u * b; };
+    uint32_t *tmem_holder = reinterpret_cast<uint32_t *>(bar_area + 40);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(bar_area + 44);
     const int ustride = c + 16;
 
     __shared__ int s_skip;
@@ -120,7 +139,7 @@ __global__ void __launch_bounds__(kGdnThreads, 1)
     if (s_skip != 0) return;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int quad = warp & 3, half = warp >> 2;
+    const int quad = warp & 3, part = warp >> 2;            // lane quadrant, quarter of the work
     const int m = quad * 32 + lane;                         // pixel row of the tile
     const int my_tiles = a.num_tiles > (int)blockIdx.x ? (a.num_tiles - 1 - (int)blockIdx.x) / (int)gridDim.x + 1 : 0;
 
@@ -128,7 +147,8 @@ __global__ void __launch_bounds__(kGdnThreads, 1)
         mbar_init(zfull(0), 1);
         mbar_init(zfull(1), 1);
         mbar_init(gbar, 1);
-        mbar_init(mma_bar, 1);
+        mbar_init(mma_bar(0), 1);
+        mbar_init(mma_bar(1), 1);
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -138,7 +158,16 @@ __global__ void __launch_bounds__(kGdnThreads, 1)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
-    for (int i = threadIdx.x; i < c; i += kGdnThreads) b_s[i] = a.b_pool[i];
+    float *bf_s = reinterpret_cast<float *>(b_s + c);
+    for (int i = threadIdx.x; i < c; i += kGdnThreads) {
+        b_s[i] = a.b_pool[i];
+        bf_s[i] = (float)a.b_pool[i];
+    }
+    // x = clamp(round(M_in v / 2^n_in)) for every v = H~ u, |v| <= 127 hb; lut_s[v]
+    const int vmax = 127 * (a.hb_next > 1 ? a.hb_next : 1);
+    const int8_t *lut_s = reinterpret_cast<const int8_t *>(smem + a.lut_off) + vmax;
+    for (int v = -vmax + (int)threadIdx.x; v <= vmax; v += kGdnThreads)
+        const_cast<int8_t *>(lut_s)[v] = (int8_t)requant8_any(a.mult_in * (long long)v, a.shift_in);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -157,96 +186,115 @@ __global__ void __launch_bounds__(kGdnThreads, 1)
         for (int j = 0; j < a.nz && j < my_tiles; ++j) issue_z(j);
     }
 
-    // TMEM: A limbs h, l at columns [0, c / 2), [c / 2, c); D_h, D_l at [c, 3c / 2), [3c / 2, 2c)
+    // TMEM: A limbs h, l at columns [0, c / 2), [c / 2, c); accumulator buffer
+    // b at c + 128 b holds D_h (64 columns) and D_l (64 columns) of one pass,
+    // i.e. 64 output channels; pass p uses buffer p & 1, so the MMAs of pass
+    // p + 1 run while the threads finish pass p.
     const uint32_t t_lane = tmem + ((uint32_t)(quad * 32) << 16);
-    const uint32_t idesc = idesc_f16(c / 2);
+    const uint32_t idesc = idesc_f16(64);
     const uint64_t gdesc0 = sdesc_sw128(smem_addr(g_s));
+    const int np = c / 64;
     bool ok = true;
     int issued = a.nz < my_tiles ? a.nz : my_tiles;
-    uint32_t mma_ph = 0;
+    uint32_t mph0 = 0, mph1 = 0;            // next phase parity of each accumulator barrier
+    bool pend0 = false, pend1 = false;      // thread 0: a commit not yet waited for
+    bool g_ready = false;
+    // thread 0: the MMAs of pass p into buffer p & 1 and their commit
+    auto issue_pass = [&](int p) {
+        tc_fence_after();
+        if (!g_ready) {
+            g_ready = mbar_wait(gbar, 0, abort_flag, a.err);
+            if (!g_ready) return;
+        }
+        const int b = p & 1;
+        for (int limb = 0; limb < 2; ++limb) {
+            const uint32_t d = tmem + (uint32_t)(c + 128 * b + 64 * limb);
+            for (int s = 0; s < c / 16; ++s) {
+                const uint64_t bd = gdesc0 + (uint64_t)(((uint32_t)p * 64u * 128u) >> 4) +
+                                    (uint64_t)(((uint32_t)(s >> 2) * c * 128u) >> 4) + (uint64_t)(2 * (s & 3));
+                umma_f16_ts(d, tmem + (uint32_t)(limb * (c / 2) + 8 * s), bd, idesc, s > 0 ? 1u : 0u);
+            }
+        }
+        umma_commit(mma_bar(b));
+        if (b) pend1 = true;
+        else pend0 = true;
+    };
     int j = 0;
     for (; j < my_tiles && ok; ++j) {
         const int b = j % a.nz;
         const uint8_t *zt = z_s + (size_t)b * zbytes;
         ok = __syncthreads_and(mbar_wait(zfull(b), (uint32_t)((j / a.nz) & 1), abort_flag, a.err));
         if (!ok) break;
-        // ---- limbs of z^2 for this pixel row into TMEM
+        // ---- limbs of z^2 for this pixel row into TMEM: this quarter's K range, both limbs
         {
             const int sw = (m >> 1) & 3;
-            for (int k0 = 0; k0 < c; k0 += 32) {
-                uint32_t cols[16];
+            for (int k = part * (c / 4); k < (part + 1) * (c / 4); k += 16) {
+                const uint4 v = *reinterpret_cast<const uint4 *>(zt + (k >> 6) * 8192 + m * 64 +
+                                                                  ((((k & 63) >> 4) ^ sw) << 4));
+                const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+                uint32_t hh[8], ll[8];
 #pragma unroll
-                for (int q = 0; q < 2; ++q) {
-                    const int k = k0 + 16 * q;
-                    const uint4 v = *reinterpret_cast<const uint4 *>(zt + (k >> 6) * 8192 + m * 64 +
-                                                                      ((((k & 63) >> 4) ^ sw) << 4));
-                    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const int z0 = (int)(int8_t)(w[i >> 1] >> (16 * (i & 1)));
-                        const int z1 = (int)(int8_t)(w[i >> 1] >> (16 * (i & 1) + 8));
-                        const uint32_t s0 = (uint32_t)(z0 * z0), s1 = (uint32_t)(z1 * z1);
-                        cols[8 * q + i] = half == 0 ? u10x2_to_f16x2(s0 >> 7, s1 >> 7)
-                                                    : u10x2_to_f16x2(s0 & 127u, s1 & 127u);
-                    }
+                for (int i = 0; i < 8; ++i) {
+                    const int z0 = (int)(int8_t)(w[i >> 1] >> (16 * (i & 1)));
+                    const int z1 = (int)(int8_t)(w[i >> 1] >> (16 * (i & 1) + 8));
+                    const uint32_t s0 = (uint32_t)(z0 * z0), s1 = (uint32_t)(z1 * z1);
+                    hh[i] = u10x2_to_f16x2(s0 >> 7, s1 >> 7);
+                    ll[i] = u10x2_to_f16x2(s0 & 127u, s1 & 127u);
                 }
-                tmem_st16(t_lane + (uint32_t)(half * (c / 2) + k0 / 2), cols);
+                tmem_st8(t_lane + (uint32_t)(k / 2), hh);
+                tmem_st8(t_lane + (uint32_t)(c / 2 + k / 2), ll);
             }
             tmem_wait_st();
         }
         tc_fence_before();
         __syncthreads();
-        for (int nh = 0; nh < 2 && ok; ++nh) {
-            // ---- MMA: D_h, D_l for output channels [nh c / 2, (nh + 1) c / 2)
-            if (threadIdx.x == 0) {
-                tc_fence_after();
-                bool gok = true;
-                if (j == 0 && nh == 0) gok = mbar_wait(gbar, 0, abort_flag, a.err);
-                if (gok) {
-                    for (int limb = 0; limb < 2; ++limb) {
-                        const uint32_t d = tmem + (uint32_t)(c + limb * (c / 2));
-                        for (int s = 0; s < c / 16; ++s) {
-                            const uint64_t bd = gdesc0 + (uint64_t)(((uint32_t)nh * (c / 2) * 128u) >> 4) +
-                                                (uint64_t)(((uint32_t)(s >> 2) * c * 128u) >> 4) + (uint64_t)(2 * (s & 3));
-                            umma_f16_ts(d, tmem + (uint32_t)(limb * (c / 2) + 8 * s), bd, idesc, s > 0 ? 1u : 0u);
-                        }
-                    }
-                    umma_commit(mma_bar);
-                }
-            }
-            ok = __syncthreads_and(mbar_wait(mma_bar, mma_ph, abort_flag, a.err));
-            mma_ph ^= 1u;
+        if (threadIdx.x == 0) {
+            issue_pass(0);
+            if (np > 1) issue_pass(1);
+        }
+        for (int p = 0; p < np && ok; ++p) {
+            const int db = p & 1;
+            ok = __syncthreads_and(mbar_wait(mma_bar(db), db ? mph1 : mph0, abort_flag, a.err));
+            if (db) { mph1 ^= 1u; pend1 = false; }
+            else { mph0 ^= 1u; pend0 = false; }
             if (!ok) break;
             tc_fence_after();
-            // ---- pool and codes u for this thread's c / 4 channels of the half
-            const int ch0 = nh * (c / 2) + half * (c / 4);
-            const int sw = (m >> 1) & 3;
-            for (int g0 = 0; g0 < c / 4; g0 += 16) {
-                const int ch = ch0 + g0;
+            // ---- pool and codes u of channels 64 p + 16 part .. + 15 of this pixel
+            {
+                const int sw = (m >> 1) & 3;
+                const int col = 16 * part;                   // column within the pass
+                const int ch = 64 * p + col;
                 uint32_t dh[16], dl[16];
-                tmem_ld16(t_lane + (uint32_t)(c + (ch - nh * (c / 2))), dh);
-                tmem_ld16(t_lane + (uint32_t)(c + c / 2 + (ch - nh * (c / 2))), dl);
-                tmem_wait_ld();
+                tmem_ld16(t_lane + (uint32_t)(c + 128 * db + col), dh);
+                tmem_ld16(t_lane + (uint32_t)(c + 128 * db + 64 + col), dl);
                 const uint4 zv = *reinterpret_cast<const uint4 *>(zt + (ch >> 6) * 8192 + m * 64 +
                                                                    ((((ch & 63) >> 4) ^ sw) << 4));
+                float bfv[16];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const float4 f4 = reinterpret_cast<const float4 *>(bf_s + ch)[q];
+                    bfv[4 * q] = f4.x; bfv[4 * q + 1] = f4.y; bfv[4 * q + 2] = f4.z; bfv[4 * q + 3] = f4.w;
+                }
+                tmem_wait_ld();
                 const uint32_t zw[4] = {zv.x, zv.y, zv.z, zv.w};
                 uint32_t out[4];
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
-                    uint32_t word = 0;
+                    int u[4];
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
                         const int e = 4 * q + i;
                         const int zi = (int)(int8_t)(zw[q] >> (8 * i));
-                        const uint32_t D = (acc_int(dh[e]) << 7) + acc_int(dl[e]) + (uint32_t)b_s[ch + e];
-                        word |= ((uint32_t)gdn_code(zi, D, a) & 0xFFu) << (8 * i);
+                        u[i] = gdn_code(zi, __uint_as_float(dh[e]), __uint_as_float(dl[e]), bfv[e], b_s + ch + e, a);
                     }
-                    out[q] = word;
+                    out[q] = prmt(prmt((uint32_t)u[0], (uint32_t)u[1], 0x0040u), prmt((uint32_t)u[2], (uint32_t)u[3], 0x0040u),
+                                  0x5410u);
                 }
                 *reinterpret_cast<uint4 *>(u_s + m * ustride + ch) = make_uint4(out[0], out[1], out[2], out[3]);
             }
             tc_fence_before();
             __syncthreads();
+            if (threadIdx.x == 0 && p + 2 < np) issue_pass(p + 2);
         }
         if (!ok) break;
         // the z buffer is free: prefetch the tile that reuses it
@@ -255,31 +303,33 @@ __global__ void __launch_bounds__(kGdnThreads, 1)
             issue_z(issued);
             ++issued;
         }
-        // ---- input transition of the next layer, 64-channel groups
-        const long long pix = (long long)((int)blockIdx.x + j * (int)gridDim.x) * 128 + m;
-        for (int grp = half; grp < c / 64; grp += 2) {
+        // ---- input transition of the next layer: 64-channel groups of u,
+        // Sylvester block (int32, exact: |H~ u| <= 127 hb), then the table of
+        // clamp(round(M_in v / 2^n_in)); work items (row, group) over all threads
+        const long long pix0 = (long long)((int)blockIdx.x + j * (int)gridDim.x) * 128;
+        for (int it = threadIdx.x; it < 128 * (c / 64); it += kGdnThreads) {
+            const int row = it & 127, grp = it >> 7;
             int v[64];
 #pragma unroll
             for (int q = 0; q < 4; ++q) {
-                const uint4 w = *reinterpret_cast<const uint4 *>(u_s + m * ustride + 64 * grp + 16 * q);
+                const uint4 w = *reinterpret_cast<const uint4 *>(u_s + row * ustride + 64 * grp + 16 * q);
                 const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
                 for (int i = 0; i < 16; ++i) v[16 * q + i] = (int)(int8_t)(ww[i >> 2] >> (8 * (i & 3)));
             }
             fwht<64>(v, a.hb_next);
-            if (pix < a.pixels) {
+            if (pix0 + row < a.pixels) {
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     uint32_t wd[4];
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {
                         const int e = 16 * q + 4 * i;
-                        wd[i] = pack4(requant8_any(a.mult_in * (long long)v[e], a.shift_in),
-                                      requant8_any(a.mult_in * (long long)v[e + 1], a.shift_in),
-                                      requant8_any(a.mult_in * (long long)v[e + 2], a.shift_in),
-                                      requant8_any(a.mult_in * (long long)v[e + 3], a.shift_in));
+                        wd[i] = prmt(prmt((uint32_t)lut_s[v[e]], (uint32_t)lut_s[v[e + 1]], 0x0040u),
+                                     prmt((uint32_t)lut_s[v[e + 2]], (uint32_t)lut_s[v[e + 3]], 0x0040u), 0x5410u);
                     }
-                    *reinterpret_cast<uint4 *>(a.y + pix * c + 64 * grp + 16 * q) = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+                    *reinterpret_cast<uint4 *>(a.y + (pix0 + row) * c + 64 * grp + 16 * q) =
+                        make_uint4(wd[0], wd[1], wd[2], wd[3]);
                 }
             }
         }
@@ -288,8 +338,12 @@ __global__ void __launch_bounds__(kGdnThreads, 1)
     // after a failure: wait (bounded) for this CTA's copies and MMAs in flight
     if (!ok && threadIdx.x == 0) {
         const long long t0 = clock64();
-        while (!mbar_try_wait(mma_bar, mma_ph ^ 1u) && clock64() - t0 < kWaitLimitCycles) {
-        }
+        if (pend0)
+            while (!mbar_try_wait(mma_bar(0), mph0) && clock64() - t0 < kWaitLimitCycles) {
+            }
+        if (pend1)
+            while (!mbar_try_wait(mma_bar(1), mph1) && clock64() - t0 < kWaitLimitCycles) {
+            }
         if (my_tiles > 0)
             while (!mbar_try_wait(gbar, 0) && clock64() - t0 < kWaitLimitCycles) {
             }

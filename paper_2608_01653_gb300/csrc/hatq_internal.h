@@ -137,12 +137,12 @@ struct GdnArgs {
     long long pixels;
     int c, inverse, hb_next, t, shift_in;
     unsigned long long P;            // R^2 ~ P / 2^t
-    float r2f;                       // P / 2^t (estimate only)
+    float sr;                        // sqrt(P / 2^t) (estimate only)
     long long mult_in;               // M_in
     const int32_t *b_pool;           // [c] B_i
     int *err;
     int num_tiles, nz;               // 128-pixel tiles, z tile buffers (1 or 2)
-    int z_off, u_off, b_off, bar_off;  // shared-memory offsets from the 1024-aligned base
+    int z_off, u_off, b_off, lut_off, bar_off;  // shared-memory offsets from the 1024-aligned base
     int tmem_cols;
 };
 
