@@ -70,7 +70,7 @@ def parse():
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--workload", default="cfg4",
-                   choices=["cfg4", "cfg2", "cfg1", "fwht", "profile", "int8mm", "orders", "decoder", "affine"],
+                   choices=["cfg4", "cfg2", "cfg1", "fwht", "profile", "int8mm", "orders", "decoder", "affine", "gdn"],
                    help="fwht: the INT8 transform+requantize pass alone on the config-4 ga2 input; "
                         "profile: the range-expansion profiling pass on the same tensor; "
                         "int8mm: torch._int_mm 8192^3, the library INT8 GEMM as a reference point; "
@@ -400,6 +400,46 @@ def run_decoder_mode(args):
         "peak_bf16_burst": tc}), flush=True)
 
 
+def run_gdn_mode(args):
+    """A GDN analysis layer at the config-4 ga2 output size (batch 8): ga2
+    (5x5 s2, 192 -> 192, DH 64) emitting the integer preactivation z, then
+    the GDN transition (pool on the tensor cores, phi_int, the next layer's
+    DH 64 input transition) on the 8 x 540 x 960 x 192 codes. Random INT8
+    operands, seeded beta / gamma of GDN's usual shape (beta ~ 1, small
+    non-negative gamma), CUDA events."""
+    import torch
+    from paper_2608_01653_gb300 import hatq as H
+    H.load()
+    peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
+    tc, hbm = peaks.get("bf16_tflops", FALLBACK_BF16_TFLOPS), peaks.get("hbm_gbs", FALLBACK_HBM_GBS)
+    n, h, w, c = 8, 1080, 1920, 192
+    g = torch.Generator(device="cuda")
+    g.manual_seed(19)
+    rng = np.random.default_rng(19)
+    beta, gamma = 0.5 + rng.random(c), np.abs(rng.standard_normal((c, c))) * 0.01
+    L = C.layer("ga2", 192, 192, 5, 2, 2, "DH", "none", hb_in=64)
+    P = H.prepare_weights(H.desc_from_spec(L), I.weights(192, 5, 5, 192, 2001), I.bias(192, 2051), 0.1, 0.05, "none", 0)
+    G = H.prepare_gdn(c, beta, gamma, 0.05, 0.02, False, 0.05, 64)
+    x = torch.randint(-127, 128, (n, h, w, c), dtype=torch.int8, device="cuda", generator=g)
+    z = torch.empty(P.out_shape(n, h, w), dtype=torch.int8, device="cuda")
+    y = torch.empty_like(z)
+    c_ms = time_events(lambda: H.conv2d_i8(x, P, y=z), args.steps, args.warmup)
+    g_ms = time_events(lambda: H.gdn(z, G, y=y), args.steps, args.warmup)
+    H.sync_status()
+    pix = z.numel() // c
+    g_bytes = 2 * z.numel()                                   # z read, x written
+    g_flops = 2 * 2 * pix * c * c                             # two limbs of the pool contraction
+    c_flops = 2 * pix * c * 25 * c
+    print(json.dumps({
+        "mode": "gdn", "batch": n, "z_shape": list(z.shape),
+        "conv": {"layer": "ga2 192->192 5x5 s2 DH64, emits z", "ms": c_ms,
+                 "tflops": c_flops / (c_ms / 1000) / 1e12, "frac": c_flops / (tc * 1e12) * 1000 / c_ms},
+        "gdn": {"ms": g_ms, "Mpixel_per_s": pix / (g_ms / 1000) / 1e6,
+                "hbm_gbs": g_bytes / (g_ms / 1000) / 1e9, "hbm_frac": g_bytes / (g_ms / 1000) / 1e9 / hbm,
+                "pool_tflops": g_flops / (g_ms / 1000) / 1e12, "tensor_frac": g_flops / (g_ms / 1000) / 1e12 / tc},
+        "peak_bf16_burst": tc, "peak_hbm_gbs": hbm}), flush=True)
+
+
 def run_affine_mode(args):
     """ga2 (5x5 s2, 192 -> 192, DH 64) with dynamic affine activations at
     batch 8 on the 1080 x 1920 fp16 input: the range + quantize passes
@@ -474,7 +514,7 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     cfg, scales = workload_chains("cfg4" if args.workload in ("cfg4", "fwht", "profile", "int8mm", "orders", "decoder",
-                                                              "affine") else args.workload)
+                                                              "affine", "gdn") else args.workload)
     if args.impl == "reference":
         run_reference(args, cfg, scales)
         return
@@ -496,6 +536,9 @@ def main():
     if args.workload == "decoder":
         run_decoder_mode(args)
         return
+    if args.workload == "gdn":
+        run_gdn_mode(args)
+        return
     if args.workload == "affine":
         run_affine_mode(args)
         return
@@ -516,7 +559,8 @@ def main():
     for ch in cfg.chains:
         params = C.chain_params(ch)
         plan = C.plan_chain(ch)
-        chain = Chain(ch.layers, params, scales[ch.name], plan, ch.out_f32, device=dev)
+        chain = Chain(ch.layers, params, scales[ch.name], plan, ch.out_f32, device=dev,
+                      f16_operands=C.f16_operand_layers(ch))
         kind = H.IN_F16 if ch.input_kind == "f16" else H.IN_I8
         x_host = C.chain_input(ch.with_batch(ch.n, ch.h, ch.w, replica_seed(ch.input_seed, rank)))
         x_pin = torch.from_numpy(x_host).pin_memory()
@@ -637,7 +681,7 @@ def main():
     roofline_fwht = {"bound": "hbm", "achieved": f_bytes / (f_ms / 1000) / 1e9, "peak": hbm_peak, "unit": "GB/s",
                      "frac": f_bytes / (f_ms / 1000) / 1e9 / hbm_peak, "ms": f_ms, "bytes": f_bytes,
                      "shape": list(f_shape), "hb": 64, "peak_source": hbm_src,
-                     "kernel": "hatq act_quant_kernel (INT8 entry, int32 butterfly, 64-bit requantization)"}
+                     "kernel": "hatq act_quant_i8_swar_kernel (INT8 entry, two 16-bit lanes per word, 32-bit requantization)"}
 
     # --- end to end through the public API (Chain.forward) with pinned host buffers: every step copies its
     # inputs in and its chain outputs back. Two input and two output slots per chain; copies run on their own

@@ -118,7 +118,23 @@ typedef struct {
     int in_affine;        /* 1: prepared by hatq_prepare_weights_affine (centred int16 operand, float output) */
     long long mult_in;    /* M_in of Eq. supp_general_input_scale */
     int8_t lut[256];      /* phi_int of Eq. supp_general_activation at z = -127..127 (index z + 127) */
+    int in_f16;           /* 1: the INT8 operand arrives as IEEE fp16 values (exact), see hatq_set_operand_format */
+    int out_f16;          /* 1: the INT8 codes are written as IEEE fp16 values (exact) */
 } hatq_prepared;
+
+/*
+ * Storage format of a prepared layer's operand and output codes (the values
+ * are the same INT8 codes either way; the paper has no counterpart: this only
+ * changes how they sit in memory). in_f16: hatq_conv2d_i8 and hatq_layer
+ * (x_kind HATQ_IN_OPERAND) read x as fp16 [n][h][w][c_in]; the tensor cores
+ * then take the operand straight from the TMA tile in shared memory, with no
+ * conversion per output-channel tile. out_f16: the layer writes its codes as
+ * fp16 (twice the bytes), the operand format of a next layer with in_f16.
+ * Both default to 0. in_f16 needs c_in % 16 == 0 and an INT8 (not affine)
+ * layer; out_f16 needs INT8 output (not float32) and is not available to the
+ * sub-pixel entry point. Host only; HATQ_ERR_INVALID_ARG / HATQ_ERR_UNSUPPORTED.
+ */
+hatq_status hatq_set_operand_format(hatq_prepared *L, int in_f16, int out_f16);
 
 /*
  * Offline preparation of a layer followed by a non-homogeneous activation

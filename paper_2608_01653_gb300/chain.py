@@ -13,11 +13,14 @@ from . import hatq
 
 
 class Chain:
-    def __init__(self, layers, params, scales, plan, out_f32_last=False, device="cuda"):
+    def __init__(self, layers, params, scales, plan, out_f32_last=False, device="cuda", f16_operands=()):
         """layers: objects with c_in, c_out, k, stride, pad, form, hb_in, hb_out, act;
         params: [(w_ohwi float32, bias float32)]; scales: [{'s_x', 's_out'}, plus 's_z' and
         's_u' for a SiLU / GELU layer]; plan: per layer the block of the next layer's DH
-        transform fused in its epilogue (0 = none)."""
+        transform fused in its epilogue (0 = none); f16_operands: indices of layers
+        whose operand (emitted directly by the layer before) is stored as fp16 codes
+        (hatq_set_operand_format), so it is converted once by its producer instead
+        of once per output-channel tile by its consumer."""
         self.layers = list(layers)
         self.plan = list(plan)
         self.prepared = []
@@ -26,6 +29,11 @@ class Chain:
             self.prepared.append(hatq.prepare_weights(
                 hatq.desc_from_spec(L), w, b, sc["s_x"], sc["s_out"], L.act, self.plan[i],
                 out_f32_last and last, device=device, s_z=sc.get("s_z"), s_u=sc.get("s_u")))
+        for i in sorted(set(f16_operands)):
+            if not 0 < i < len(self.layers) or not (self.plan[i - 1] or self.layers[i].form == "WH"):
+                raise ValueError(f"layer {i} does not take its operand straight from the layer before")
+            hatq.set_operand_format(self.prepared[i], True, self.prepared[i].out_f16)
+            hatq.set_operand_format(self.prepared[i - 1], self.prepared[i - 1].in_f16, True)
 
     def input_kinds(self, x_kind, s_in):
         """(kind, scale) of each layer's input, mirroring what each epilogue emits."""
@@ -54,7 +62,7 @@ class Chain:
         for P in self.prepared:
             scratch = max(scratch, n * hh * ww * P.c_in)
             s = P.out_shape(n, hh, ww)
-            outs.append(torch.empty(s, dtype=torch.float32 if P.out_f32 else torch.int8, device=device))
+            outs.append(torch.empty(s, dtype=getattr(torch, P.out_dtype), device=device))
             hh, ww = s[1], s[2]
         return outs, torch.empty(max(scratch, 16), dtype=torch.int8, device=device)
 

@@ -649,6 +649,8 @@ hatq_status upload_layer(const hatq_conv_desc &dop, const Geometry &g, const Hos
     out->s_u = gen ? gen->s_u : 0.f;
     out->shift_in = gen ? gen->shift_in : 0;
     out->in_affine = 0;
+    out->in_f16 = 0;
+    out->out_f16 = 0;
     out->mult_in = gen ? gen->mult_in : 0;
     if (gen) std::memcpy(out->lut, gen->lut, sizeof out->lut);
     else std::memset(out->lut, 0, sizeof out->lut);
@@ -891,9 +893,14 @@ hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared 
     a.gather = g.gather;
     // exact fp32 chunks: 1024 products of |x| <= 127 (INT8 codes), 512 of |x| <= 255 (centred affine codes)
     a.affine = L->in_affine ? 1 : 0;
+    a.a_f16 = L->in_f16 ? 1 : 0;
+    a.out_f16 = L->out_f16 ? 1 : 0;
+    if (a.a_f16 && (g.gather || a.affine)) return fail(HATQ_ERR_UNSUPPORTED, "an fp16 operand needs c_in % 16 == 0 and INT8 codes");
+    if (a.out_f16 && (L->out_f32 || (og && og->d2s)))
+        return fail(HATQ_ERR_UNSUPPORTED, "fp16 code output needs INT8 output without the sub-pixel rearrangement");
     a.chunk_kb = a.affine ? 8 : 16;
     a.b_bytes = a.n_t * 128;
-    a.raw_bytes = g.gather ? 0 : (a.affine ? 16384 : 8192);
+    a.raw_bytes = g.gather ? 0 : ((a.affine || a.a_f16) ? 16384 : 8192);
     a.n_tiles_n = d->c_out / a.n_t;
     {
         const long long nt = (long long)n * a.tiles_w * a.tiles_h * a.n_tiles_n;
@@ -984,16 +991,18 @@ hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared 
     if (!g.gather) {
         EncodeTiledFn enc = encode_fn();
         if (!enc) return fail(HATQ_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
-        // INT8 codes (64-byte box rows, 64-byte swizzle) or centred int16 affine codes (128-byte rows)
-        const cuuint64_t es = a.affine ? 2 : 1;
+        // INT8 codes (64-byte box rows, 64-byte swizzle), or centred int16 affine codes / fp16
+        // operand codes (128-byte rows, 128-byte swizzle)
+        const bool wide = a.affine || a.a_f16;
+        const cuuint64_t es = wide ? 2 : 1;
         const cuuint64_t dims[4] = {(cuuint64_t)d->c_in, (cuuint64_t)w, (cuuint64_t)h, (cuuint64_t)n};
         const cuuint64_t strides[3] = {(cuuint64_t)d->c_in * es, (cuuint64_t)w * d->c_in * es,
                                        (cuuint64_t)h * w * d->c_in * es};
         const cuuint32_t box[4] = {64, (cuuint32_t)(a.tw * d->stride), (cuuint32_t)(a.th * d->stride), 1};
         const cuuint32_t estr[4] = {1, (cuuint32_t)d->stride, (cuuint32_t)d->stride, 1};
-        CUresult r = enc(&tmA, a.affine ? CU_TENSOR_MAP_DATA_TYPE_UINT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 4,
+        CUresult r = enc(&tmA, wide ? CU_TENSOR_MAP_DATA_TYPE_UINT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 4,
                          const_cast<void *>(x), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                         a.affine ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+                         wide ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
                          CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "activation tensor map encoding failed (%d)", (int)r);
     } else if (a.win_tma) {
@@ -1299,6 +1308,7 @@ hatq_status hatq_conv_transpose2d_i8(const int8_t *x, int n, int h, int w, const
 int hatq_layer_launches(int x_kind, float s_in, const hatq_prepared *L) {
     if (!L) return -1;
     if (x_kind == HATQ_IN_OPERAND) return 1;
+    if (L->in_f16) return -1;
     if (L->d.form == HATQ_TRANSFORM) return x_kind == HATQ_IN_I8 ? 1 : -1;
     if (L->d.form == HATQ_DH && !pow2(L->d.hb_in)) return -1;   // paper order: operand from the transform layer
     if (x_kind == HATQ_IN_I8) return (L->d.form == HATQ_WH && s_in == L->s_x) ? 1 : 2;
@@ -1312,6 +1322,8 @@ hatq_status hatq_layer(const void *x, int x_kind, float s_in, int n, int h, int 
     if (n == 0 && h >= 1 && w >= 1) return HATQ_OK;                    // empty batch: nothing to do
     if (!x || !y) return fail(HATQ_ERR_INVALID_ARG, "null argument");
     const hatq_conv_desc *d = &L->d;
+    if (L->in_f16 && x_kind != HATQ_IN_OPERAND)
+        return fail(HATQ_ERR_UNSUPPORTED, "a layer with an fp16 operand takes it as HATQ_IN_OPERAND");
     if (x_kind == HATQ_IN_OPERAND || (x_kind == HATQ_IN_I8 && d->form == HATQ_WH && s_in == L->s_x) ||
         (x_kind == HATQ_IN_I8 && d->form == HATQ_TRANSFORM))
         return hatq_conv2d_i8(static_cast<const int8_t *>(x), n, h, w, L, y, stream);
@@ -1488,6 +1500,18 @@ hatq_status hatq_gdn(const int8_t *z, int n, int h, int w, const hatq_prepared_g
     if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "preactivation tensor map encoding failed (%d)", (int)r);
     if ((e = hatq::launch_gdn(tmZ, tmG, a, smem, reinterpret_cast<cudaStream_t>(stream))) != cudaSuccess)
         return cuda_fail(e, "GDN launch");
+    return HATQ_OK;
+}
+
+hatq_status hatq_set_operand_format(hatq_prepared *L, int in_f16, int out_f16) {
+    if (!L) return fail(HATQ_ERR_INVALID_ARG, "null layer");
+    if ((in_f16 != 0 && in_f16 != 1) || (out_f16 != 0 && out_f16 != 1))
+        return fail(HATQ_ERR_INVALID_ARG, "in_f16 and out_f16 must be 0 or 1");
+    if (in_f16 && (L->gather || L->in_affine || L->d.form == HATQ_TRANSFORM))
+        return fail(HATQ_ERR_UNSUPPORTED, "an fp16 operand needs an INT8 convolution with c_in %% 16 == 0");
+    if (out_f16 && L->out_f32) return fail(HATQ_ERR_UNSUPPORTED, "fp16 code output needs INT8 output");
+    L->in_f16 = in_f16;
+    L->out_f16 = out_f16;
     return HATQ_OK;
 }
 

@@ -553,7 +553,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t idesc = idesc_f16(a.n_t);
             // weight descriptor of stage 0, block 0; a stage / block moves its start address field
             const uint64_t desc0 = sdesc_sw128(smem_addr(smem) + (uint32_t)a.b_off);
+            // fp16 operand codes: the A tile of the stage (128 rows of 128 bytes per block, 128-byte swizzle)
+            const uint64_t adesc0 = sdesc_sw128(smem_addr(smem) + (uint32_t)a.raw_off);
             const uint32_t stage_step = (uint32_t)a.stage_bytes >> 4, blk_step = (uint32_t)a.b_bytes >> 4;
+            const uint32_t raw_step = (uint32_t)a.raw_bytes >> 4;
             bool ok = true;
             int s = 0, slot = 0;
             uint32_t ph = 0;
@@ -578,14 +581,18 @@ __global__ void __launch_bounds__(kThreads, 1)
                     tc_fence_after();
                     const uint64_t db0 = desc0 + (uint64_t)((uint32_t)s * stage_step);
                     const uint32_t a_t = tmem + (uint32_t)(a.a_col + slot * SUB * 32);
+                    const uint64_t da0 = adesc0 + (uint64_t)((uint32_t)s * stage_step);
 #pragma unroll
                     for (int u = 0; u < SUB; ++u) {
                         if (u >= nsub) break;
                         const uint64_t db = db0 + (uint64_t)((uint32_t)u * blk_step);
+                        const uint64_t da = da0 + (uint64_t)((uint32_t)u * raw_step);
 #pragma unroll
-                        for (int kk = 0; kk < kBlockK / 16; ++kk)   // K = 16 per instruction: 8 TMEM columns, 32 bytes of B
-                            umma_f16_ts(d_tmem, a_t + (uint32_t)(u * 32 + kk * 8), db + (uint64_t)(2 * kk), idesc,
-                                        (ck + u > 0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < kBlockK / 16; ++kk) {  // K = 16 per instruction: 8 TMEM columns, 32 bytes of B
+                            const uint32_t accu = (ck + u > 0 || kk > 0) ? 1u : 0u;
+                            if (a.a_f16) umma_f16_ss(d_tmem, da + (uint64_t)(2 * kk), db + (uint64_t)(2 * kk), idesc, accu);
+                            else umma_f16_ts(d_tmem, a_t + (uint32_t)(u * 32 + kk * 8), db + (uint64_t)(2 * kk), idesc, accu);
+                        }
                     }
                     umma_commit(empty_bar(s));
                     umma_commit(a_free(slot));
@@ -658,7 +665,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     i8x4_to_f16x4(v[q].w, h[8 * q + 6], h[8 * q + 7]);
                 }
             };
-            const int row_in = a.affine ? 128 : 64;     // bytes of one operand row of a 64-wide block
+            const int row_in = (a.affine || a.a_f16) ? 128 : 64;   // bytes of one operand row of a 64-wide block
             for (int j = 0; j < my_tiles && ok; ++j) {
                 for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB) {
                     const int nsub = min(SUB, a.num_kb - kb0);
@@ -666,6 +673,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!ok) break;
                     const uint8_t *raw = smem + (size_t)s * a.stage_bytes + a.raw_off + m * row_in;
                     const uint32_t t_slot = t_lane + (uint32_t)(slot * SUB * 32);
+                    if (a.a_f16) {
+                        // the MMAs read the fp16 tile itself; only the hand-off remains
+                        ok = slot_free();
+                        if (!ok) break;
+                        tc_fence_before();
+                        mbar_arrive(conv_bar(s));
+                        advance();
+                        continue;
+                    }
                     uint32_t h[32];
                     convert_row(raw, h);              // the first block is converted before the slot frees up
                     ok = slot_free();
@@ -893,7 +909,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                         if (!a.d2s) {
                             const long long pix = ((long long)img * a.y_h + gy) * a.y_w + gx;
                             const int4 v = *reinterpret_cast<const int4 *>(src + c * 16);
-                            *reinterpret_cast<int4 *>(static_cast<uint8_t *>(a.y) + pix * a.co + n0 + c * 16) = v;
+                            if (a.out_f16) {
+                                // the same codes as fp16 (exact): 16 codes -> 32 bytes
+                                uint32_t hh[8];
+                                i8x4_to_f16x4((uint32_t)v.x, hh[0], hh[1]);
+                                i8x4_to_f16x4((uint32_t)v.y, hh[2], hh[3]);
+                                i8x4_to_f16x4((uint32_t)v.z, hh[4], hh[5]);
+                                i8x4_to_f16x4((uint32_t)v.w, hh[6], hh[7]);
+                                int4 *dst = reinterpret_cast<int4 *>(static_cast<uint16_t *>(a.y) + pix * a.co + n0 + c * 16);
+                                dst[0] = make_int4((int)hh[0], (int)hh[1], (int)hh[2], (int)hh[3]);
+                                dst[1] = make_int4((int)hh[4], (int)hh[5], (int)hh[6], (int)hh[7]);
+                            } else {
+                                *reinterpret_cast<int4 *>(static_cast<uint8_t *>(a.y) + pix * a.co + n0 + c * 16) = v;
+                            }
                         } else {
                             // sub-pixel rearrangement: channel cd r^2 + i r + j of pixel (gy, gx) goes to
                             // channel cd of pixel (gy r + i, gx r + j); chunk c holds 16 destination channels

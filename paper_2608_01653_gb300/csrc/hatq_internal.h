@@ -122,6 +122,8 @@ struct ConvArgs {
     const float *affine_s;
     const float *s_w;
     int general, shift_in;
+    int a_f16;                       // operand codes as fp16 in the TMA tile: the MMA reads A from shared memory
+    int out_f16;                     // codes written as fp16
     int lut_off;                     // offset of the table copy from the barrier area
     long long mult_in;
     int8_t lut[256];

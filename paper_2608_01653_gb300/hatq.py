@@ -45,7 +45,8 @@ class PreparedStruct(ctypes.Structure):
                 ("mult", ctypes.c_void_p), ("deq", ctypes.c_void_p), ("s_w", ctypes.c_void_p),
                 ("opaque", ctypes.c_uint64 * 16),
                 ("s_z", ctypes.c_float), ("s_u", ctypes.c_float), ("shift_in", ctypes.c_int),
-                ("in_affine", ctypes.c_int), ("mult_in", ctypes.c_longlong), ("lut", ctypes.c_int8 * 256)]
+                ("in_affine", ctypes.c_int), ("mult_in", ctypes.c_longlong), ("lut", ctypes.c_int8 * 256),
+                ("in_f16", ctypes.c_int), ("out_f16", ctypes.c_int)]
 
 
 MAX_TRANSPOSED_CLASSES = 4
@@ -122,6 +123,7 @@ def load(build: bool = True) -> ctypes.CDLL:
                                            ctypes.POINTER(ctypes.c_longlong), ctypes.POINTER(_I)]),
             "hatq_prepare_gdn": (_I, [_I, _P, _P, _F, _F, _I, _F, _I, ctypes.POINTER(PreparedGdnStruct), _P]),
             "hatq_gdn": (_I, [_P, _I, _I, _I, ctypes.POINTER(PreparedGdnStruct), _P, _P]),
+            "hatq_set_operand_format": (_I, [ctypes.POINTER(PreparedStruct), _I, _I]),
             "hatq_version": (_I, []),
         }
         for name, (res, args) in sig.items():
@@ -250,6 +252,19 @@ class PreparedLayer:
     @property
     def s_x(self):
         return float(self.struct.s_x)
+
+    @property
+    def in_f16(self):
+        return bool(self.struct.in_f16)
+
+    @property
+    def out_f16(self):
+        return bool(self.struct.out_f16)
+
+    @property
+    def out_dtype(self):
+        """torch dtype name of the layer's output tensor."""
+        return "float32" if self.out_f32 else ("float16" if self.out_f16 else "int8")
 
     @property
     def s_y(self):
@@ -612,9 +627,10 @@ def _check_layer_io(x, x_kind, L, y=None, scratch=None):
     n, h, w, c = x.shape
     if c != L.c_in:
         raise ValueError(f"x has {c} channels, the layer takes {L.c_in}")
-    _check_tensor(x, "x", _KIND_DTYPE[x_kind])
+    f16_op = x_kind == IN_OPERAND and getattr(L, "in_f16", False)
+    _check_tensor(x, "x", "float16" if f16_op else _KIND_DTYPE[x_kind])
     if y is not None:
-        _check_tensor(y, "y", "float32" if L.out_f32 else "int8", L.out_shape(n, h, w))
+        _check_tensor(y, "y", getattr(L, "out_dtype", "float32" if L.out_f32 else "int8"), L.out_shape(n, h, w))
     if scratch is not None:
         _check_tensor(scratch, "scratch", "int8")
     _check_cuda(("x", x), ("y", y), ("scratch", scratch))
@@ -644,12 +660,20 @@ def quantize_act(x, x_kind, s_in, hb, s_out, y=None, s_used=None, workspace=None
     return (y, s_used) if s_out <= 0 else y
 
 
+def set_operand_format(L: PreparedLayer, in_f16: bool, out_f16: bool):
+    """hatq_set_operand_format: the layer's operand (in_f16) and / or its
+    output codes (out_f16) stored as fp16 values instead of int8."""
+    _check(load().hatq_set_operand_format(ctypes.byref(L.struct), int(bool(in_f16)), int(bool(out_f16))))
+    return L
+
+
 def conv2d_i8(x, L: PreparedLayer, y=None, stream=None):
-    """hatq_conv2d_i8: convolution + fused requantize epilogue on the INT8 operand x (NHWC)."""
+    """hatq_conv2d_i8: convolution + fused requantize epilogue on the INT8 operand x (NHWC; fp16 codes
+    for a layer with in_f16)."""
     n, h, w, c = _check_layer_io(x, IN_OPERAND, L, y)
     torch = _torch()
     if y is None:
-        y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32 if L.out_f32 else torch.int8, device=x.device)
+        y = torch.empty(L.out_shape(n, h, w), dtype=getattr(torch, L.out_dtype), device=x.device)
     _check(load().hatq_conv2d_i8(_ptr(x), n, h, w, ctypes.byref(L.struct), _ptr(y), _stream(stream)))
     return y
 
@@ -659,7 +683,7 @@ def layer(x, x_kind, s_in, L: PreparedLayer, y=None, scratch=None, stream=None):
     n, h, w, c = _check_layer_io(x, x_kind, L, y, scratch)
     torch = _torch()
     if y is None:
-        y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32 if L.out_f32 else torch.int8, device=x.device)
+        y = torch.empty(L.out_shape(n, h, w), dtype=getattr(torch, L.out_dtype), device=x.device)
     nbytes = 0
     if layer_launches(x_kind, s_in, L) > 1:
         if scratch is None:
@@ -721,7 +745,7 @@ def layer_noalloc(x, x_kind, s_in, L: PreparedLayer, y=None, stream=None):
     n, h, w, c = _check_layer_io(x, x_kind, L, y)
     torch = _torch()
     if y is None:
-        y = torch.empty(L.out_shape(n, h, w), dtype=torch.float32 if L.out_f32 else torch.int8, device=x.device)
+        y = torch.empty(L.out_shape(n, h, w), dtype=getattr(torch, L.out_dtype), device=x.device)
     _check(load().hatq_layer_noalloc(_ptr(x), int(x_kind), float(s_in), n, h, w, ctypes.byref(L.struct), _ptr(y),
                                      _stream(stream)))
     return y

@@ -45,7 +45,8 @@ def run():
     out = []
     for ch in C.CONFIGS["cfg4"].chains:
         params = C.chain_params(ch)
-        chain = Chain(ch.layers, params, _scales(ch), C.plan_chain(ch), ch.out_f32)
+        chain = Chain(ch.layers, params, _scales(ch), C.plan_chain(ch), ch.out_f32,
+                      f16_operands=C.f16_operand_layers(ch))
         x = C.chain_input(ch)
         outs = chain.forward(torch.from_numpy(x).cuda(), H.IN_I8, ch.s_in)
         out.append((ch, params, x, outs))
@@ -92,6 +93,8 @@ def _check_chain(ch, params, x, outs):
         acc = O.conv_codes_at(cur, p.w_int, p.stride, p.pad, pix)
         ref = O.epilogue_int(acc, p)
         got = y.cpu().numpy()
+        if got.dtype == np.float16:                       # codes stored as fp16 for an fp16-operand layer
+            got = got.astype(np.int8)
         sel = got[pix[:, 0], pix[:, 1], pix[:, 2], :]
         bad = np.argwhere(sel != ref)
         assert bad.size == 0, (f"{ch.name}/{L.name}: {len(bad)} of {ref.size} sampled codes differ, first at pixel "
@@ -119,4 +122,5 @@ def test_cfg4_analysis_image0_end_to_end(run):
     preps = O.prepare_chain(ch.layers, params, _scales(ch), ch.out_f32)
     refs = O.chain_forward(ch.layers, preps, x[:1], ch.input_kind, ch.s_in)
     for i, (g, r) in enumerate(zip(outs, refs)):
-        assert np.array_equal(g[:1].cpu().numpy(), r), f"layer {ch.layers[i].name} differs on image 0"
+        assert np.array_equal(g[:1].cpu().numpy().astype(np.int64), r.astype(np.int64)), \
+            f"layer {ch.layers[i].name} differs on image 0"
