@@ -465,3 +465,26 @@ def test_prepare_gdn_rejects_on_the_host(lib):
     with pytest.raises(ValueError):
         H.prepare_gdn_host(64, beta[:10], gamma, 0.1, 0.1, False, 0.1)
     assert lib.hatq_gdn(None, 1, 1, 1, None, None, None) == H.ERR_INVALID_ARG
+
+
+def test_set_operand_format_checks_on_the_host(lib):
+    """hatq_set_operand_format is host-only: it validates the layer kind and
+    writes the two flags (no device buffers are touched)."""
+    P = H.PreparedStruct()
+    P.d = H.make_desc(192, 192, 3, 1, 1, "DH", hb_in=64)
+    assert lib.hatq_set_operand_format(ctypes.byref(P), 1, 1) == H.OK and (P.in_f16, P.out_f16) == (1, 1)
+    assert lib.hatq_set_operand_format(ctypes.byref(P), 0, 0) == H.OK and (P.in_f16, P.out_f16) == (0, 0)
+    assert lib.hatq_set_operand_format(ctypes.byref(P), 2, 0) == H.ERR_INVALID_ARG
+    P.gather = 1
+    assert lib.hatq_set_operand_format(ctypes.byref(P), 1, 0) == H.ERR_UNSUPPORTED
+    P.gather, P.in_affine = 0, 1
+    assert lib.hatq_set_operand_format(ctypes.byref(P), 1, 0) == H.ERR_UNSUPPORTED
+    P.in_affine, P.out_f32 = 0, 1
+    assert lib.hatq_set_operand_format(ctypes.byref(P), 0, 1) == H.ERR_UNSUPPORTED
+    assert lib.hatq_set_operand_format(None, 0, 0) == H.ERR_INVALID_ARG
+
+
+def test_f16_operand_policy_picks_narrow_fed_layers():
+    for ch in C.CONFIGS["cfg4"].chains:
+        got = C.f16_operand_layers(ch)
+        assert got == ((1, 2) if ch.name.startswith("slice") else ())
