@@ -559,8 +559,7 @@ def main():
     for ch in cfg.chains:
         params = C.chain_params(ch)
         plan = C.plan_chain(ch)
-        chain = Chain(ch.layers, params, scales[ch.name], plan, ch.out_f32, device=dev,
-                      f16_operands=C.f16_operand_layers(ch))
+        chain = Chain(ch.layers, params, scales[ch.name], plan, ch.out_f32, device=dev)
         kind = H.IN_F16 if ch.input_kind == "f16" else H.IN_I8
         x_host = C.chain_input(ch.with_batch(ch.n, ch.h, ch.w, replica_seed(ch.input_seed, rank)))
         x_pin = torch.from_numpy(x_host).pin_memory()

@@ -557,6 +557,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint64_t adesc0 = sdesc_sw128(smem_addr(smem) + (uint32_t)a.raw_off);
             const uint32_t stage_step = (uint32_t)a.stage_bytes >> 4, blk_step = (uint32_t)a.b_bytes >> 4;
             const uint32_t raw_step = (uint32_t)a.raw_bytes >> 4;
+            const bool a_f16 = a.a_f16 != 0;
             bool ok = true;
             int s = 0, slot = 0;
             uint32_t ph = 0;
@@ -580,18 +581,28 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (!mbar_wait(conv_bar(s), ph, abort_flag, a.err)) { ok = false; break; }
                     tc_fence_after();
                     const uint64_t db0 = desc0 + (uint64_t)((uint32_t)s * stage_step);
-                    const uint32_t a_t = tmem + (uint32_t)(a.a_col + slot * SUB * 32);
-                    const uint64_t da0 = adesc0 + (uint64_t)((uint32_t)s * stage_step);
+                    if (!a_f16) {
+                        const uint32_t a_t = tmem + (uint32_t)(a.a_col + slot * SUB * 32);
 #pragma unroll
-                    for (int u = 0; u < SUB; ++u) {
-                        if (u >= nsub) break;
-                        const uint64_t db = db0 + (uint64_t)((uint32_t)u * blk_step);
-                        const uint64_t da = da0 + (uint64_t)((uint32_t)u * raw_step);
+                        for (int u = 0; u < SUB; ++u) {
+                            if (u >= nsub) break;
+                            const uint64_t db = db0 + (uint64_t)((uint32_t)u * blk_step);
 #pragma unroll
-                        for (int kk = 0; kk < kBlockK / 16; ++kk) {  // K = 16 per instruction: 8 TMEM columns, 32 bytes of B
-                            const uint32_t accu = (ck + u > 0 || kk > 0) ? 1u : 0u;
-                            if (a.a_f16) umma_f16_ss(d_tmem, da + (uint64_t)(2 * kk), db + (uint64_t)(2 * kk), idesc, accu);
-                            else umma_f16_ts(d_tmem, a_t + (uint32_t)(u * 32 + kk * 8), db + (uint64_t)(2 * kk), idesc, accu);
+                            for (int kk = 0; kk < kBlockK / 16; ++kk)   // K = 16 per instruction: 8 TMEM columns, 32 bytes of B
+                                umma_f16_ts(d_tmem, a_t + (uint32_t)(u * 32 + kk * 8), db + (uint64_t)(2 * kk), idesc,
+                                            (ck + u > 0 || kk > 0) ? 1u : 0u);
+                        }
+                    } else {
+                        const uint64_t da0 = adesc0 + (uint64_t)((uint32_t)s * stage_step);
+#pragma unroll
+                        for (int u = 0; u < SUB; ++u) {
+                            if (u >= nsub) break;
+                            const uint64_t db = db0 + (uint64_t)((uint32_t)u * blk_step);
+                            const uint64_t da = da0 + (uint64_t)((uint32_t)u * raw_step);
+#pragma unroll
+                            for (int kk = 0; kk < kBlockK / 16; ++kk)   // both operands in shared memory, 32 bytes each
+                                umma_f16_ss(d_tmem, da + (uint64_t)(2 * kk), db + (uint64_t)(2 * kk), idesc,
+                                            (ck + u > 0 || kk > 0) ? 1u : 0u);
                         }
                     }
                     umma_commit(empty_bar(s));

@@ -109,18 +109,6 @@ def plan_chain(chain: ChainSpec):
     return [L[i + 1].hb_in if i + 1 < len(L) and L[i + 1].form == DH else 0 for i in range(len(L))]
 
 
-def f16_operand_layers(chain: ChainSpec):
-    """Layers of a chain that take their operand as fp16 codes (storage only:
-    the codes are the same): those fed straight by the layer before (it
-    applies their DH transform, or they are WH) with at most 128 output
-    channels, where converting the INT8 operand for the tensor cores dominates
-    the layer; wider layers keep INT8 operands, which cost half the bytes."""
-    L = chain.layers
-    plan = plan_chain(chain)
-    return tuple(i for i in range(1, len(L))
-                 if (plan[i - 1] or L[i].form == WH) and L[i].c_out <= 128 and L[i].c_in % 16 == 0)
-
-
 def _cfg0():
     ch = ChainSpec(
         name="dh1x1_128", n=1, h=16, w=16, input_kind="f16", s_in=1.0,

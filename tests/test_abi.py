@@ -483,8 +483,3 @@ def test_set_operand_format_checks_on_the_host(lib):
     assert lib.hatq_set_operand_format(ctypes.byref(P), 0, 1) == H.ERR_UNSUPPORTED
     assert lib.hatq_set_operand_format(None, 0, 0) == H.ERR_INVALID_ARG
 
-
-def test_f16_operand_policy_picks_narrow_fed_layers():
-    for ch in C.CONFIGS["cfg4"].chains:
-        got = C.f16_operand_layers(ch)
-        assert got == ((1, 2) if ch.name.startswith("slice") else ())

@@ -45,8 +45,7 @@ def run():
     out = []
     for ch in C.CONFIGS["cfg4"].chains:
         params = C.chain_params(ch)
-        chain = Chain(ch.layers, params, _scales(ch), C.plan_chain(ch), ch.out_f32,
-                      f16_operands=C.f16_operand_layers(ch))
+        chain = Chain(ch.layers, params, _scales(ch), C.plan_chain(ch), ch.out_f32)
         x = C.chain_input(ch)
         outs = chain.forward(torch.from_numpy(x).cuda(), H.IN_I8, ch.s_in)
         out.append((ch, params, x, outs))
