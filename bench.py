@@ -295,6 +295,16 @@ def run_layer_mode(args, cfg, scales):
     raise SystemExit(f"unknown layer {args.layer}")
 
 
+def conv_source_sha() -> str:
+    """sha256 prefix of the conv kernel's sources (the kernel file and the
+    device-helper header it includes), the key of committed counter captures."""
+    import hashlib
+    h = hashlib.sha256()
+    for f in ("hatq_conv.cu", "hatq_tc.h"):
+        h.update(open(os.path.join(ROOT, "paper_2608_01653_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
 def fwht_pass(batch, steps, warmup, device="cuda"):
     """The INT8-entry transform + requantize pass (hb 64) on an NHWC tensor
     shaped like the config-4 ga2 input (8 x 1080 x 1920 x 192 at batch 8,
@@ -661,10 +671,8 @@ def main():
     prof = os.path.join(ROOT, "profiles", "conv_cfg4_traffic.json")
     if os.path.exists(prof):
         # the captured counters stand for the kernel source they were taken on, and for no later one
-        import hashlib
         rec = json.load(open(prof))
-        src = os.path.join(ROOT, "paper_2608_01653_gb300", "csrc", "hatq_conv.cu")
-        if hashlib.sha256(open(src, "rb").read()).hexdigest()[:16] == rec.get("kernel_source_sha256_16"):
+        if conv_source_sha() == rec.get("kernel_source_sha256_16"):
             traffic = rec.get("dram_bytes_per_launch")
     roofline_peaks = {"tensor_tflops": tc_peak, "hbm_gbs": hbm_peak, "int_tops": INT_OPS_PEAK / 1e12,
                       "int_source": "derived: 152 SMs x 4 sub-partitions x 32 lanes x 2.07 GHz (half-rate ALU + "
