@@ -34,9 +34,12 @@
 //   pool   each thread finishes 16 channels of its pixel per pass: the float
 //          estimate of the code, exact 64-bit comparisons near a rounding
 //          boundary, u into a shared-memory row;
-//   out    (pixel, 64-channel group) items over all threads: Sylvester block
-//          of u (int32, exact), then a table of clamp(round(M_in v / 2^n_in))
-//          over |v| <= 127 hb built once per CTA, 16-byte stores.
+//   out    after each pass, that pass's 64-channel group: four lanes per
+//          pixel row, 16 values each, Sylvester block of u (int32, exact;
+//          the two widest stages through lane shuffles), then a table of
+//          clamp(round(M_in v / 2^n_in)) over |v| <= 127 hb built once per
+//          CTA, 16-byte stores. The last group's transition runs next to the
+//          next tile's limbs, whose MMAs then start early.
 // Every wait is bounded; the CTA leaves its loop together after a failure.
 #include <cuda_fp16.h>
 
@@ -219,39 +222,112 @@ __global__ void __launch_bounds__(kGdnThreads, 1)
         if (b) pend1 = true;
         else pend0 = true;
     };
-    int j = 0;
-    for (; j < my_tiles && ok; ++j) {
-        const int b = j % a.nz;
-        const uint8_t *zt = z_s + (size_t)b * zbytes;
-        ok = __syncthreads_and(mbar_wait(zfull(b), (uint32_t)((j / a.nz) & 1), abort_flag, a.err));
-        if (!ok) break;
-        // ---- limbs of z^2 for this pixel row into TMEM: this quarter's K range, both limbs
-        {
-            const int sw = (m >> 1) & 3;
-            for (int k = part * (c / 4); k < (part + 1) * (c / 4); k += 16) {
-                const uint4 v = *reinterpret_cast<const uint4 *>(zt + (k >> 6) * 8192 + m * 64 +
-                                                                  ((((k & 63) >> 4) ^ sw) << 4));
-                const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-                uint32_t hh[8], ll[8];
+    // ---- limbs of z^2 of this pixel row into TMEM: this quarter's K range, both limbs
+    auto limbs = [&](const uint8_t *zt) {
+        const int sw = (m >> 1) & 3;
+        for (int k = part * (c / 4); k < (part + 1) * (c / 4); k += 16) {
+            const uint4 v = *reinterpret_cast<const uint4 *>(zt + (k >> 6) * 8192 + m * 64 +
+                                                              ((((k & 63) >> 4) ^ sw) << 4));
+            const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+            uint32_t hh[8], ll[8];
 #pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int z0 = (int)(int8_t)(w[i >> 1] >> (16 * (i & 1)));
-                    const int z1 = (int)(int8_t)(w[i >> 1] >> (16 * (i & 1) + 8));
-                    const uint32_t s0 = (uint32_t)(z0 * z0), s1 = (uint32_t)(z1 * z1);
-                    hh[i] = u10x2_to_f16x2(s0 >> 7, s1 >> 7);
-                    ll[i] = u10x2_to_f16x2(s0 & 127u, s1 & 127u);
-                }
-                tmem_st8(t_lane + (uint32_t)(k / 2), hh);
-                tmem_st8(t_lane + (uint32_t)(c / 2 + k / 2), ll);
+            for (int i = 0; i < 8; ++i) {
+                const int z0 = (int)(int8_t)(w[i >> 1] >> (16 * (i & 1)));
+                const int z1 = (int)(int8_t)(w[i >> 1] >> (16 * (i & 1) + 8));
+                const uint32_t s0 = (uint32_t)(z0 * z0), s1 = (uint32_t)(z1 * z1);
+                hh[i] = u10x2_to_f16x2(s0 >> 7, s1 >> 7);
+                ll[i] = u10x2_to_f16x2(s0 & 127u, s1 & 127u);
             }
-            tmem_wait_st();
+            tmem_st8(t_lane + (uint32_t)(k / 2), hh);
+            tmem_st8(t_lane + (uint32_t)(c / 2 + k / 2), ll);
         }
-        tc_fence_before();
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            issue_pass(0);
-            if (np > 1) issue_pass(1);
+        tmem_wait_st();
+    };
+    // ---- pool and codes u of channels 64 p + 16 part .. + 15 of this pixel (accumulator buffer db)
+    auto pool = [&](const uint8_t *zt, int p, int db) {
+        const int sw = (m >> 1) & 3;
+        const int col = 16 * part;                       // column within the pass
+        const int ch = 64 * p + col;
+        uint32_t dh[16], dl[16];
+        tmem_ld16(t_lane + (uint32_t)(c + 128 * db + col), dh);
+        tmem_ld16(t_lane + (uint32_t)(c + 128 * db + 64 + col), dl);
+        const uint4 zv = *reinterpret_cast<const uint4 *>(zt + (ch >> 6) * 8192 + m * 64 +
+                                                           ((((ch & 63) >> 4) ^ sw) << 4));
+        float bfv[16];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const float4 f4 = reinterpret_cast<const float4 *>(bf_s + ch)[q];
+            bfv[4 * q] = f4.x; bfv[4 * q + 1] = f4.y; bfv[4 * q + 2] = f4.z; bfv[4 * q + 3] = f4.w;
         }
+        tmem_wait_ld();
+        const uint32_t zw[4] = {zv.x, zv.y, zv.z, zv.w};
+        uint32_t out[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            int u[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int e = 4 * q + i;
+                const int zi = (int)(int8_t)(zw[q] >> (8 * i));
+                u[i] = gdn_code(zi, __uint_as_float(dh[e]), __uint_as_float(dl[e]), bfv[e], b_s + ch + e, a);
+            }
+            out[q] = prmt(prmt((uint32_t)u[0], (uint32_t)u[1], 0x0040u), prmt((uint32_t)u[2], (uint32_t)u[3], 0x0040u),
+                          0x5410u);
+        }
+        *reinterpret_cast<uint4 *>(u_s + m * ustride + ch) = make_uint4(out[0], out[1], out[2], out[3]);
+    };
+    // ---- input transition of the next layer on channel group p (64 channels) of
+    // tile jt: four consecutive lanes share a pixel row, 16 values each; block
+    // stages 1..8 in the lane, 16 and 32 across the four lanes; Sylvester block in
+    // int32 (exact: |H~ u| <= 127 hb), then the table of clamp(round(M_in v / 2^n_in))
+    auto transition = [&](int jt, int p) {
+        const int r = (int)threadIdx.x >> 2, sub = (int)threadIdx.x & 3;
+        const uint4 w = *reinterpret_cast<const uint4 *>(u_s + r * ustride + 64 * p + 16 * sub);
+        const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
+        int v[16];
+#pragma unroll
+        for (int i = 0; i < 16; ++i) v[i] = (int)(int8_t)(ww[i >> 2] >> (8 * (i & 3)));
+        const int hb = a.hb_next;
+        fwht<16>(v, hb < 16 ? hb : 16);
+        for (int mm = 1; mm <= 2; mm <<= 1) {
+            if (16 * mm >= hb) break;
+            const bool upper = (sub & mm) != 0;
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+                const int q = __shfl_xor_sync(0xffffffffu, v[i], mm);
+                v[i] = upper ? q - v[i] : v[i] + q;
+            }
+        }
+        const long long pix = (long long)((int)blockIdx.x + jt * (int)gridDim.x) * 128 + r;
+        if (pix < a.pixels) {
+            uint32_t wd[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                wd[q] = prmt(prmt((uint32_t)lut_s[v[4 * q]], (uint32_t)lut_s[v[4 * q + 1]], 0x0040u),
+                             prmt((uint32_t)lut_s[v[4 * q + 2]], (uint32_t)lut_s[v[4 * q + 3]], 0x0040u), 0x5410u);
+            *reinterpret_cast<uint4 *>(a.y + pix * c + 64 * p + 16 * sub) = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+        }
+    };
+
+    // Schedule per tile: [MMA wait, pool of pass p, barrier, MMAs of pass p + 2,
+    // transition of group p] for each pass, except that the last group's
+    // transition runs next to the limbs of the next tile, whose first MMAs then
+    // start while this tile's last writes drain.
+    int j = 0;
+    if (my_tiles > 0) {
+        ok = __syncthreads_and(mbar_wait(zfull(0), 0, abort_flag, a.err));
+        if (ok) {
+            limbs(z_s);
+            tc_fence_before();
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                issue_pass(0);
+                if (np > 1) issue_pass(1);
+            }
+        }
+    }
+    for (; j < my_tiles && ok; ++j) {
+        const uint8_t *zt = z_s + (size_t)(j % a.nz) * zbytes;
         for (int p = 0; p < np && ok; ++p) {
             const int db = p & 1;
             ok = __syncthreads_and(mbar_wait(mma_bar(db), db ? mph1 : mph0, abort_flag, a.err));
@@ -259,81 +335,32 @@ __global__ void __launch_bounds__(kGdnThreads, 1)
             else { mph0 ^= 1u; pend0 = false; }
             if (!ok) break;
             tc_fence_after();
-            // ---- pool and codes u of channels 64 p + 16 part .. + 15 of this pixel
-            {
-                const int sw = (m >> 1) & 3;
-                const int col = 16 * part;                   // column within the pass
-                const int ch = 64 * p + col;
-                uint32_t dh[16], dl[16];
-                tmem_ld16(t_lane + (uint32_t)(c + 128 * db + col), dh);
-                tmem_ld16(t_lane + (uint32_t)(c + 128 * db + 64 + col), dl);
-                const uint4 zv = *reinterpret_cast<const uint4 *>(zt + (ch >> 6) * 8192 + m * 64 +
-                                                                   ((((ch & 63) >> 4) ^ sw) << 4));
-                float bfv[16];
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const float4 f4 = reinterpret_cast<const float4 *>(bf_s + ch)[q];
-                    bfv[4 * q] = f4.x; bfv[4 * q + 1] = f4.y; bfv[4 * q + 2] = f4.z; bfv[4 * q + 3] = f4.w;
-                }
-                tmem_wait_ld();
-                const uint32_t zw[4] = {zv.x, zv.y, zv.z, zv.w};
-                uint32_t out[4];
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    int u[4];
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const int e = 4 * q + i;
-                        const int zi = (int)(int8_t)(zw[q] >> (8 * i));
-                        u[i] = gdn_code(zi, __uint_as_float(dh[e]), __uint_as_float(dl[e]), bfv[e], b_s + ch + e, a);
-                    }
-                    out[q] = prmt(prmt((uint32_t)u[0], (uint32_t)u[1], 0x0040u), prmt((uint32_t)u[2], (uint32_t)u[3], 0x0040u),
-                                  0x5410u);
-                }
-                *reinterpret_cast<uint4 *>(u_s + m * ustride + ch) = make_uint4(out[0], out[1], out[2], out[3]);
-            }
+            pool(zt, p, db);
             tc_fence_before();
-            __syncthreads();
+            __syncthreads();                               // codes of group p complete; buffer db free
             if (threadIdx.x == 0 && p + 2 < np) issue_pass(p + 2);
+            if (p + 1 < np) transition(j, p);
         }
         if (!ok) break;
-        // the z buffer is free: prefetch the tile that reuses it
+        // every pool of this tile is done: its z buffer takes the tile that reuses it
         if (threadIdx.x == 0 && issued < my_tiles) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             issue_z(issued);
             ++issued;
         }
-        // ---- input transition of the next layer: 64-channel groups of u,
-        // Sylvester block (int32, exact: |H~ u| <= 127 hb), then the table of
-        // clamp(round(M_in v / 2^n_in)); work items (row, group) over all threads
-        const long long pix0 = (long long)((int)blockIdx.x + j * (int)gridDim.x) * 128;
-        for (int it = threadIdx.x; it < 128 * (c / 64); it += kGdnThreads) {
-            const int row = it & 127, grp = it >> 7;
-            int v[64];
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const uint4 w = *reinterpret_cast<const uint4 *>(u_s + row * ustride + 64 * grp + 16 * q);
-                const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-                for (int i = 0; i < 16; ++i) v[16 * q + i] = (int)(int8_t)(ww[i >> 2] >> (8 * (i & 3)));
-            }
-            fwht<64>(v, a.hb_next);
-            if (pix0 + row < a.pixels) {
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    uint32_t wd[4];
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const int e = 16 * q + 4 * i;
-                        wd[i] = prmt(prmt((uint32_t)lut_s[v[e]], (uint32_t)lut_s[v[e + 1]], 0x0040u),
-                                     prmt((uint32_t)lut_s[v[e + 2]], (uint32_t)lut_s[v[e + 3]], 0x0040u), 0x5410u);
-                    }
-                    *reinterpret_cast<uint4 *>(a.y + (pix0 + row) * c + 64 * grp + 16 * q) =
-                        make_uint4(wd[0], wd[1], wd[2], wd[3]);
-                }
+        transition(j, np - 1);
+        if (j + 1 < my_tiles) {
+            const int b1 = (j + 1) % a.nz;
+            ok = __syncthreads_and(mbar_wait(zfull(b1), (uint32_t)(((j + 1) / a.nz) & 1), abort_flag, a.err));
+            if (!ok) break;
+            limbs(z_s + (size_t)b1 * zbytes);              // the A columns are free: pass np - 1 was waited for
+            tc_fence_before();
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                issue_pass(0);
+                if (np > 1) issue_pass(1);
             }
         }
-        __syncthreads();                                   // u rows are rewritten by the next tile
     }
     // after a failure: wait (bounded) for this CTA's copies and MMAs in flight
     if (!ok && threadIdx.x == 0) {
