@@ -512,8 +512,9 @@ hatq_status hatq_prepare_gdn(int c, const double *beta, const double *gamma, flo
                              float s_y, int hb_next, hatq_prepared_gdn *out, hatq_stream stream);
 
 /* The GDN / IGDN transition on device tensors: z [n][h][w][c] INT8
- * preactivation codes, y [n][h][w][c] the next layer's INT8 operand (both
- * 16-byte aligned, not overlapping). The pool runs on the tensor cores (the
+ * preactivation codes in [-127, 127] (Eq. supp_general_preactivation clamps
+ * to that range; -128 is outside the contract), y [n][h][w][c] the next
+ * layer's INT8 operand (both 16-byte aligned, not overlapping). The pool runs on the tensor cores (the
  * squared codes in two exact fp16 limbs times G, fp32 sums below 2^24).
  * Stream-ordered; device errors surface through hatq_sync_status(). */
 hatq_status hatq_gdn(const int8_t *z, int n, int h, int w, const hatq_prepared_gdn *g, int8_t *y, hatq_stream stream);
