@@ -54,9 +54,12 @@ Readings the paper leaves open (the same list is kept with the design notes):
      zero, decided exactly: the largest k with (2k - 1)^2 D_i 2^t <= 4 P z_i^2
      (GDN) or (2k - 1)^2 2^t <= 4 P z_i^2 D_i (IGDN); u_i takes the sign of z_i.
 
-parity unpinned: the rounding convention R2 and the (M, n) rule R3 are
-conventions of this implementation (the paper fixes neither); the oracle pins
-them against exact rational arithmetic, not against the paper.
+Pins (tests/test_oracle_pins.py) hold every function to something other
+than itself: closed forms, the paper's printed values, brute force and exact
+rational arithmetic. R2 and R3 are readings (the paper fixes no rounding
+convention and no rule for n); what they define is pinned against exact
+rationals: the shift equals the exact rational v / 2^n rounded half to even,
+and (M, n) is the largest admissible n with |M - rho 2^n| <= 1/2.
 """
 from __future__ import annotations
 
