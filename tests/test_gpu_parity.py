@@ -65,11 +65,12 @@ def test_quantize_i8_static_bit_exact(H, shape, hb):
 
 # (shape, hb, s_in, rho = s_in / (sqrt(hb) s_x)): rho <= 1 takes the packed
 # 16-bit-pair kernel; rho = 1/4 at hb = 64 gives M = 2^(n-2), where rounding
-# ties occur; rho = 1 gives M = 2^n; odd totals leave a lane half-empty.
+# ties occur; rho = 1 gives M = 2^n; odd totals leave a lane half-empty;
+# 4096 codes are exactly one warp tile, 4160 one tile and a 64-code tail.
 PACKED = [((2, 37, 41, 192), 64, 0.05, 0.3), ((1, 4, 6, 64), 64, 0.5, 0.25), ((1, 5, 5, 64), 64, 0.5, 1.0),
           ((1, 1, 3, 48), 16, 0.05, 0.7), ((1, 1, 5, 16), 16, 0.05, 0.9), ((1, 3, 7, 96), 32, 0.05, 0.05),
           ((1, 2, 9, 48), 1, 0.05, 0.9), ((1, 6, 7, 64), 2, 0.05, 0.5), ((3, 3, 5, 32), 8, 0.05, 0.4),
-          ((1, 7, 3, 128), 4, 0.05, 0.6)]
+          ((1, 7, 3, 128), 4, 0.05, 0.6), ((1, 8, 8, 64), 64, 0.05, 0.3), ((1, 1, 65, 64), 64, 0.05, 0.3)]
 
 
 @pytest.mark.parametrize("shape,hb,s_in,rho", PACKED)
