@@ -323,14 +323,37 @@ def fwht_pass(batch, steps, warmup, device="cuda"):
 
 
 def run_fwht_mode(args):
+    """The transform + quantize pass (hb 64) on the ga2-shaped tensor in its
+    three modes: INT8 entry with a static scale (the benchmark's pass), INT8
+    entry with the dynamic per-tensor scale (max-abs pass, parameter kernel,
+    quantize pass: 3 B/element read + written), FP16 entry with a static scale
+    (fp16 read, codes written: 3 B/element)."""
+    import torch
     from paper_2608_01653_gb300 import hatq as H
     H.load()
     ms, nbytes, shape = fwht_pass(args.batch, args.steps, args.warmup)
     peaks = json.load(open(PEAKS)) if os.path.exists(PEAKS) else {}
     peak = peaks.get("hbm_gbs", FALLBACK_HBM_GBS)
     gbs = nbytes / (ms / 1000) / 1e9
+    g = torch.Generator(device="cuda")
+    g.manual_seed(10)
+    x = torch.randint(-127, 128, shape, dtype=torch.int8, device="cuda", generator=g)
+    y = torch.empty_like(x)
+    s_used = torch.empty(1, dtype=torch.float32, device="cuda")
+    ws = torch.empty(64, dtype=torch.uint8, device="cuda")
+    d_ms = time_events(lambda: H.quantize_act(x, H.IN_I8, 0.05, 64, 0.0, y=y, s_used=s_used, workspace=ws),
+                       args.steps, args.warmup)
+    del x
+    xf = torch.randn(shape, device="cuda", generator=g).to(torch.float16)
+    f_ms = time_events(lambda: H.quantize_act(xf, H.IN_F16, 1.0, 64, 0.05, y=y), args.steps, args.warmup)
+    H.sync_status()
+    n = y.numel()
     print(json.dumps({"mode": "fwht", "shape": list(shape), "hb": 64, "ms": ms, "GB/s": gbs, "peak_hbm_gbs": peak,
-                      "frac": gbs / peak}), flush=True)
+                      "frac": gbs / peak,
+                      "i8_dynamic": {"ms": d_ms, "GB/s": 3 * n / (d_ms / 1000) / 1e9,
+                                     "frac": 3 * n / (d_ms / 1000) / 1e9 / peak},
+                      "f16_static": {"ms": f_ms, "GB/s": 3 * n / (f_ms / 1000) / 1e9,
+                                     "frac": 3 * n / (f_ms / 1000) / 1e9 / peak}}), flush=True)
 
 
 def run_orders_mode(args, cfg, scales):

@@ -131,6 +131,7 @@ __global__ void __launch_bounds__(kThreads) act_quant_kernel(ActQuantArgs a) {
     long long mult = a.mult;
     int shift = a.shift;
     float inv = a.inv;
+    if (MODE == 1 && !F16 && a.dyn->packed) return;   // the packed-pair pass quantizes this tensor
     if (MODE == 1) {
         mult = a.dyn->mult;
         shift = a.dyn->shift;
@@ -455,11 +456,32 @@ __device__ __forceinline__ uint32_t smem_addr(const void *p) {
 }
 __device__ __forceinline__ int swz(int row, int chunk) { return row * 128 + ((chunk ^ (row & 7)) << 4); }
 
-template <int HB, bool TIES>
+__device__ __forceinline__ uint32_t min_s16x2(uint32_t a, uint32_t b) {
+    uint32_t d;
+    asm("min.s16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+
+// MODE 0: static scale, constants sp from the host. MODE 1: dynamic scale,
+// constants from the parameter block (the kernel returns at once when the
+// block says the packed pass does not apply; the general kernel then runs).
+// MODE 2: the max-abs pass of the dynamic mode (max and min of the pairs, no
+// stores).
+template <int HB, bool TIES, int MODE>
 __global__ void __launch_bounds__(kSwarWarps * 32) act_quant_i8_swar_kernel(ActQuantArgs a, SwarParams sp) {
     constexpr uint32_t kBlo = HB >= 2 ? 128u * HB : 0u;
     constexpr uint32_t kBias2 = 256u * 65537u;      // the two halves' input bias after one stage
     __shared__ __align__(128) uint8_t stage[kSwarWarps][kSwarStages][4096];
+    if constexpr (MODE == 1) {
+        const DynParams *dp = a.dyn;
+        if (!dp->packed) return;
+        sp.clo = dp->clo;
+        sp.clow = dp->clow;
+        sp.chigh = dp->chigh;
+        sp.mult = (uint32_t)dp->mult;
+        sp.shift = dp->shift;
+    }
+    uint32_t vmx = 0x80008000u, vmn = 0x7FFF7FFFu;  // running max / min of the (biased) pairs
     const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
     const long long warp = (long long)blockIdx.x * kSwarWarps + wib;
     const long long nwarps = (long long)gridDim.x * kSwarWarps;
@@ -528,6 +550,14 @@ __global__ void __launch_bounds__(kSwarWarps * 32) act_quant_i8_swar_kernel(ActQ
                 }
             }
         }
+        if constexpr (MODE == 2) {
+            // zero-filled codes past the end transform to zeros, which do not change max |y|
+#pragma unroll
+            for (int i = 0; i < 64; ++i) {
+                vmx = max_s16x2(vmx, x[i]);
+                vmn = min_s16x2(vmn, x[i]);
+            }
+        } else {
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
             uint32_t oa[4], ob[4];
@@ -557,10 +587,23 @@ __global__ void __launch_bounds__(kSwarWarps * 32) act_quant_i8_swar_kernel(ActQ
                 *reinterpret_cast<int4 *>(a.y + e0 + 16 * c) = *reinterpret_cast<const int4 *>(buf + swz(c >> 3, c & 7));
         }
         __syncwarp();                                  // every lane has read the stage back
+        }
         issue(t + kSwarStages * nwarps, slot);
         slot = slot + 1 == kSwarStages ? 0 : slot + 1;
     }
     asm volatile("cp.async.wait_group 0;" ::: "memory");
+    if constexpr (MODE == 2) {
+        // max |y| of the lane: low halves carry kBlo (HB >= 2) or 128 (HB = 1), high halves 0 or 128
+        const int blo = HB >= 2 ? (int)kBlo : 128, bhi = HB >= 2 ? 0 : 128;
+        int m = 0;
+        if (vmx != 0x80008000u) {                      // the lane saw at least one tile
+            const int lmx = (int)(int16_t)(vmx & 0xFFFFu) - blo, lmn = (int)(int16_t)(vmn & 0xFFFFu) - blo;
+            const int hmx = ((int)vmx >> 16) - bhi, hmn = ((int)vmn >> 16) - bhi;
+            m = max(max(abs(lmx), abs(lmn)), max(abs(hmx), abs(hmn)));
+        }
+        m = __reduce_max_sync(0xffffffffu, m);
+        if (lane == 0 && m) atomicMax(&a.dyn->maxbits, (unsigned int)m);
+    }
 }
 
 // round(num / den) half to even for num, den > 0.
@@ -581,7 +624,7 @@ __global__ void act_dyn_params_kernel(DynParams *p, int f16, int hb, float s_in,
     const unsigned int mb = p->maxbits;
     const double sq = sqrt((double)hb);
     if (mb == 0) {
-        p->mult = 0; p->shift = 0; p->inv = 0.f;
+        p->mult = 0; p->shift = 0; p->packed = 0;
         if (s_used) *s_used = 1.0f;
         return;
     }
@@ -608,7 +651,28 @@ __global__ void act_dyn_params_kernel(DynParams *p, int f16, int hb, float s_in,
     }
     p->mult = M;
     p->shift = found;
-    p->inv = 0.f;
+    p->packed = 0;
+    // the packed-pair pass (blocks <= 64, 32-bit requantization, codes that step
+    // by at most one): clamp bound vmax = the largest y <= 127 hb whose code is
+    // <= 127, round half to even in full (ties are not excluded here)
+    if (hb <= 64 && found >= 1 && found <= 30 && M >= 1 && M <= (1LL << found)) {
+        auto rne = [&](long long v) { return (v + ((1LL << (found - 1)) - 1) + ((v >> found) & 1)) >> found; };
+        long long lo = 0, hi = 127LL * hb;
+        if (rne(M * hi) > 127) {
+            while (lo < hi) {
+                const long long mid = (lo + hi + 1) / 2;
+                if (rne(M * mid) <= 127) lo = mid;
+                else hi = mid - 1;
+            }
+        }
+        const uint32_t blo = hb >= 2 ? 128u * hb : 128u, bhi = hb >= 2 ? 0u : 128u;
+        const long long clo_lo = -hi + (long long)blo, clo_hi = -hi + (long long)bhi;
+        p->clo = (uint32_t)(clo_lo & 0xFFFF) | ((uint32_t)(clo_hi & 0xFFFF) << 16);
+        const uint32_t half = (1u << (found - 1)) - 1u;
+        p->clow = half - (uint32_t)M * blo;
+        p->chigh = half - (uint32_t)M * bhi;
+        p->packed = 1;
+    }
     if (s_used) *s_used = (float)(((double)s_in * (double)mb) / (sq * 127.0));
 }
 
@@ -656,6 +720,17 @@ long long host_rne(long long p, int n) {
     return (p + ((1LL << (n - 1)) - 1) + ((p >> n) & 1)) >> n;
 }
 
+// One wave of the packed kernel: its resident blocks, at most one warp per 4096-code tile.
+template <typename K>
+int swar_grid(const ActQuantArgs &a, K k) {
+    const long long want = ((a.total + 4095) / 4096 + kSwarWarps - 1) / kSwarWarps;
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kSwarWarps * 32, 0) != cudaSuccess || per_sm < 1)
+        per_sm = 4;
+    const long long cap = (long long)num_sms() * per_sm;
+    return (int)(want < 1 ? 1 : (want < cap ? want : cap));
+}
+
 template <int HB>
 cudaError_t launch_swar(const ActQuantArgs &a, cudaStream_t s) {
     const long long m = a.mult;
@@ -688,20 +763,12 @@ cudaError_t launch_swar(const ActQuantArgs &a, cudaStream_t s) {
     sp.clow = half - (uint32_t)m * blo;
     sp.chigh = half - (uint32_t)m * bhi;
     sp.shift = n;
-    auto grid = [&](auto k) {
-        const long long want = ((a.total + 4095) / 4096 + kSwarWarps - 1) / kSwarWarps;
-        int per_sm = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kSwarWarps * 32, 0) != cudaSuccess || per_sm < 1)
-            per_sm = 4;
-        const long long cap = (long long)num_sms() * per_sm;
-        return (int)(want < cap ? want : cap);
-    };
     if (ties) {
-        auto k = act_quant_i8_swar_kernel<HB, true>;
-        k<<<grid(k), kSwarWarps * 32, 0, s>>>(a, sp);
+        auto k = act_quant_i8_swar_kernel<HB, true, 0>;
+        k<<<swar_grid(a, k), kSwarWarps * 32, 0, s>>>(a, sp);
     } else {
-        auto k = act_quant_i8_swar_kernel<HB, false>;
-        k<<<grid(k), kSwarWarps * 32, 0, s>>>(a, sp);
+        auto k = act_quant_i8_swar_kernel<HB, false, 0>;
+        k<<<swar_grid(a, k), kSwarWarps * 32, 0, s>>>(a, sp);
     }
     return cudaGetLastError();
 }
@@ -750,16 +817,52 @@ cudaError_t launch_act_affine(const AffineQuantArgs &a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+// Packed-pair max-abs pass (mode 2) or quantize pass (mode 1) of the dynamic mode.
+template <int HB>
+cudaError_t launch_swar_dyn(const ActQuantArgs &a, int mode, cudaStream_t s) {
+    SwarParams sp{};
+    if (mode == 2) {
+        auto k = act_quant_i8_swar_kernel<HB, false, 2>;
+        k<<<swar_grid(a, k), kSwarWarps * 32, 0, s>>>(a, sp);
+    } else {
+        auto k = act_quant_i8_swar_kernel<HB, true, 1>;
+        k<<<swar_grid(a, k), kSwarWarps * 32, 0, s>>>(a, sp);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_swar_dyn_hb(const ActQuantArgs &a, int mode, cudaStream_t s) {
+    switch (a.hb) {
+        case 1: return launch_swar_dyn<1>(a, mode, s);
+        case 2: return launch_swar_dyn<2>(a, mode, s);
+        case 4: return launch_swar_dyn<4>(a, mode, s);
+        case 8: return launch_swar_dyn<8>(a, mode, s);
+        case 16: return launch_swar_dyn<16>(a, mode, s);
+        case 32: return launch_swar_dyn<32>(a, mode, s);
+        default: return launch_swar_dyn<64>(a, mode, s);
+    }
+}
+
+// Dynamic scale: max-abs pass, one-thread parameter kernel, quantize pass. The
+// INT8 entry with blocks <= 64 takes the packed-pair kernels; its quantize pass
+// launches the packed kernel and the general one, and the parameter block
+// (written on the device) lets exactly one of them work.
 cudaError_t launch_act_dynamic(const ActQuantArgs &a, float s_in, float *s_used, cudaStream_t s) {
     cudaError_t e = cudaMemsetAsync(a.dyn, 0, sizeof(DynParams), s);
     if (e != cudaSuccess) return e;
+    const bool packed = !a.f16 && a.hb <= 64;
     if (a.f16) act_quant_kernel<true, 2><<<grid_for(a.total, act_quant_kernel<true, 2>), kThreads, 0, s>>>(a);
+    else if (packed) { if ((e = launch_swar_dyn_hb(a, 2, s)) != cudaSuccess) return e; }
     else act_quant_kernel<false, 2><<<grid_for(a.total, act_quant_kernel<false, 2>), kThreads, 0, s>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     act_dyn_params_kernel<<<1, 32, 0, s>>>(a.dyn, a.f16, a.hb, s_in, s_used, a.err);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    if (a.f16) act_quant_kernel<true, 1><<<grid_for(a.total, act_quant_kernel<true, 1>), kThreads, 0, s>>>(a);
-    else act_quant_kernel<false, 1><<<grid_for(a.total, act_quant_kernel<false, 1>), kThreads, 0, s>>>(a);
+    if (a.f16) {
+        act_quant_kernel<true, 1><<<grid_for(a.total, act_quant_kernel<true, 1>), kThreads, 0, s>>>(a);
+        return cudaGetLastError();
+    }
+    if (packed && (e = launch_swar_dyn_hb(a, 1, s)) != cudaSuccess) return e;
+    act_quant_kernel<false, 1><<<grid_for(a.total, act_quant_kernel<false, 1>), kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

@@ -36,10 +36,13 @@ struct DynParams {
     unsigned int maxbits;   // max |H~ x| (integer, or fp32 bits for FP16 entry)
     int shift;
     long long mult;
-    float inv;
-    float pad_;
-    unsigned long long reserved;
+    union {
+        float inv;          // FP16 entry: 127 / max|v|
+        uint32_t packed;    // INT8 entry: 1 when the packed-pair quantize pass applies (M <= 2^n, n <= 30, hb <= 64)
+    };
+    uint32_t clo, clow, chigh;  // the packed-pair pass's constants (lower clamp, low / high requant addends)
 };
+static_assert(sizeof(DynParams) == 32, "the dynamic-mode workspace is 32 bytes");
 
 // Device-side state of the dynamic affine quantizer (Eqs. uniform_q, affine_q;
 // lives in the caller's workspace): order-preserving keys of max v and of

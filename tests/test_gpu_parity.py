@@ -107,6 +107,31 @@ def test_quantize_i8_dynamic(H, hb):
     assert float(host(s_used)[0]) == np.float32(s_ref)
 
 
+@pytest.mark.parametrize("shape,hb", [((2, 37, 41, 192), 64), ((1, 9, 7, 64), 2), ((1, 5, 11, 96), 32),
+                                      ((1, 3, 3, 48), 1), ((1, 4, 4, 64), 8), ((1, 1, 65, 64), 64)])
+def test_quantize_i8_dynamic_packed_pairs(H, shape, hb):
+    """Dynamic scale through the packed-pair max-abs and quantize passes (the
+    parameter block selects the packed pass on the device)."""
+    x = I.activations_i8(shape, seed=500 + hb, s_in=0.05)
+    y, s_used = H.quantize_act(dev(x), H.IN_I8, 0.05, hb, 0.0)
+    H.sync_status()
+    ref, s_ref = O.quantize_act_dynamic_i8(x, hb, 0.05)
+    assert np.array_equal(host(y), ref)
+    assert float(host(s_used)[0]) == np.float32(s_ref)
+    assert (np.abs(ref.astype(int)) == 127).any()
+
+
+def test_quantize_i8_dynamic_general_fallback(H):
+    """Codes in [-1, 1]: max |y| < 127 gives M > 2^n, so the parameter block
+    leaves the quantize pass to the general kernel."""
+    x = np.random.default_rng(6).integers(-1, 2, (1, 7, 9, 64)).astype(np.int8)
+    y, s_used = H.quantize_act(dev(x), H.IN_I8, 0.05, 4, 0.0)
+    H.sync_status()
+    ref, s_ref = O.quantize_act_dynamic_i8(x, 4, 0.05)
+    assert np.array_equal(host(y), ref)
+    assert float(host(s_used)[0]) == np.float32(s_ref)
+
+
 def test_quantize_f16_dynamic(H):
     x = I.activations_f16((1, 16, 16, 128), seed=0)
     y, s_used = H.quantize_act(dev(x), H.IN_F16, 1.0, 128, 0.0)
