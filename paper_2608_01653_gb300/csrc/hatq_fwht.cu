@@ -606,6 +606,118 @@ __global__ void __launch_bounds__(kSwarWarps * 32) act_quant_i8_swar_kernel(ActQ
     }
 }
 
+// FP16 entry, static scale, blocks of at most 64: a lane owns one 64-element
+// block (128 bytes of fp16) of a 2048-element warp tile, staged in through
+// shared memory like the packed INT8 pass (coalesced `cp.async` chunks, rows
+// XOR-swizzled), transformed in fp32 in the lane and quantized as
+// clamp(rint(f inv)); its 64 codes go back through the stage as half of a
+// 128-byte row (chunk positions XOR-swizzled by row, conflict-free for 8
+// lanes) and leave as coalesced 16-byte stores.
+// MODE 0: static scale (a.inv). MODE 1: dynamic scale, inv from the parameter
+// block. MODE 2: the max-abs pass of the dynamic mode (no stores).
+template <int HB, int MODE>
+__global__ void __launch_bounds__(kSwarWarps * 32) act_quant_f16_wide_kernel(ActQuantArgs a) {
+    __shared__ __align__(128) uint8_t stage[kSwarWarps][kSwarStages][4096];
+    float fmx = 0.f;
+    const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
+    const long long warp = (long long)blockIdx.x * kSwarWarps + wib;
+    const long long nwarps = (long long)gridDim.x * kSwarWarps;
+    const long long tiles = (a.total + 2047) >> 11;
+    const uint8_t *xg = static_cast<const uint8_t *>(a.x);
+    const float inv = MODE == 1 ? a.dyn->inv : a.inv;
+    auto issue = [&](long long t, int slot) {
+        if (t < tiles) {
+            const long long e0 = t << 11;              // first element of the tile
+            uint8_t *buf = stage[wib][slot];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                const int c = 32 * i + lane;           // 16-byte chunk = 8 elements
+                const bool ok = e0 + 8 * c < a.total;
+                const uint8_t *src = ok ? xg + 2 * (e0 + 8 * c) : xg;
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(buf + swz(c >> 3, c & 7))),
+                             "l"(src), "r"(ok ? 16 : 0)
+                             : "memory");
+            }
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+#pragma unroll
+    for (int k = 0; k < kSwarStages; ++k) issue(warp + k * nwarps, k);
+    int slot = 0;
+    for (long long t = warp; t < tiles; t += nwarps) {
+        asm volatile("cp.async.wait_group %0;" ::"n"(kSwarStages - 1) : "memory");
+        __syncwarp();
+        uint8_t *buf = stage[wib][slot];
+        float f[64];
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const uint4 r = *reinterpret_cast<const uint4 *>(buf + swz(lane, q));
+            const uint32_t w[4] = {r.x, r.y, r.z, r.w};
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 v = __half22float2(*reinterpret_cast<const __half2 *>(&w[i]));
+                f[8 * q + 2 * i] = v.x;
+                f[8 * q + 2 * i + 1] = v.y;
+            }
+        }
+        __syncwarp();                                  // the stage is free for this tile's codes
+#pragma unroll
+        for (int h = 1; h < HB; h <<= 1) {
+#pragma unroll
+            for (int i = 0; i < 64; ++i) {
+                if (i & h) continue;
+                const float u = f[i], v = f[i + h];
+                f[i] = u + v;
+                f[i + h] = u - v;
+            }
+        }
+        if constexpr (MODE == 2) {
+            // zero-filled elements past the end transform to zeros
+#pragma unroll
+            for (int i = 0; i < 64; ++i) fmx = fmaxf(fmx, fabsf(f[i]));
+            issue(t + kSwarStages * nwarps, slot);
+            slot = slot + 1 == kSwarStages ? 0 : slot + 1;
+            continue;
+        } else {
+        // clamp(rint(f inv)) as in the general kernel: the clamp first, then
+        // 1.5 * 2^23 rounds half to even into the low mantissa byte
+        const int orow = lane >> 1, ocol = 4 * (lane & 1);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            uint32_t o[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                uint32_t c[4];
+#pragma unroll
+                for (int k = 0; k < 4; ++k)
+                    c[k] = __float_as_uint(fminf(fmaxf(f[16 * q + 4 * i + k] * inv, -127.f), 127.f) + 12582912.f);
+                o[i] = pack4p((int)c[0], (int)c[1], (int)c[2], (int)c[3]);
+            }
+            *reinterpret_cast<uint4 *>(buf + orow * 128 + (((ocol + q) ^ (orow & 7)) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+        }
+        __syncwarp();
+        const long long o0 = t << 11;                  // first code of the tile
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int c = 32 * i + lane;
+            const int row = c >> 3;
+            if (o0 + 16 * c < a.total)
+                *reinterpret_cast<uint4 *>(a.y + o0 + 16 * c) =
+                    *reinterpret_cast<const uint4 *>(buf + row * 128 + (((c & 7) ^ (row & 7)) << 4));
+        }
+        __syncwarp();                                  // every lane has read the stage back
+        issue(t + kSwarStages * nwarps, slot);
+        slot = slot + 1 == kSwarStages ? 0 : slot + 1;
+        }
+    }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    if constexpr (MODE == 2) {
+        // nonnegative floats order as their bit patterns
+        const unsigned int m = __reduce_max_sync(0xffffffffu, __float_as_uint(fmx));
+        if (lane == 0 && m) atomicMax(&a.dyn->maxbits, m);
+    }
+}
+
 // round(num / den) half to even for num, den > 0.
 __device__ long long div_rne(unsigned long long num, unsigned long long den) {
     unsigned long long q = num / den, r = num % den;
@@ -773,6 +885,29 @@ cudaError_t launch_swar(const ActQuantArgs &a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+template <int HB, int MODE>
+cudaError_t launch_f16_wide(const ActQuantArgs &a, cudaStream_t s) {
+    auto k = act_quant_f16_wide_kernel<HB, MODE>;
+    // swar_grid counts 4096-element tiles; a tile here is 2048 elements
+    ActQuantArgs g = a;
+    g.total = 2 * a.total;
+    k<<<swar_grid(g, k), kSwarWarps * 32, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+template <int MODE>
+cudaError_t launch_f16_wide_hb(const ActQuantArgs &a, cudaStream_t s) {
+    switch (a.hb) {
+        case 1: return launch_f16_wide<1, MODE>(a, s);
+        case 2: return launch_f16_wide<2, MODE>(a, s);
+        case 4: return launch_f16_wide<4, MODE>(a, s);
+        case 8: return launch_f16_wide<8, MODE>(a, s);
+        case 16: return launch_f16_wide<16, MODE>(a, s);
+        case 32: return launch_f16_wide<32, MODE>(a, s);
+        default: return launch_f16_wide<64, MODE>(a, s);
+    }
+}
+
 cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s) {
     // packed pairs: INT8 entry, blocks of at most 64, 32-bit requantization
     // (1 <= n <= 30) and M <= 2^n (codes step by at most one)
@@ -789,6 +924,7 @@ cudaError_t launch_act_quant(const ActQuantArgs &a, cudaStream_t s) {
         }
     }
     if (a.f16) {
+        if (a.hb <= 64) return launch_f16_wide_hb<0>(a, s);
         act_quant_kernel<true, 0><<<grid_for(a.total, act_quant_kernel<true, 0>), kThreads, 0, s>>>(a);
         return cudaGetLastError();
     }
@@ -851,12 +987,15 @@ cudaError_t launch_act_dynamic(const ActQuantArgs &a, float s_in, float *s_used,
     cudaError_t e = cudaMemsetAsync(a.dyn, 0, sizeof(DynParams), s);
     if (e != cudaSuccess) return e;
     const bool packed = !a.f16 && a.hb <= 64;
-    if (a.f16) act_quant_kernel<true, 2><<<grid_for(a.total, act_quant_kernel<true, 2>), kThreads, 0, s>>>(a);
+    const bool wide16 = a.f16 && a.hb <= 64;
+    if (wide16) { if ((e = launch_f16_wide_hb<2>(a, s)) != cudaSuccess) return e; }
+    else if (a.f16) act_quant_kernel<true, 2><<<grid_for(a.total, act_quant_kernel<true, 2>), kThreads, 0, s>>>(a);
     else if (packed) { if ((e = launch_swar_dyn_hb(a, 2, s)) != cudaSuccess) return e; }
     else act_quant_kernel<false, 2><<<grid_for(a.total, act_quant_kernel<false, 2>), kThreads, 0, s>>>(a);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
     act_dyn_params_kernel<<<1, 32, 0, s>>>(a.dyn, a.f16, a.hb, s_in, s_used, a.err);
     if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (wide16) return launch_f16_wide_hb<1>(a, s);
     if (a.f16) {
         act_quant_kernel<true, 1><<<grid_for(a.total, act_quant_kernel<true, 1>), kThreads, 0, s>>>(a);
         return cudaGetLastError();

@@ -87,7 +87,8 @@ def test_quantize_i8_packed_pairs_bit_exact(H, shape, hb, s_in, rho):
 
 
 @pytest.mark.parametrize("shape,hb", [((1, 16, 16, 128), 128), ((2, 5, 7, 192), 64), ((1, 3, 3, 256), 256),
-                                      ((1, 4, 5, 32), 16)])
+                                      ((1, 4, 5, 32), 16), ((1, 1, 65, 64), 64), ((3, 7, 5, 32), 32),
+                                      ((1, 2, 9, 48), 1), ((2, 9, 11, 64), 2), ((1, 8, 8, 64), 8)])
 def test_quantize_f16_static_within_tolerance(H, shape, hb):
     x = I.activations_f16(shape, seed=200 + hb)
     y_real = O.transform_real(x.astype(np.float64), hb)
@@ -130,6 +131,18 @@ def test_quantize_i8_dynamic_general_fallback(H):
     ref, s_ref = O.quantize_act_dynamic_i8(x, 4, 0.05)
     assert np.array_equal(host(y), ref)
     assert float(host(s_used)[0]) == np.float32(s_ref)
+
+
+@pytest.mark.parametrize("shape,hb", [((2, 5, 7, 192), 64), ((1, 3, 3, 48), 16), ((1, 1, 65, 64), 64), ((1, 6, 7, 64), 1)])
+def test_quantize_f16_dynamic_wide(H, shape, hb):
+    """FP16 entry, dynamic scale, blocks <= 64: the lane-per-block max-abs and
+    quantize passes."""
+    x = I.activations_f16(shape, seed=700 + hb)
+    y, s_used = H.quantize_act(dev(x), H.IN_F16, 1.0, hb, 0.0)
+    H.sync_status()
+    ref, s_ref = O.quantize_act_dynamic_f16(x, hb)
+    assert_codes_close(host(y), ref)
+    assert abs(float(host(s_used)[0]) - s_ref) <= 1e-6 * s_ref
 
 
 def test_quantize_f16_dynamic(H):
