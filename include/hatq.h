@@ -102,8 +102,9 @@ typedef struct {
                              entries (kx, c_in) padded with zero weights to a multiple of 8 */
     float s_x;            /* scale of the INT8 operand this layer consumes */
     float s_y;            /* scale of the INT8 codes it emits */
-    int8_t *w_i8;         /* [c_out][k_pad] weight codes w_int, K order (kh, kw, c_in); c_in padded to a
-                             multiple of 64 per tap (gather == 0) or kw*c_in padded to 8 per row */
+    int8_t *w_i8;         /* [c_out][k_pad] weight codes w_int, K order (kh, kw, c_in); gather == 0: c_in
+                             padded to a multiple of 64 per tap, except c_in % 64 == 32 (taps unpadded,
+                             the total padded to a multiple of 64); gather == 1: kw*c_in padded to 8 per row */
     uint16_t *w_f16;      /* [c_out][k_pad] the same codes as IEEE fp16 (exact), tensor-core operand */
     int32_t *b_int;       /* [c_out] bias codes, Eq. supp_bias_quantization */
     int32_t *mult;        /* [c_out] multipliers M_c, Eq. integer_fixed_point_scale */
@@ -130,8 +131,8 @@ typedef struct {
  * then take the operand straight from the TMA tile in shared memory, with no
  * conversion per output-channel tile. out_f16: the layer writes its codes as
  * fp16 (twice the bytes), the operand format of a next layer with in_f16.
- * Both default to 0. in_f16 needs c_in % 16 == 0 and an INT8 (not affine)
- * layer; out_f16 needs INT8 output (not float32) and is not available to the
+ * Both default to 0. in_f16 needs c_in % 16 == 0, c_in % 64 != 32 and an
+ * INT8 (not affine) layer; out_f16 needs INT8 output (not float32) and is not available to the
  * sub-pixel entry point. Host only; HATQ_ERR_INVALID_ARG / HATQ_ERR_UNSUPPORTED.
  */
 hatq_status hatq_set_operand_format(hatq_prepared *L, int in_f16, int out_f16);

@@ -188,7 +188,7 @@ EncodeTiledFn encode_fn() {
 // ------------------------------------------------------------ geometry
 
 struct Geometry {
-    int gather, cin_pad, seg, k_pad, n_t, G;
+    int gather, half, cin_pad, seg, k_pad, n_t, G;
 };
 
 hatq_status check_desc(const hatq_conv_desc *d) {
@@ -224,13 +224,17 @@ hatq_status check_desc(const hatq_conv_desc *d) {
 
 hatq_status geometry(const hatq_conv_desc *d, int hb_next, Geometry *g) {
     // Packed reduction order. c_in % 16 == 0: (ky, kx, ci) with ci padded to a
-    // multiple of 64 per tap. Otherwise (small c_in): kernel row ky holds the
-    // kw * c_in entries (kx, ci) of one contiguous input-row segment, padded
-    // with zero weights to seg (a multiple of 8), rows back to back.
+    // multiple of 64 per tap, except c_in % 64 == 32, where the taps follow one
+    // another unpadded (a 64-wide block is two 32-channel pieces, possibly of
+    // two taps) and only the total is padded to a multiple of 64. Otherwise
+    // (small c_in): kernel row ky holds the kw * c_in entries (kx, ci) of one
+    // contiguous input-row segment, padded with zero weights to seg (a
+    // multiple of 8), rows back to back.
     g->gather = d->c_in % 16 != 0;
-    g->cin_pad = (d->c_in + 63) / 64 * 64;
+    g->half = !g->gather && d->c_in % 64 == 32;
+    g->cin_pad = g->half ? d->c_in : (d->c_in + 63) / 64 * 64;
     g->seg = (d->kw * d->c_in + 7) / 8 * 8;
-    g->k_pad = g->gather ? (d->kh * g->seg + 63) / 64 * 64 : d->kh * d->kw * g->cin_pad;
+    g->k_pad = g->gather ? (d->kh * g->seg + 63) / 64 * 64 : (d->kh * d->kw * g->cin_pad + 63) / 64 * 64;
     const int hb_out = d->form == HATQ_WH ? d->hb_out : 0;
     int G = 32;
     if (hb_out > G) G = hb_out;
@@ -890,12 +894,15 @@ hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared 
     }
     a.num_kb = g.k_pad / 64;
     a.cin_kb = g.cin_pad / 64;
+    a.half = g.half;
+    a.cin_h = g.cin_pad / 32;
     a.gather = g.gather;
     // exact fp32 chunks: 1024 products of |x| <= 127 (INT8 codes), 512 of |x| <= 255 (centred affine codes)
     a.affine = L->in_affine ? 1 : 0;
     a.a_f16 = L->in_f16 ? 1 : 0;
     a.out_f16 = L->out_f16 ? 1 : 0;
-    if (a.a_f16 && (g.gather || a.affine)) return fail(HATQ_ERR_UNSUPPORTED, "an fp16 operand needs c_in % 16 == 0 and INT8 codes");
+    if (a.a_f16 && (g.gather || g.half || a.affine))
+        return fail(HATQ_ERR_UNSUPPORTED, "an fp16 operand needs c_in %% 64 == 0 or 16 or 48, and INT8 codes");
     if (a.out_f16 && (L->out_f32 || (og && og->d2s)))
         return fail(HATQ_ERR_UNSUPPORTED, "fp16 code output needs INT8 output without the sub-pixel rearrangement");
     a.chunk_kb = a.affine ? 8 : 16;
@@ -992,17 +999,20 @@ hatq_status conv_launch(const void *x, int n, int h, int w, const hatq_prepared 
         EncodeTiledFn enc = encode_fn();
         if (!enc) return fail(HATQ_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
         // INT8 codes (64-byte box rows, 64-byte swizzle), or centred int16 affine codes / fp16
-        // operand codes (128-byte rows, 128-byte swizzle)
+        // operand codes (128-byte rows, 128-byte swizzle); 32-channel boxes take half the row and
+        // the swizzle of that width
         const bool wide = a.affine || a.a_f16;
         const cuuint64_t es = wide ? 2 : 1;
         const cuuint64_t dims[4] = {(cuuint64_t)d->c_in, (cuuint64_t)w, (cuuint64_t)h, (cuuint64_t)n};
         const cuuint64_t strides[3] = {(cuuint64_t)d->c_in * es, (cuuint64_t)w * d->c_in * es,
                                        (cuuint64_t)h * w * d->c_in * es};
-        const cuuint32_t box[4] = {64, (cuuint32_t)(a.tw * d->stride), (cuuint32_t)(a.th * d->stride), 1};
+        // c_in % 64 == 32: 32-channel boxes (32- or 64-byte rows, swizzled to match), two per block
+        const cuuint32_t box[4] = {g.half ? 32u : 64u, (cuuint32_t)(a.tw * d->stride), (cuuint32_t)(a.th * d->stride), 1};
         const cuuint32_t estr[4] = {1, (cuuint32_t)d->stride, (cuuint32_t)d->stride, 1};
         CUresult r = enc(&tmA, wide ? CU_TENSOR_MAP_DATA_TYPE_UINT16 : CU_TENSOR_MAP_DATA_TYPE_UINT8, 4,
                          const_cast<void *>(x), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-                         wide ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+                         g.half ? (wide ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B)
+                                : (wide ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B),
                          CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return fail(HATQ_ERR_CUDA, "activation tensor map encoding failed (%d)", (int)r);
     } else if (a.win_tma) {
@@ -1507,8 +1517,11 @@ hatq_status hatq_set_operand_format(hatq_prepared *L, int in_f16, int out_f16) {
     if (!L) return fail(HATQ_ERR_INVALID_ARG, "null layer");
     if ((in_f16 != 0 && in_f16 != 1) || (out_f16 != 0 && out_f16 != 1))
         return fail(HATQ_ERR_INVALID_ARG, "in_f16 and out_f16 must be 0 or 1");
-    if (in_f16 && (L->gather || L->in_affine || L->d.form == HATQ_TRANSFORM))
-        return fail(HATQ_ERR_UNSUPPORTED, "an fp16 operand needs an INT8 convolution with c_in %% 16 == 0");
+    // the fp16 tile is read by the MMAs in place as whole 64-channel rows, which a layer whose taps
+    // are packed at 32-channel granularity (c_in % 64 == 32) does not have
+    if (in_f16 && (L->gather || L->in_affine || L->d.form == HATQ_TRANSFORM || L->d.c_in % 64 == 32))
+        return fail(HATQ_ERR_UNSUPPORTED, "an fp16 operand needs an INT8 convolution with c_in %% 16 == 0 and "
+                                          "c_in %% 64 != 32");
     if (out_f16 && L->out_f32) return fail(HATQ_ERR_UNSUPPORTED, "fp16 code output needs INT8 output");
     L->in_f16 = in_f16;
     L->out_f16 = out_f16;

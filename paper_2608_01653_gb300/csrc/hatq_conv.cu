@@ -129,30 +129,18 @@ __device__ __forceinline__ void scale_f32(const EpiCtx &e, int col, const int (&
 // thread's row of the shared-memory output tile (copied out coalesced later).
 template <int G>
 __device__ __forceinline__ void store_codes(const ConvArgs &a, uint8_t *row, int col, const long long (&t)[G]) {
-    if (a.shift > 32) {
+    if (a.shift >= 32) {
+        // lower clamp in the round-shift, upper clamp in the saturating pack
         const int sh = a.shift - 32;
-        const int kh = (1 << (sh - 1)) - 1;
+        const long long kadd = (1LL << (a.shift - 1)) - 1;
 #pragma unroll
         for (int i = 0; i < G / 16; ++i) {
             uint32_t w[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const int b = 16 * i + 4 * j;
-                w[j] = pack4(requant8_hi(t[b], sh, kh), requant8_hi(t[b + 1], sh, kh), requant8_hi(t[b + 2], sh, kh),
-                             requant8_hi(t[b + 3], sh, kh));
-            }
-            reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
-        }
-        return;
-    }
-    if (a.shift == 32) {
-#pragma unroll
-        for (int i = 0; i < G / 16; ++i) {
-            uint32_t w[4];
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                const int b = 16 * i + 4 * j;
-                w[j] = pack4(requant8_32(t[b]), requant8_32(t[b + 1]), requant8_32(t[b + 2]), requant8_32(t[b + 3]));
+                w[j] = pack4_sat(requant8_lo(t[b], kadd, sh), requant8_lo(t[b + 1], kadd, sh),
+                                 requant8_lo(t[b + 2], kadd, sh), requant8_lo(t[b + 3], kadd, sh));
             }
             reinterpret_cast<int4 *>(row + col)[i] = make_int4((int)w[0], (int)w[1], (int)w[2], (int)w[3]);
         }
@@ -518,12 +506,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int u = 0; u < SUB; ++u) {
                         if (u >= nsub) break;
                         tma_load_2d(st + a.b_off + u * a.b_bytes, &tmB, full_bar(s), (kb0 + u) * kBlockK, n0);
-                        if (!a.gather) {
+                        if (!a.gather && !a.half) {
                             tma_load_4d(st + a.raw_off + u * a.raw_bytes, &tmA, full_bar(s), cb * kBlockK,
                                         wo0 * a.stride + kx - a.pad_x, ho0 * a.stride + ky - a.pad_y, img);
                             if (++cb == a.cin_kb) {
                                 cb = 0;
                                 if (++kx == a.kw) { kx = 0; ++ky; }
+                            }
+                        } else if (!a.gather) {
+                            // two 32-channel pieces (cb counts pieces); past the last tap the
+                            // weights are zero and the box, in or out of the image, is read as is
+#pragma unroll
+                            for (int hp = 0; hp < 2; ++hp) {
+                                tma_load_4d(st + a.raw_off + u * a.raw_bytes + hp * (a.raw_bytes >> 1), &tmA,
+                                            full_bar(s), cb * 32, wo0 * a.stride + kx - a.pad_x,
+                                            ho0 * a.stride + ky - a.pad_y, img);
+                                if (++cb == a.cin_h) {
+                                    cb = 0;
+                                    if (++kx == a.kw) { kx = 0; ++ky; }
+                                }
                             }
                         }
                     }
@@ -652,11 +653,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             // 64-byte swizzle) -> 32 columns of fp16 pairs
             auto convert_row = [&](const uint8_t *raw, uint32_t (&h)[32]) {
                 if (a.affine) {
-                    // row m of a 64-wide int16 box (128 bytes, 16-byte chunks permuted by the 128-byte swizzle)
-                    const int sw = m & 7;
+                    // row m of a 64-wide int16 box (128 bytes, 16-byte chunks permuted by the 128-byte
+                    // swizzle), or of two 32-wide boxes (64-byte rows, 64-byte swizzle)
+                    const int sw = a.half ? (m >> 1) & 3 : m & 7;
+                    const int hb = a.raw_bytes >> 1;
 #pragma unroll
                     for (int q = 0; q < 8; ++q) {
-                        const uint4 v = *reinterpret_cast<const uint4 *>(raw + ((q ^ sw) << 4));
+                        const int off = a.half ? (q >> 2) * hb + (((q & 3) ^ sw) << 4) : (q ^ sw) << 4;
+                        const uint4 v = *reinterpret_cast<const uint4 *>(raw + off);
                         h[4 * q + 0] = i16x2_to_f16x2(v.x);
                         h[4 * q + 1] = i16x2_to_f16x2(v.y);
                         h[4 * q + 2] = i16x2_to_f16x2(v.z);
@@ -664,10 +668,19 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
                     return;
                 }
-                const int sw = (m >> 1) & 3;
                 uint4 v[4];
+                if (a.half) {
+                    // two 32-wide boxes: 32-byte rows, chunk pairs swapped by the 32-byte swizzle
+                    const int sw = (m >> 2) & 1;
+                    const int hb = a.raw_bytes >> 1;
 #pragma unroll
-                for (int q = 0; q < 4; ++q) v[q] = *reinterpret_cast<const uint4 *>(raw + ((q ^ sw) << 4));
+                    for (int q = 0; q < 4; ++q)
+                        v[q] = *reinterpret_cast<const uint4 *>(raw + (q >> 1) * hb + (((q & 1) ^ sw) << 4));
+                } else {
+                    const int sw = (m >> 1) & 3;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) v[q] = *reinterpret_cast<const uint4 *>(raw + ((q ^ sw) << 4));
+                }
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
                     i8x4_to_f16x4(v[q].x, h[8 * q + 0], h[8 * q + 1]);
@@ -676,7 +689,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                     i8x4_to_f16x4(v[q].w, h[8 * q + 6], h[8 * q + 7]);
                 }
             };
-            const int row_in = (a.affine || a.a_f16) ? 128 : 64;   // bytes of one operand row of a 64-wide block
+            // bytes of one operand row of a 64-wide block (of one of its 32-wide boxes with a.half)
+            const int row_in = ((a.affine || a.a_f16) ? 128 : 64) >> (a.half ? 1 : 0);
             for (int j = 0; j < my_tiles && ok; ++j) {
                 for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB) {
                     const int nsub = min(SUB, a.num_kb - kb0);
@@ -996,7 +1010,8 @@ cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const Co
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
     if (dev < 0 || dev >= kMaxDev) return cudaErrorInvalidDevice;
-    if ((a.sub != 1 && a.sub != 2 && a.sub != 4) || (a.gather && a.sub != 1) || a.chunk_kb % a.sub)
+    if ((a.sub != 1 && a.sub != 2 && a.sub != 4) || (a.gather && a.sub != 1) || a.chunk_kb % a.sub ||
+        (a.half && (a.gather || a.a_f16 || a.cin_h < 1)))
         return cudaErrorInvalidValue;   // gathered tiles: one block per stage
     const int v = a.sub == 4 ? 2 : (a.sub == 2 ? 1 : 0);
     void (*const kern)(const CUtensorMap, const CUtensorMap, const ConvArgs) =

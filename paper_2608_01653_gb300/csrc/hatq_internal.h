@@ -91,6 +91,8 @@ struct ConvArgs {
     int n_t;                         // output channels per tile
     int num_kb;                      // 64-wide reduction blocks
     int cin_kb;                      // reduction blocks per kernel tap (tiled loader)
+    int half;                        // tiled loader, c % 64 == 32: a block is two 32-channel boxes
+    int cin_h;                       // half: 32-channel pieces per kernel tap
     int gather;                      // small-channel loader
     int seg;                         // small-channel loader: reduction entries per kernel row (kw * c, padded to 8)
     int chunk_kb;                    // reduction blocks per exact fp32 chunk

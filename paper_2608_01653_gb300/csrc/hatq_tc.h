@@ -195,6 +195,22 @@ __device__ __forceinline__ int requant8_32(long long v) {
     const int c = (lo > 0x80000000u || (lo == 0x80000000u && (hi & 1))) ? 1 : 0;
     return min(max(hi + c, -127), 127);
 }
+// The same rounding for 32 <= n <= 62 with only the lower clamp (the
+// saturating pack below does the upper one): the 64-bit sum
+// v + (2^(n-1) - 1) + bit_n(v) (kadd = 2^(n-1) - 1, s = n - 32; no overflow for
+// |v| < 2^62) shifted by n is its high word shifted by s.
+__device__ __forceinline__ int requant8_lo(long long v, long long kadd, int s) {
+    const int bit = ((int)((unsigned long long)v >> 32) >> s) & 1;
+    const unsigned long long u = (unsigned long long)(v + kadd) + (unsigned long long)bit;
+    return max((int)(u >> 32) >> s, -127);
+}
+// bytes (q0, q1, q2, q3) of a word, each q saturated to [-128, 127]
+__device__ __forceinline__ uint32_t pack4_sat(int q0, int q1, int q2, int q3) {
+    uint32_t hi, d;
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(hi) : "r"(q3), "r"(q2), "r"(0u));
+    asm("cvt.pack.sat.s8.s32.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(q1), "r"(q0), "r"(hi));
+    return d;
+}
 // requant8 with the 32-bit-piece paths for shifts >= 32 (n is uniform).
 __device__ __forceinline__ int requant8_any(long long v, int n) {
     if (n > 32) return requant8_hi(v, n - 32, (1 << (n - 33)) - 1);

@@ -117,8 +117,10 @@ def test_version_and_last_error(lib):
     (H.make_desc(3, 192, 5, 2, 2, "WH", hb_out=64), 128),       # small-channel packing 5 x 16 -> 128
     (H.make_desc(3, 64, 3, 1, 1, "WH", hb_out=64), 64),         # 3 x 16 -> 64
     (H.make_desc(5, 64, 5, 1, 2, "WH", hb_out=64), 192),        # 5 x 32 -> 192
-    (H.make_desc(32, 224, 3, 1, 1, "DH", hb_in=32), 9 * 64),    # c_in padded to 64 per tap
-    (H.make_desc(224, 128, 3, 1, 1, "WH", hb_out=128), 9 * 256),
+    (H.make_desc(32, 224, 3, 1, 1, "DH", hb_in=32), 320),       # c_in % 64 == 32: taps unpadded, 288 -> 320
+    (H.make_desc(224, 128, 3, 1, 1, "WH", hb_out=128), 9 * 224 + 32),
+    (H.make_desc(96, 64, 1, 1, 0, "DH", hb_in=32), 128),
+    (H.make_desc(48, 64, 3, 1, 1, "DH", hb_in=16), 9 * 64),     # c_in % 64 == 48: padded to 64 per tap
     (H.make_desc(128, 128, 1, 1, 0, "DH", hb_in=128), 128),
 ])
 def test_prepared_sizes(desc, k_pad):
@@ -162,10 +164,10 @@ def _oracle_packed(p, desc, k_pad):
         tmp[:, :, :kw * ci] = p.w_int.reshape(co, kh, kw * ci)
         out[:, :kh * seg] = tmp.reshape(co, -1)
     else:
-        cin_pad = (ci + 63) // 64 * 64
+        cin_pad = ci if ci % 64 == 32 else (ci + 63) // 64 * 64
         tmp = np.zeros((co, kh * kw, cin_pad), np.int8)
         tmp[:, :, :ci] = p.w_int.reshape(co, kh * kw, ci)
-        out[:] = tmp.reshape(co, -1)
+        out[:, :kh * kw * cin_pad] = tmp.reshape(co, -1)
     return out
 
 
@@ -481,5 +483,9 @@ def test_set_operand_format_checks_on_the_host(lib):
     assert lib.hatq_set_operand_format(ctypes.byref(P), 1, 0) == H.ERR_UNSUPPORTED
     P.in_affine, P.out_f32 = 0, 1
     assert lib.hatq_set_operand_format(ctypes.byref(P), 0, 1) == H.ERR_UNSUPPORTED
+    P.out_f32 = 0
+    P.d = H.make_desc(224, 128, 3, 1, 1, "DH", hb_in=32)      # taps packed at 32-channel granularity
+    assert lib.hatq_set_operand_format(ctypes.byref(P), 1, 0) == H.ERR_UNSUPPORTED
+    assert lib.hatq_set_operand_format(ctypes.byref(P), 0, 1) == H.OK
     assert lib.hatq_set_operand_format(None, 0, 0) == H.ERR_INVALID_ARG
 

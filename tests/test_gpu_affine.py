@@ -45,6 +45,7 @@ CASES = [
     ("wh3x3_hb128_relu", C.layer("a", 128, 128, 3, 1, 1, "WH", "relu", hb_out=128), (1, 12, 17), "relu"),
     ("wh1x1_hb64_drain", C.layer("a", 640, 192, 1, 1, 0, "WH", "none", hb_out=64), (1, 9, 7), "signed"),
     ("dh3x3_k2304_drains", C.layer("a", 256, 64, 3, 1, 1, "DH", "relu", hb_in=128), (1, 8, 9), "relu"),
+    ("dh3x3_c96_pieces", C.layer("a", 96, 64, 3, 1, 1, "DH", "relu", hb_in=32), (1, 10, 14), "shifted"),
 ]
 
 

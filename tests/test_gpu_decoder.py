@@ -48,6 +48,7 @@ TRANSPOSED = [
     ("dh3x3s2_p2_negative_offset", C.layer("t", 64, 64, 3, 2, 2, "DH", "none", hb_in=64), (1, 9, 8), 1, 0),
     ("wh5x5s2_c3_gather", C.layer("t", 3, 64, 5, 2, 2, "WH", "relu", hb_out=32), (1, 12, 15), 1, 0),
     ("dh3x3s1_p1", C.layer("t", 64, 96, 3, 1, 1, "DH", "relu", hb_in=32), (2, 6, 7), 0, 32),
+    ("dh5x5s2_c96_pieces", C.layer("t", 96, 64, 5, 2, 2, "DH", "relu", hb_in=32), (1, 8, 9), 1, 0),
 ]
 
 

@@ -35,8 +35,8 @@ CASES = [
     ("dh3x3_drain_next64", C.layer("a", 192, 192, 3, 1, 1, "DH", "relu", hb_in=64), (2, 13, 37), 64),
     ("dh5x5s2_ragged", C.layer("a", 192, 192, 5, 2, 2, "DH", "none", hb_in=64), (3, 19, 45), 0),
     ("wh3x3_c640_128_next128", C.layer("a", 320, 640, 3, 1, 1, "WH", "relu", hb_out=128), (1, 7, 10), 128),
-    ("wh3x3_224_128_next128", C.layer("a", 224, 128, 3, 1, 1, "WH", "relu", hb_out=128), (2, 11, 21), 128),
-    ("dh3x3_c32_box", C.layer("a", 32, 224, 3, 1, 1, "DH", "relu", hb_in=32), (2, 9, 17), 0),
+    ("wh3x3_256_128_next128", C.layer("a", 256, 128, 3, 1, 1, "WH", "relu", hb_out=128), (2, 11, 21), 128),
+    ("dh3x3_c64_box", C.layer("a", 64, 224, 3, 1, 1, "DH", "relu", hb_in=32), (2, 9, 17), 0),
     ("dh1x1_c640_n5", C.layer("a", 640, 640, 1, 1, 0, "DH", "none", hb_in=128), (1, 9, 23), 0),
 ]
 
@@ -89,6 +89,13 @@ def test_f16_operand_rejections(H):
     with pytest.raises(H.HatqError) as e:                    # small-channel (gather) layer
         H.set_operand_format(P, True, False)
     assert e.value.status == H.ERR_UNSUPPORTED
+    for c_in in (32, 224):                                   # taps packed at 32-channel granularity
+        L = C.layer("a", c_in, 64, 3, 1, 1, "DH", "none", hb_in=32)
+        P = H.prepare_weights(H.desc_from_spec(L), I.weights(64, 3, 3, c_in, 1), None, 0.05, 0.05, "none", 0, False)
+        with pytest.raises(H.HatqError) as e:
+            H.set_operand_format(P, True, False)
+        assert e.value.status == H.ERR_UNSUPPORTED
+        H.set_operand_format(P, False, True)                 # the fp16 output format is still open
     L = CASES[0][1]
     P = H.prepare_weights(H.desc_from_spec(L), I.weights(192, 3, 3, 192, 2), None, 0.1, 0.1, "relu", 64, False)
     H.set_operand_format(P, True, False)

@@ -224,6 +224,11 @@ LAYER_CASES = [
     ("wh5x5s2_c3_tma_window", C.layer("a", 3, 192, 5, 2, 2, "WH", "relu", hb_out=64), (2, 41, 64), 64),
     ("wh3x3_c4_tma_window", C.layer("a", 4, 64, 3, 1, 1, "WH", "relu", hb_out=64), (1, 21, 36), 0),
     ("wh7x7_c8_tma_window", C.layer("a", 8, 64, 7, 1, 3, "WH", "none", hb_out=32), (2, 19, 34), 32),
+    # c_in % 64 == 32: taps packed at 32-channel granularity, two 32-channel boxes per 64-wide block
+    # (blocks straddling two taps, a last block half past the last tap, drains)
+    ("dh5x5s2_c160_pieces_drain", C.layer("a", 160, 128, 5, 2, 2, "DH", "relu", hb_in=32), (1, 21, 30), 0),
+    ("dh1x1_c32_pieces", C.layer("a", 32, 64, 1, 1, 0, "DH", "none", hb_in=32), (2, 7, 13), 0),
+    ("wh5x5s2_c32_pieces_next64", C.layer("a", 32, 192, 5, 2, 2, "WH", "relu", hb_out=64), (1, 19, 26), 64),
 ]
 
 
