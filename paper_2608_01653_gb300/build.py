@@ -19,7 +19,8 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libhatq.so")
-SOURCES = ["hatq_api.cu", "hatq_fwht.cu", "hatq_conv.cu", "hatq_gdn.cu", "hatq_noalloc.cu", "hatq_profile.cu"]
+SOURCES = ["hatq_api.cu", "hatq_fwht.cu", "hatq_conv.cu", "hatq_conv_pieces.cu", "hatq_gdn.cu", "hatq_noalloc.cu",
+           "hatq_profile.cu"]
 HEADERS = [os.path.join(CSRC, "hatq_internal.h"), os.path.join(CSRC, "hatq_tc.h"), os.path.join(INCLUDE, "hatq.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

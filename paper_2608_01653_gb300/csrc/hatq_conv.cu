@@ -33,6 +33,14 @@
 // Every mbarrier wait is bounded: on expiry the kernel records an error word,
 // raises a CTA-wide abort flag and unwinds (waiting, again bounded, for its own
 // MMAs and copies) before freeing TMEM.
+// This file is compiled twice: as itself (the kernels for activation blocks of
+// whole 64-channel boxes, the launcher, the self test) and, through
+// hatq_conv_pieces.cu with HATQ_CONV_PIECES = 1, for the kernels whose blocks
+// arrive as two 32-channel boxes; two translation units build in parallel.
+#ifndef HATQ_CONV_PIECES
+#define HATQ_CONV_PIECES 0
+#endif
+
 #include <cuda_fp16.h>
 
 #include "hatq_internal.h"
@@ -364,8 +372,10 @@ __device__ __forceinline__ void epi_split128(const EpiCtx &e, const ConvArgs &a,
 // one chunk per tile epilogue warpgroup w takes the tiles of region w; with
 // several, both warpgroups drain every chunk into int32 register partials
 // (half of the 32-column groups each) and finish the tile together.
-// SUB: 64-wide reduction blocks per pipeline stage (1, 2 or 4)
-template <int SUB>
+// SUB: 64-wide reduction blocks per pipeline stage (1, 2 or 4). PIECES: the
+// activation blocks arrive as two 32-channel boxes (c % 64 == 32); a separate
+// instantiation, so that the other layers' kernels carry none of its code.
+template <int SUB, bool PIECES>
 __global__ void __launch_bounds__(kThreads, 1)
     conv_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                 const __grid_constant__ ConvArgs a) {
@@ -506,14 +516,16 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int u = 0; u < SUB; ++u) {
                         if (u >= nsub) break;
                         tma_load_2d(st + a.b_off + u * a.b_bytes, &tmB, full_bar(s), (kb0 + u) * kBlockK, n0);
-                        if (!a.gather && !a.half) {
-                            tma_load_4d(st + a.raw_off + u * a.raw_bytes, &tmA, full_bar(s), cb * kBlockK,
-                                        wo0 * a.stride + kx - a.pad_x, ho0 * a.stride + ky - a.pad_y, img);
-                            if (++cb == a.cin_kb) {
-                                cb = 0;
-                                if (++kx == a.kw) { kx = 0; ++ky; }
+                        if constexpr (!PIECES) {
+                            if (!a.gather) {
+                                tma_load_4d(st + a.raw_off + u * a.raw_bytes, &tmA, full_bar(s), cb * kBlockK,
+                                            wo0 * a.stride + kx - a.pad_x, ho0 * a.stride + ky - a.pad_y, img);
+                                if (++cb == a.cin_kb) {
+                                    cb = 0;
+                                    if (++kx == a.kw) { kx = 0; ++ky; }
+                                }
                             }
-                        } else if (!a.gather) {
+                        } else {
                             // two 32-channel pieces (cb counts pieces); past the last tap the
                             // weights are zero and the box, in or out of the image, is read as is
 #pragma unroll
@@ -655,11 +667,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (a.affine) {
                     // row m of a 64-wide int16 box (128 bytes, 16-byte chunks permuted by the 128-byte
                     // swizzle), or of two 32-wide boxes (64-byte rows, 64-byte swizzle)
-                    const int sw = a.half ? (m >> 1) & 3 : m & 7;
+                    const int sw = PIECES ? (m >> 1) & 3 : m & 7;
                     const int hb = a.raw_bytes >> 1;
 #pragma unroll
                     for (int q = 0; q < 8; ++q) {
-                        const int off = a.half ? (q >> 2) * hb + (((q & 3) ^ sw) << 4) : (q ^ sw) << 4;
+                        const int off = PIECES ? (q >> 2) * hb + (((q & 3) ^ sw) << 4) : (q ^ sw) << 4;
                         const uint4 v = *reinterpret_cast<const uint4 *>(raw + off);
                         h[4 * q + 0] = i16x2_to_f16x2(v.x);
                         h[4 * q + 1] = i16x2_to_f16x2(v.y);
@@ -669,7 +681,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     return;
                 }
                 uint4 v[4];
-                if (a.half) {
+                if constexpr (PIECES) {
                     // two 32-wide boxes: 32-byte rows, chunk pairs swapped by the 32-byte swizzle
                     const int sw = (m >> 2) & 1;
                     const int hb = a.raw_bytes >> 1;
@@ -690,7 +702,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             };
             // bytes of one operand row of a 64-wide block (of one of its 32-wide boxes with a.half)
-            const int row_in = ((a.affine || a.a_f16) ? 128 : 64) >> (a.half ? 1 : 0);
+            const int row_in = ((a.affine || a.a_f16) ? 128 : 64) >> (PIECES ? 1 : 0);
             for (int j = 0; j < my_tiles && ok; ++j) {
                 for (int kb0 = 0; kb0 < a.num_kb; kb0 += SUB) {
                     const int nsub = min(SUB, a.num_kb - kb0);
@@ -981,6 +993,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
 }
 
+#if !HATQ_CONV_PIECES
 // Failure-detection self test: one thread waits, through the pipeline's
 // bounded wait, on an mbarrier nothing arrives at; the wait expires after
 // `limit` cycles and records kErrWaitTimeout in the error word.
@@ -994,8 +1007,15 @@ __global__ void wait_selftest_kernel(int *err, long long limit) {
     (void)mbar_wait(smem_addr(&bar), 0, &abort_flag, err, limit);
 }
 
+#endif
+
 }  // namespace
 
+#if HATQ_CONV_PIECES
+ConvKernelFn conv_pieces_kernel(int sub) {
+    return sub == 4 ? conv_kernel<4, true> : (sub == 2 ? conv_kernel<2, true> : conv_kernel<1, true>);
+}
+#else
 cudaError_t launch_wait_selftest(int *err, long long limit_cycles, cudaStream_t s) {
     wait_selftest_kernel<<<1, 32, 0, s>>>(err, limit_cycles);
     return cudaGetLastError();
@@ -1004,7 +1024,7 @@ cudaError_t launch_wait_selftest(int *err, long long limit_cycles, cudaStream_t 
 cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const ConvArgs &a, int smem_bytes, cudaStream_t s) {
     // the shared-memory opt-in and the SM count are per device
     constexpr int kMaxDev = 64;
-    static int configured_smem[kMaxDev][3] = {};
+    static int configured_smem[kMaxDev][6] = {};
     static int sms_of[kMaxDev] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -1013,9 +1033,9 @@ cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const Co
     if ((a.sub != 1 && a.sub != 2 && a.sub != 4) || (a.gather && a.sub != 1) || a.chunk_kb % a.sub ||
         (a.half && (a.gather || a.a_f16 || a.cin_h < 1)))
         return cudaErrorInvalidValue;   // gathered tiles: one block per stage
-    const int v = a.sub == 4 ? 2 : (a.sub == 2 ? 1 : 0);
-    void (*const kern)(const CUtensorMap, const CUtensorMap, const ConvArgs) =
-        v == 2 ? conv_kernel<4> : (v == 1 ? conv_kernel<2> : conv_kernel<1>);
+    const int v = (a.sub == 4 ? 2 : (a.sub == 2 ? 1 : 0)) + (a.half ? 3 : 0);
+    const ConvKernelFn kern = a.half ? conv_pieces_kernel(a.sub)
+                                     : (v == 2 ? conv_kernel<4, false> : (v == 1 ? conv_kernel<2, false> : conv_kernel<1, false>));
     if (smem_bytes > configured_smem[dev][v]) {
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
         if (e != cudaSuccess) return e;
@@ -1031,5 +1051,7 @@ cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const Co
     kern<<<grid, kThreads, smem_bytes, s>>>(tmA, tmB, a);
     return cudaGetLastError();
 }
+
+#endif  // HATQ_CONV_PIECES
 
 }  // namespace hatq

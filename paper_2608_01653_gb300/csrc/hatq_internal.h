@@ -134,6 +134,10 @@ struct ConvArgs {
     int8_t lut[256];
 };
 
+// the convolution kernel for layers whose activation blocks arrive as two 32-channel boxes (a.half),
+// with sub 64-wide blocks per pipeline stage (compiled in its own translation unit)
+using ConvKernelFn = void (*)(const CUtensorMap, const CUtensorMap, const ConvArgs);
+ConvKernelFn conv_pieces_kernel(int sub);
 cudaError_t launch_conv(const CUtensorMap &tmA, const CUtensorMap &tmB, const ConvArgs &a,
                         int smem_bytes, cudaStream_t s);
 
