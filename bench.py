@@ -300,7 +300,7 @@ def conv_source_sha() -> str:
     device-helper header it includes), the key of committed counter captures."""
     import hashlib
     h = hashlib.sha256()
-    for f in ("hatq_conv.cu", "hatq_tc.h"):
+    for f in ("hatq_conv.cu", "hatq_conv_pieces.cu", "hatq_tc.h"):
         h.update(open(os.path.join(ROOT, "paper_2608_01653_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
