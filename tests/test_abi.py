@@ -202,6 +202,28 @@ def test_host_prepare_matches_oracle_bit_exact(case):
         assert np.array_equal(got.mult.astype(np.int64), ref.M)
 
 
+@pytest.mark.parametrize("L,hb_next", [
+    (C.layer("p", 32, 192, 5, 2, 2, "WH", "relu", hb_out=64), 64),     # 25 taps of 32: 800 -> 832
+    (C.layer("p", 96, 64, 3, 1, 1, "DH", "none", hb_in=32), 0),        # blocks straddling taps
+    (C.layer("p", 160, 128, 1, 1, 0, "DH", "relu", hb_in=32), 128),    # one tap, 160 -> 192
+    (C.layer("p", 224, 128, 5, 2, 2, "WH", "relu", hb_out=128), 0),    # 5600 -> 5632, drains
+], ids=lambda v: getattr(v, "name", str(v)) if not isinstance(v, int) else str(v))
+def test_host_packing_at_32_channel_granularity(L, hb_next):
+    """c_in % 64 == 32: the taps follow one another unpadded (k = tap c_in + c),
+    the total padded with zero weights to a multiple of 64; codes, bias and
+    (M, n) equal the oracle's."""
+    w, b = I.weights(L.c_out, L.k, L.k, L.c_in, seed=L.c_in), I.bias(L.c_out, seed=L.c_in + 1)
+    desc = H.desc_from_spec(L)
+    got = H.prepare_weights_host(desc, w, b, 0.05, 0.07, L.act, hb_next, False)
+    ref = O.prepare_layer(w, b, L.form, L.hb_in, L.hb_out, 0.05, 0.07, L.act, hb_next, False, L.stride, L.pad)
+    k_real = L.k * L.k * L.c_in
+    assert got.w_i8.shape[1] == (k_real + 63) // 64 * 64
+    assert np.array_equal(got.w_i8[:, :k_real], ref.w_int.reshape(L.c_out, k_real))
+    assert not got.w_i8[:, k_real:].any()
+    assert np.array_equal(got.b_int, ref.b_int) and got.shift == ref.n
+    assert np.array_equal(got.mult.astype(np.int64), ref.M)
+
+
 def test_host_prepare_zero_weights_and_no_bias():
     d = H.make_desc(64, 64, 1, 1, 0, "DH", hb_in=64)
     w = np.zeros((64, 1, 1, 64), np.float32)
